@@ -1,0 +1,159 @@
+"""CPU oracle for the token-selection path (fp64, plain loops, written in C).
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
+benchmark's ``cpu_baseline`` / reference leg may import this package. The CUDA
+product path never does, and this package imports nothing from it.
+
+The arithmetic lives in ``litevlm_oracle.c`` (its header states the definition
+and every reading of the paper it takes). This module only compiles that file
+with gcc and marshals numpy arrays through ctypes.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+from typing import Optional
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "litevlm_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB = os.path.join(_BUILD, "liblitevlm_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+DTYPE_CODES = {"f32": 0, "bf16": 1, "e4m3": 2}
+
+
+def build(src: str = _SRC, out: str = _LIB, extra_flags=()) -> str:
+    """Compile the oracle with gcc (no fused multiply-add contraction)."""
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    tmp = out + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-std=c99", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
+           *extra_flags, "-o", tmp, src, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
+def load(path: Optional[str] = None):
+    """ctypes handle of the oracle library, built on first use."""
+    global _lib
+    if path is not None:
+        return _bind(ctypes.CDLL(path))
+    with _lock:
+        if _lib is None:
+            if (not os.path.exists(_LIB)) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+                build()
+            _lib = _bind(ctypes.CDLL(_LIB))
+    return _lib
+
+
+def _bind(lib):
+    P = ctypes.c_void_p
+    i32, i64, f64, f32 = ctypes.c_int32, ctypes.c_int64, ctypes.c_double, ctypes.c_float
+    lib.litevlm_oracle_decode.argtypes = [i32, P, i64]
+    lib.litevlm_oracle_decode.restype = f64
+    lib.litevlm_oracle_score.argtypes = [i32, P, P, i32, i32, i32, i32, P, P, f64, f64, P, P, P, P]
+    lib.litevlm_oracle_score.restype = ctypes.c_int
+    lib.litevlm_oracle_keep_count.argtypes = [i32, f32]
+    lib.litevlm_oracle_keep_count.restype = i64
+    lib.litevlm_oracle_topk.argtypes = [i32, P, P, P, f32, P, P]
+    lib.litevlm_oracle_topk.restype = ctypes.c_int
+    lib.litevlm_oracle_compact.argtypes = [i64, P, P, P, i64]
+    lib.litevlm_oracle_compact.restype = ctypes.c_int
+    return lib
+
+
+def _ptr(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def decode(dtype: str, raw: np.ndarray, lib=None) -> np.ndarray:
+    """Element-wise decode of f32 / bf16 bits / e4m3 codes to float64."""
+    lib = lib or load()
+    raw = np.ascontiguousarray(raw)
+    flat = raw.reshape(-1)
+    code = DTYPE_CODES[dtype]
+    return np.array([lib.litevlm_oracle_decode(code, _ptr(flat), i) for i in range(flat.size)],
+                    dtype=np.float64).reshape(raw.shape)
+
+
+def score(q: np.ndarray, k: np.ndarray, seq_offsets, text_offsets, hq: int, hkv: int, head_dim: int,
+          dtype: str = "bf16", q_scale: float = 1.0, k_scale: float = 1.0, lib=None, details: bool = False):
+    """Per-visual-token importance scores (fp32), and with details=True also the
+    unrounded fp64 scores, per-(b,h,i) softmax row sums and log-sum-exp values."""
+    lib = lib or load()
+    so = np.ascontiguousarray(seq_offsets, dtype=np.int32)
+    to = np.ascontiguousarray(text_offsets, dtype=np.int32)
+    batch = so.size - 1
+    n_tot, t_tot = int(so[-1]), int(to[-1])
+    q = np.ascontiguousarray(q)
+    k = np.ascontiguousarray(k)
+    out = np.zeros(n_tot, dtype=np.float32)
+    s64 = np.zeros(n_tot, dtype=np.float64) if details else None
+    rows = np.zeros(hq * t_tot, dtype=np.float64) if details else None
+    lse = np.zeros(hq * t_tot, dtype=np.float64) if details else None
+    rc = lib.litevlm_oracle_score(batch, _ptr(so), _ptr(to), hq, hkv, head_dim, DTYPE_CODES[dtype],
+                                  _ptr(q), _ptr(k), float(q_scale), float(k_scale),
+                                  _ptr(out), _ptr(s64), _ptr(rows), _ptr(lse))
+    if rc != 0:
+        raise OracleError(f"litevlm_oracle_score returned {rc}")
+    if details:
+        return out, s64, rows, lse
+    return out
+
+
+def keep_count(n: int, keep_ratio: float, lib=None) -> int:
+    lib = lib or load()
+    return int(lib.litevlm_oracle_keep_count(int(n), float(keep_ratio)))
+
+
+def topk(seq_offsets, scores: np.ndarray, keep_k=None, keep_ratio: float = 0.0, lib=None):
+    """(kept_idx int32 [sum k_b], out_offsets int32 [B+1])."""
+    lib = lib or load()
+    so = np.ascontiguousarray(seq_offsets, dtype=np.int32)
+    batch = so.size - 1
+    scores = np.ascontiguousarray(scores, dtype=np.float32)
+    kk = None if keep_k is None else np.ascontiguousarray(keep_k, dtype=np.int32)
+    if kk is not None:
+        total = int(kk.sum())
+    else:
+        total = sum(keep_count(int(so[b + 1] - so[b]), keep_ratio, lib) for b in range(batch))
+    kept = np.zeros(max(total, 1), dtype=np.int32)
+    out_off = np.zeros(batch + 1, dtype=np.int32)
+    rc = lib.litevlm_oracle_topk(batch, _ptr(so), _ptr(scores), _ptr(kk), float(keep_ratio),
+                                 _ptr(kept), _ptr(out_off))
+    if rc != 0:
+        raise OracleError(f"litevlm_oracle_topk returned {rc}")
+    return kept[:total], out_off
+
+
+def compact(kept_idx: np.ndarray, src: np.ndarray, lib=None) -> np.ndarray:
+    """Rows src[kept_idx] copied byte for byte (src is [rows, ...], any dtype)."""
+    lib = lib or load()
+    src = np.ascontiguousarray(src)
+    kept = np.ascontiguousarray(kept_idx, dtype=np.int32)
+    row_bytes = src.dtype.itemsize * (int(np.prod(src.shape[1:])) if src.ndim > 1 else 1)
+    dst = np.zeros((kept.size,) + src.shape[1:], dtype=src.dtype)
+    rc = lib.litevlm_oracle_compact(kept.size, _ptr(kept), _ptr(src), _ptr(dst), row_bytes)
+    if rc != 0:
+        raise OracleError(f"litevlm_oracle_compact returned {rc}")
+    return dst
+
+
+def select(w_inputs: dict, hq: int, hkv: int, head_dim: int, dtype: str, keep_k=None, keep_ratio=0.0,
+           gather=("hidden",), lib=None):
+    """The whole path on one batch: scores, kept indices, offsets and gathered rows."""
+    s = score(w_inputs["q"], w_inputs["k"], w_inputs["seq_offsets"], w_inputs["text_offsets"], hq, hkv,
+              head_dim, dtype, w_inputs.get("q_scale", 1.0), w_inputs.get("k_scale", 1.0), lib=lib)
+    kept, off = topk(w_inputs["seq_offsets"], s, keep_k=keep_k, keep_ratio=keep_ratio, lib=lib)
+    rows = {name: compact(kept, w_inputs[name], lib=lib) for name in gather}
+    return s, kept, off, rows

@@ -1,0 +1,240 @@
+/*
+ * CPU oracle for LiteVLM's Token Selection Module (arXiv 2506.07416).
+ *
+ * TEST INFRASTRUCTURE ONLY. Only the tests, the package smoke check and the
+ * benchmark's CPU-baseline leg may load this library. It shares no code, header,
+ * table or helper with the CUDA path; its inputs come from the seeded generator
+ * module and from the caller.
+ *
+ * What it computes (Design section, "Token Selection Module"; Related Work,
+ * FastV-style pruning by self-attention scores; Results, "Visual Token
+ * Compression", ratio r):
+ *
+ *   For request b with N_b visual tokens and T_b text tokens, query heads Hq,
+ *   key/value heads Hkv (G = Hq / Hkv), head dimension d:
+ *     s[h][i][j] = (q[i,h,:] . k[j,g(h),:]) * q_scale * k_scale / sqrt(d),
+ *                  g(h) = floor(h / G)
+ *     m[h][i]    = max_j s[h][i][j]
+ *     l[h][i]    = sum_j exp(s[h][i][j] - m[h][i])
+ *     P[h][i][j] = exp(s[h][i][j] - m[h][i]) / l[h][i]
+ *     score[j]   = (sum_h sum_i P[h][i][j]) / (Hq * T_b)      (fp64, rounded once to fp32)
+ *   k_b = keep_k[b] if given, else floor((double)r * N_b) clamped to [0, N_b].
+ *   The kept set is the first k_b tokens under the order (score descending,
+ *   token index ascending); NaN ranks below every number and -0 equals +0.
+ *   kept_idx lists the kept global row indices in ascending order;
+ *   out_offsets[b+1] = out_offsets[b] + k_b.
+ *   Compaction copies each kept row byte for byte.
+ *
+ * Readings where the paper leaves a choice open (each one is a decision of this
+ * oracle, not a statement of the paper):
+ *   R1  queries are all text tokens of the request;
+ *   R2  the softmax normaliser runs over the request's visual tokens only;
+ *   R3  no causal mask is applied (text follows the image, so every text query
+ *       already sees every visual key);
+ *   R4  heads and queries are reduced by their arithmetic mean, so the scores
+ *       of a request sum to 1;
+ *   R5  grouped-query attention maps query head h to key head floor(h / G);
+ *   R6  the logit scale is 1/sqrt(d), times the per-tensor scales for e4m3;
+ *   R7  finetuning changes only the weights that produce q and k, not this formula;
+ *   R8  r is the fraction of visual tokens kept (text tokens are always kept);
+ *   R9  k from r rounds down;
+ *   R10 ties go to the lower token index;
+ *   R11 kept rows stay in their original order;
+ *   R12 NaN scores rank below everything, +inf above;
+ *   R13 N_b = 0 or k_b = 0 give an empty output; N_b > 0 with T_b = 0 is an error.
+ *
+ * Element decoding: bf16 is the top half of an IEEE binary32; e4m3 follows the
+ * OCP 8-bit floating point specification (E4M3, bias 7, no infinities, the
+ * all-ones code is NaN, subnormals m * 2^-9).
+ *
+ * Build: plain C99, -O2 -ffp-contract=off (no fused multiply-add contraction,
+ * so x86 and Arm hosts give the same doubles).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OR_F32 0
+#define OR_BF16 1
+#define OR_E4M3 2
+
+#define OR_OK 0
+#define OR_ERR_ARG -1
+#define OR_ERR_NOMEM -2
+
+double litevlm_oracle_decode(int32_t dtype, const void* base, int64_t index)
+{
+    if (dtype == OR_F32) {
+        float f;
+        memcpy(&f, (const char*)base + 4 * index, 4);
+        return (double)f;
+    }
+    if (dtype == OR_BF16) {
+        uint16_t h;
+        uint32_t u;
+        float f;
+        memcpy(&h, (const char*)base + 2 * index, 2);
+        u = (uint32_t)h << 16;
+        memcpy(&f, &u, 4);
+        return (double)f;
+    }
+    if (dtype == OR_E4M3) {
+        uint8_t c = ((const uint8_t*)base)[index];
+        int sign = c >> 7, e = (c >> 3) & 0xF, m = c & 0x7;
+        double v;
+        if (e == 0xF && m == 0x7) return NAN;
+        if (e == 0) v = ldexp((double)m, -9);          /* m/8 * 2^(1-7)  */
+        else v = ldexp((double)(8 + m), e - 10);       /* (1+m/8) * 2^(e-7) */
+        return sign ? -v : v;
+    }
+    return NAN;
+}
+
+/*
+ * scores      [sum N_b]             fp32 result
+ * scores64    [sum N_b] (nullable)  the same before the final rounding
+ * row_sums    [sum_b Hq*T_b] (nullable)  sum_j P[h][i][j] per (b, h, i), h-major
+ * row_lse     [sum_b Hq*T_b] (nullable)  m + ln(l) per (b, h, i)
+ */
+int litevlm_oracle_score(int32_t batch, const int32_t* seq_offsets, const int32_t* text_offsets,
+                         int32_t hq, int32_t hkv, int32_t head_dim, int32_t dtype,
+                         const void* q, const void* k, double q_scale, double k_scale,
+                         float* scores, double* scores64, double* row_sums, double* row_lse)
+{
+    int64_t row_out = 0;
+    if (batch < 0 || hq <= 0 || hkv <= 0 || head_dim <= 0 || hq % hkv != 0) return OR_ERR_ARG;
+    if (dtype != OR_F32 && dtype != OR_BF16 && dtype != OR_E4M3) return OR_ERR_ARG;
+    for (int32_t b = 0; b < batch; ++b) {
+        if (seq_offsets[b + 1] < seq_offsets[b] || text_offsets[b + 1] < text_offsets[b]) return OR_ERR_ARG;
+        if (seq_offsets[b + 1] > seq_offsets[b] && text_offsets[b + 1] == text_offsets[b]) return OR_ERR_ARG;
+    }
+    const int32_t group = hq / hkv;
+    const double scale = q_scale * k_scale / sqrt((double)head_dim);
+
+    for (int32_t b = 0; b < batch; ++b) {
+        const int64_t n0 = seq_offsets[b], nb = seq_offsets[b + 1] - seq_offsets[b];
+        const int64_t t0 = text_offsets[b], tb = text_offsets[b + 1] - text_offsets[b];
+        if (nb == 0) {
+            /* rows of this request still get their (empty) stats slots */
+            if (row_sums) for (int64_t r = 0; r < (int64_t)hq * tb; ++r) row_sums[row_out + r] = 0.0;
+            if (row_lse) for (int64_t r = 0; r < (int64_t)hq * tb; ++r) row_lse[row_out + r] = -INFINITY;
+            row_out += (int64_t)hq * tb;
+            continue;
+        }
+        double* acc = (double*)calloc((size_t)nb, sizeof(double));
+        double* s = (double*)malloc((size_t)nb * sizeof(double));
+        if (!acc || !s) { free(acc); free(s); return OR_ERR_NOMEM; }
+
+        for (int32_t h = 0; h < hq; ++h) {
+            const int32_t g = h / group;
+            for (int64_t i = 0; i < tb; ++i) {
+                const int64_t qrow = ((t0 + i) * hq + h) * head_dim;
+                double m = -INFINITY, l = 0.0, psum = 0.0;
+                for (int64_t j = 0; j < nb; ++j) {
+                    const int64_t krow = ((n0 + j) * hkv + g) * head_dim;
+                    double dot = 0.0;
+                    for (int32_t c = 0; c < head_dim; ++c)
+                        dot += litevlm_oracle_decode(dtype, q, qrow + c) * litevlm_oracle_decode(dtype, k, krow + c);
+                    s[j] = dot * scale;
+                    if (s[j] > m) m = s[j];
+                }
+                for (int64_t j = 0; j < nb; ++j) l += exp(s[j] - m);
+                for (int64_t j = 0; j < nb; ++j) {
+                    const double p = exp(s[j] - m) / l;
+                    acc[j] += p;
+                    psum += p;
+                }
+                if (row_sums) row_sums[row_out] = psum;
+                if (row_lse) row_lse[row_out] = m + log(l);
+                ++row_out;
+            }
+        }
+        const double denom = (double)hq * (double)tb;
+        for (int64_t j = 0; j < nb; ++j) {
+            const double v = acc[j] / denom;
+            scores[n0 + j] = (float)v;
+            if (scores64) scores64[n0 + j] = v;
+        }
+        free(acc);
+        free(s);
+    }
+    return OR_OK;
+}
+
+typedef struct {
+    float key;
+    int32_t idx;
+} oracle_item;
+
+/* score descending, index ascending; NaN after every number; -0 == +0 */
+static int oracle_rank_cmp(const void* pa, const void* pb)
+{
+    const oracle_item* a = (const oracle_item*)pa;
+    const oracle_item* b = (const oracle_item*)pb;
+    const int an = isnan(a->key) != 0, bn = isnan(b->key) != 0;
+    if (an != bn) return an ? 1 : -1;
+    if (!an && a->key != b->key) return a->key > b->key ? -1 : 1;
+    return (a->idx > b->idx) - (a->idx < b->idx);
+}
+
+static int oracle_index_cmp(const void* pa, const void* pb)
+{
+    const oracle_item* a = (const oracle_item*)pa;
+    const oracle_item* b = (const oracle_item*)pb;
+    return (a->idx > b->idx) - (a->idx < b->idx);
+}
+
+int64_t litevlm_oracle_keep_count(int32_t n, float keep_ratio)
+{
+    double kd = floor((double)keep_ratio * (double)n);
+    if (kd < 0) kd = 0;
+    if (kd > n) kd = n;
+    return (int64_t)kd;
+}
+
+/*
+ * keep_k may be NULL: then k_b = floor((double)keep_ratio * N_b) clamped to [0, N_b].
+ * kept_idx receives sum_b k_b global indices; out_offsets has batch+1 entries.
+ */
+int litevlm_oracle_topk(int32_t batch, const int32_t* seq_offsets, const float* scores,
+                        const int32_t* keep_k, float keep_ratio,
+                        int32_t* kept_idx, int32_t* out_offsets)
+{
+    int64_t out = 0;
+    if (batch < 0) return OR_ERR_ARG;
+    if (!keep_k && !(keep_ratio >= 0.0f && keep_ratio <= 1.0f)) return OR_ERR_ARG;
+    out_offsets[0] = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int64_t n0 = seq_offsets[b], nb = seq_offsets[b + 1] - seq_offsets[b];
+        int64_t kb;
+        if (nb < 0) return OR_ERR_ARG;
+        kb = keep_k ? keep_k[b] : litevlm_oracle_keep_count((int32_t)nb, keep_ratio);
+        if (kb < 0 || kb > nb) return OR_ERR_ARG;
+        if (kb > 0) {
+            oracle_item* it = (oracle_item*)malloc((size_t)nb * sizeof(oracle_item));
+            if (!it) return OR_ERR_NOMEM;
+            for (int64_t j = 0; j < nb; ++j) {
+                it[j].key = scores[n0 + j];
+                it[j].idx = (int32_t)j;
+            }
+            qsort(it, (size_t)nb, sizeof(oracle_item), oracle_rank_cmp);
+            qsort(it, (size_t)kb, sizeof(oracle_item), oracle_index_cmp);
+            for (int64_t r = 0; r < kb; ++r) kept_idx[out + r] = (int32_t)(n0 + it[r].idx);
+            free(it);
+        }
+        out += kb;
+        out_offsets[b + 1] = (int32_t)out;
+    }
+    return OR_OK;
+}
+
+/* dst[r] = src[kept_idx[r]] for rows of row_bytes bytes */
+int litevlm_oracle_compact(int64_t total_kept, const int32_t* kept_idx,
+                           const void* src, void* dst, int64_t row_bytes)
+{
+    if (total_kept < 0 || row_bytes < 0) return OR_ERR_ARG;
+    for (int64_t r = 0; r < total_kept; ++r)
+        memcpy((char*)dst + r * row_bytes, (const char*)src + (int64_t)kept_idx[r] * row_bytes, (size_t)row_bytes);
+    return OR_OK;
+}

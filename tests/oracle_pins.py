@@ -1,0 +1,278 @@
+"""Pins of the CPU oracle to facts that do not come from the oracle itself.
+
+Each ``pin_*`` function takes a loaded oracle library and raises AssertionError
+when the oracle disagrees with the fact it checks. ``test_oracle_pins.py`` runs
+them on the real oracle; ``test_oracle_mutations.py`` runs them on copies of the
+oracle with a planted mistake and expects at least one to fail for every mistake.
+
+Sources of truth used here (none of them is the oracle's own formula):
+  * a hand-worked example (2 heads, 4 visual tokens) with closed-form scores;
+  * closed forms: identical keys give uniform scores 1/N;
+  * a special case that is a library routine: one head and one query give
+    scipy.special.softmax of the scaled logits;
+  * invariants: softmax rows sum to 1, a request's scores sum to 1, permuting
+    visual tokens permutes the scores, replicating grouped K heads (GQA -> MHA)
+    leaves the scores unchanged, salient keys aligned with the queries rank first;
+  * brute force: top-k against Python's sorted() on small inputs with ties, -0, NaN;
+  * the paper's Table 1 token counts (ratio meaning and rounding);
+  * torch's own bf16 and float8_e4m3fn decoders;
+  * numpy fancy indexing for the gather.
+"""
+from __future__ import annotations
+
+import json
+import math
+import os
+
+import numpy as np
+
+import oracle
+from paper_2506_07416_gb300 import inputs
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _bf16(x) -> np.ndarray:
+    return inputs.f32_to_bf16_bits(np.asarray(x, dtype=np.float32))
+
+
+def _bf16_value(bits: np.ndarray) -> np.ndarray:
+    return inputs.bf16_bits_to_f32(bits).astype(np.float64)
+
+
+# ---------------------------------------------------------------------------
+# element decoders
+# ---------------------------------------------------------------------------
+
+def pin_bf16_decode(lib):
+    import torch
+    codes = np.arange(0, 1 << 16, 97, dtype=np.uint16)  # strided sweep over every exponent
+    codes = np.concatenate([codes, np.array([0x0000, 0x8000, 0x3F80, 0xBF80, 0x7F80, 0xFF80, 0x0001, 0x7F7F],
+                                            dtype=np.uint16)])
+    got = oracle.decode("bf16", codes, lib=lib)
+    ref = torch.from_numpy(codes.view(np.int16).copy()).view(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(got, ref)
+
+
+def pin_e4m3_decode(lib):
+    import torch
+    codes = np.arange(256, dtype=np.uint8)
+    got = oracle.decode("e4m3", codes, lib=lib)
+    ref = torch.from_numpy(codes.copy()).view(torch.float8_e4m3fn).to(torch.float64).numpy()
+    np.testing.assert_array_equal(got, ref)
+    assert got[0x7E] == 448.0 and got[0x01] == 2.0 ** -9 and np.isnan(got[0x7F])
+
+
+# ---------------------------------------------------------------------------
+# scores
+# ---------------------------------------------------------------------------
+
+def worked_example():
+    """2 query/key heads, d = 4 (logit scale 1/2), 2 text and 4 visual tokens.
+
+    Head 0: q0 = [2,0,0,0], q1 = [0,2,0,0]; k0 = [1,0,0,0], k1 = [0,1,0,0],
+    k2 = k3 = 0, so the logit rows are [1,0,0,0] and [0,1,0,0].
+    Head 1: both queries are zero, so every softmax entry is 1/4 whatever the keys.
+    score0 = score1 = (e/(e+3) + 1/(e+3) + 1/2) / 4 and score2 = score3 = (2/(e+3) + 1/2) / 4.
+    """
+    q = np.zeros((2, 2, 4), np.float32)
+    q[0, 0, 0] = 2.0
+    q[1, 0, 1] = 2.0
+    k = np.zeros((4, 2, 4), np.float32)
+    k[0, 0, 0] = 1.0
+    k[1, 0, 1] = 1.0
+    k[:, 1, :] = np.array([[0.5, -1.0, 2.0, 0.25], [3.0, 0.0, -0.5, 1.0],
+                           [-2.0, 1.5, 0.75, 0.0], [1.0, 1.0, 1.0, -1.0]], np.float32)
+    e = math.e
+    hi = (e / (e + 3) + 1 / (e + 3) + 0.5) / 4
+    lo = (2 / (e + 3) + 0.5) / 4
+    return q, k, np.array([hi, hi, lo, lo])
+
+
+def pin_worked_example(lib):
+    q, k, expect = worked_example()
+    so, to = np.array([0, 4], np.int32), np.array([0, 2], np.int32)
+    # the same example with the two heads swapped must give the same scores
+    qs, ks = q[:, ::-1, :].copy(), k[:, ::-1, :].copy()
+    for dtype, qq, kk in (("f32", q, k), ("bf16", _bf16(q), _bf16(k)), ("f32", qs, ks)):
+        s, s64, rows, _ = oracle.score(qq, kk, so, to, 2, 2, 4, dtype, lib=lib, details=True)
+        np.testing.assert_allclose(s64, expect, rtol=1e-14, atol=0)
+        np.testing.assert_array_equal(s, expect.astype(np.float32))
+        np.testing.assert_allclose(rows, 1.0, rtol=0, atol=1e-14)
+        assert abs(s64.sum() - 1.0) < 1e-14
+        kept, off = oracle.topk(so, s, keep_k=[1], lib=lib)
+        assert kept.tolist() == [0] and off.tolist() == [0, 1]
+        kept, off = oracle.topk(so, s, keep_k=[3], lib=lib)
+        assert kept.tolist() == [0, 1, 2] and off.tolist() == [0, 3]
+
+
+def pin_uniform_keys(lib):
+    """Identical key rows: every logit of a row is equal, so every score is 1/N
+    and the top-k is the first k indices (the tie-break)."""
+    rng = np.random.Generator(np.random.PCG64(11))
+    n, t, hq, hkv, d = 37, 5, 6, 3, 8
+    q = rng.standard_normal((t, hq, d)).astype(np.float32)
+    k = np.broadcast_to(rng.standard_normal((1, hkv, d)).astype(np.float32), (n, hkv, d)).copy()
+    so, to = np.array([0, n], np.int32), np.array([0, t], np.int32)
+    s, s64, _, _ = oracle.score(q, k, so, to, hq, hkv, d, "f32", lib=lib, details=True)
+    np.testing.assert_allclose(s64, 1.0 / n, rtol=1e-13)
+    assert np.all(s == s[0])
+    kept, _ = oracle.topk(so, s, keep_k=[9], lib=lib)
+    assert kept.tolist() == list(range(9))
+
+
+def pin_single_query_is_softmax(lib):
+    """One head and one query: the score vector is softmax(q.K^T / sqrt(d))."""
+    from scipy.special import softmax
+    rng = np.random.Generator(np.random.PCG64(12))
+    n, d = 50, 16
+    q = _bf16(rng.standard_normal((1, 1, d)) * 0.7)
+    k = _bf16(rng.standard_normal((n, 1, d)) * 0.7)
+    so, to = np.array([0, n], np.int32), np.array([0, 1], np.int32)
+    _, s64, _, lse = oracle.score(q, k, so, to, 1, 1, d, "bf16", lib=lib, details=True)
+    logits = _bf16_value(k)[:, 0, :] @ _bf16_value(q)[0, 0, :] / math.sqrt(d)
+    np.testing.assert_allclose(s64, softmax(logits), rtol=1e-12, atol=0)
+    from scipy.special import logsumexp
+    np.testing.assert_allclose(lse, [logsumexp(logits)], rtol=1e-13)
+
+
+def _ragged(seed, hq, hkv, d, n_vis, n_txt, sigma=0.6):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    q = rng.standard_normal((sum(n_txt), hq, d)).astype(np.float32) * sigma
+    k = rng.standard_normal((sum(n_vis), hkv, d)).astype(np.float32) * sigma
+    so = np.concatenate([[0], np.cumsum(n_vis)]).astype(np.int32)
+    to = np.concatenate([[0], np.cumsum(n_txt)]).astype(np.int32)
+    return q, k, so, to
+
+
+def pin_row_and_total_sums(lib):
+    q, k, so, to = _ragged(13, 4, 2, 16, [20, 0, 33, 7], [3, 2, 5, 1])
+    _, s64, rows, _ = oracle.score(q, k, so, to, 4, 2, 16, "f32", lib=lib, details=True)
+    row_req = np.repeat(np.arange(4), 4 * np.diff(to))
+    np.testing.assert_allclose(rows[row_req != 1], 1.0, rtol=0, atol=1e-13)
+    for b in range(4):
+        if so[b + 1] > so[b]:
+            assert abs(s64[so[b]:so[b + 1]].sum() - 1.0) < 1e-13
+
+
+def pin_permutation_equivariance(lib):
+    q, k, so, to = _ragged(14, 4, 4, 16, [41], [6])
+    perm = np.random.Generator(np.random.PCG64(15)).permutation(41)
+    _, a, _, _ = oracle.score(q, k, so, to, 4, 4, 16, "f32", lib=lib, details=True)
+    _, b, _, _ = oracle.score(q, k[perm], so, to, 4, 4, 16, "f32", lib=lib, details=True)
+    np.testing.assert_allclose(b, a[perm], rtol=1e-12)
+
+
+def pin_gqa_replication(lib):
+    """Query head h reads key head floor(h / G): replicating each key head G
+    times in order (GQA -> MHA) must not change the scores."""
+    hq, hkv, d = 6, 2, 16
+    q, k, so, to = _ragged(16, hq, hkv, d, [29, 18], [4, 3])
+    _, a, _, _ = oracle.score(q, k, so, to, hq, hkv, d, "f32", lib=lib, details=True)
+    k_rep = np.repeat(k, hq // hkv, axis=1)
+    _, b, _, _ = oracle.score(q, k_rep, so, to, hq, hq, d, "f32", lib=lib, details=True)
+    np.testing.assert_allclose(a, b, rtol=1e-12)
+
+
+def pin_scale_placement(lib):
+    """The per-tensor scales multiply the logits: (2q, k) with scales 1 equals
+    (q, k) with q_scale 2, and likewise for k (powers of two are exact)."""
+    q, k, so, to = _ragged(17, 2, 2, 8, [23], [3])
+    _, a, _, _ = oracle.score(2 * q, k, so, to, 2, 2, 8, "f32", lib=lib, details=True)
+    _, b, _, _ = oracle.score(q, k, so, to, 2, 2, 8, "f32", q_scale=2.0, lib=lib, details=True)
+    _, c, _, _ = oracle.score(q, 2 * k, so, to, 2, 2, 8, "f32", lib=lib, details=True)
+    _, e, _, _ = oracle.score(q, k, so, to, 2, 2, 8, "f32", k_scale=2.0, lib=lib, details=True)
+    np.testing.assert_allclose(b, a, rtol=1e-13)
+    np.testing.assert_allclose(e, c, rtol=1e-13)
+    np.testing.assert_allclose(a, c, rtol=1e-13)
+
+
+def pin_e4m3_scores(lib):
+    """e4m3 codes with scales score like the decoded values in f32 (e4m3 values
+    and power-of-two scales are exact in f32)."""
+    import torch
+    q, k, so, to = _ragged(18, 2, 1, 16, [31], [4], sigma=2.0)
+    q8 = torch.from_numpy(q).to(torch.float8_e4m3fn)
+    k8 = torch.from_numpy(k).to(torch.float8_e4m3fn)
+    qv, kv = q8.to(torch.float32).numpy(), k8.to(torch.float32).numpy()
+    _, a, _, _ = oracle.score(q8.view(torch.uint8).numpy(), k8.view(torch.uint8).numpy(), so, to, 2, 1, 16,
+                              "e4m3", q_scale=0.5, k_scale=0.25, lib=lib, details=True)
+    _, b, _, _ = oracle.score(qv * 0.5, kv * 0.25, so, to, 2, 1, 16, "f32", lib=lib, details=True)
+    np.testing.assert_allclose(a, b, rtol=1e-13)
+
+
+def pin_salient_tokens_rank_first(lib):
+    """Keys aligned with the mean query direction get the largest logits, so
+    the tiny workload's 8 salient tokens are the top 8 (sign of the logit)."""
+    w = inputs.workload("tiny")
+    x = inputs.make_numpy(w)
+    s = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, "bf16", lib=lib)
+    pos = x["salient"][0]
+    top = np.sort(np.argsort(-s.astype(np.float64), kind="stable")[:w.salient_count])
+    assert top.tolist() == pos.tolist()
+
+
+# ---------------------------------------------------------------------------
+# top-k
+# ---------------------------------------------------------------------------
+
+def brute_topk(scores: np.ndarray, k: int):
+    def key(j):
+        v = float(scores[j])
+        return (1, 0.0, j) if math.isnan(v) else (0, -v, j)
+    return sorted(sorted(range(len(scores)), key=key)[:k])
+
+
+def pin_topk_bruteforce(lib):
+    rng = np.random.Generator(np.random.PCG64(19))
+    specials = np.array([0.0, -0.0, np.nan, np.inf, -np.inf, 1e-38, -1e-38], np.float32)
+    for trial in range(300):
+        n = int(rng.integers(1, 65))
+        pool = rng.choice(rng.standard_normal(max(1, n // 3)).astype(np.float32), size=n)
+        m = rng.random(n) < 0.2
+        pool[m] = rng.choice(specials, size=int(m.sum()))
+        k = int(rng.integers(0, n + 1))
+        so = np.array([0, n], np.int32)
+        kept, off = oracle.topk(so, pool, keep_k=[k], lib=lib)
+        assert kept.tolist() == brute_topk(pool, k), (trial, pool.tolist(), k)
+        assert off.tolist() == [0, k]
+
+
+def pin_topk_batch_and_ratio(lib):
+    rng = np.random.Generator(np.random.PCG64(20))
+    n_vis = [10, 0, 25, 1, 64]
+    so = np.concatenate([[0], np.cumsum(n_vis)]).astype(np.int32)
+    s = np.round(rng.standard_normal(so[-1]), 1).astype(np.float32)  # many ties
+    for r in (0.0, 0.1, 0.3, 0.5, 0.999, 1.0):
+        kept, off = oracle.topk(so, s, keep_ratio=r, lib=lib)
+        ks = [int(math.floor(float(np.float32(r)) * n)) for n in n_vis]
+        assert np.diff(off).tolist() == ks
+        exp = []
+        for b in range(len(n_vis)):
+            exp += [so[b] + j for j in brute_topk(s[so[b]:so[b + 1]], ks[b])]
+        assert kept.tolist() == exp
+
+
+def pin_table1_token_counts(lib):
+    """Table 1: r is the kept fraction of visual tokens and k rounds down."""
+    with open(os.path.join(GOLDEN, "table1_token_counts.json")) as f:
+        g = json.load(f)
+    for row in g["rows"]:
+        n = int(round(row["tiles"] * g["visual_tokens_per_tile"]))
+        kept = oracle.keep_count(n, row["r"], lib=lib)
+        assert kept + g["text_tokens"] == row["input_tokens"], row
+
+
+def pin_compact(lib):
+    rng = np.random.Generator(np.random.PCG64(21))
+    src = rng.integers(0, 256, size=(40, 24), dtype=np.uint8)
+    idx = np.sort(rng.choice(40, size=17, replace=False)).astype(np.int32)
+    np.testing.assert_array_equal(oracle.compact(idx, src, lib=lib), src[idx])
+    hid = _bf16(rng.standard_normal((40, 8)))
+    np.testing.assert_array_equal(oracle.compact(idx, hid, lib=lib), hid[idx])
+
+
+ALL_PINS = [pin_bf16_decode, pin_e4m3_decode, pin_worked_example, pin_uniform_keys, pin_single_query_is_softmax,
+            pin_row_and_total_sums, pin_permutation_equivariance, pin_gqa_replication, pin_scale_placement,
+            pin_e4m3_scores, pin_salient_tokens_rank_first, pin_topk_bruteforce, pin_topk_batch_and_ratio,
+            pin_table1_token_counts, pin_compact]

@@ -1,0 +1,56 @@
+"""Pin strength: plant one plausible mistake at a time into a copy of the
+oracle's C source, compile it on the CPU, and require that the pin suite
+rejects every mutant. The real oracle is never modified."""
+import os
+import shutil
+
+import pytest
+
+import oracle
+import oracle_pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "litevlm_oracle.c")
+
+# (name, original text, planted text)
+MUTANTS = [
+    ("gqa_head_map_modulo", "const int32_t g = h / group;", "const int32_t g = h % hkv;"),
+    ("key_head_always_zero", "const int64_t krow = ((n0 + j) * hkv + g) * head_dim;",
+     "const int64_t krow = ((n0 + j) * hkv + 0) * head_dim;"),
+    ("scale_1_over_d", "/ sqrt((double)head_dim)", "/ (double)head_dim"),
+    ("logit_sign", "s[j] = dot * scale;", "s[j] = -dot * scale;"),
+    ("no_mean_over_queries", "const double denom = (double)hq * (double)tb;", "const double denom = (double)hq;"),
+    ("softmax_unnormalised", "const double p = exp(s[j] - m) / l;", "const double p = exp(s[j] - m);"),
+    ("normaliser_without_max", "for (int64_t j = 0; j < nb; ++j) l += exp(s[j] - m);",
+     "for (int64_t j = 0; j < nb; ++j) l += exp(s[j]);"),
+    ("ascending_scores", "return a->key > b->key ? -1 : 1;", "return a->key > b->key ? 1 : -1;"),
+    ("tie_to_higher_index",
+     "return a->key > b->key ? -1 : 1;\n    return (a->idx > b->idx) - (a->idx < b->idx);",
+     "return a->key > b->key ? -1 : 1;\n    return (a->idx < b->idx) - (a->idx > b->idx);"),
+    ("nan_ranks_first", "if (an != bn) return an ? 1 : -1;", "if (an != bn) return an ? -1 : 1;"),
+    ("ratio_rounds_to_nearest", "double kd = floor((double)keep_ratio * (double)n);",
+     "double kd = floor((double)keep_ratio * (double)n + 0.5);"),
+    ("kept_in_rank_order", "qsort(it, (size_t)kb, sizeof(oracle_item), oracle_index_cmp);", ""),
+    ("e4m3_exponent_bias", "else v = ldexp((double)(8 + m), e - 10);", "else v = ldexp((double)(8 + m), e - 9);"),
+    ("e4m3_subnormal_scale", "if (e == 0) v = ldexp((double)m, -9);", "if (e == 0) v = ldexp((double)m, -10);"),
+    ("bf16_shift", "u = (uint32_t)h << 16;", "u = (uint32_t)h << 15;"),
+    ("gather_wrong_row", "(const char*)src + (int64_t)kept_idx[r] * row_bytes",
+     "(const char*)src + (int64_t)r * row_bytes"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_reject_mutant(tmp_path, name, old, new):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation site for {name} not found exactly once"
+    mut = tmp_path / "mutant.c"
+    mut.write_text(src.replace(old, new))
+    so = oracle.build(str(mut), str(tmp_path / "libmutant.so"))
+    lib = oracle.load(so)
+    caught = []
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(lib)
+        except (AssertionError, oracle.OracleError) as e:
+            caught.append(pin.__name__)
+            break
+    assert caught, f"no pin rejects the planted mistake {name}"
