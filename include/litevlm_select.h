@@ -1,0 +1,180 @@
+/*
+ * litevlm_select.h -- C-ABI of the GB300 (sm_103a) token-selection library.
+ *
+ * The library implements the Token Selection Module of LiteVLM (arXiv
+ * 2506.07416, Design section, "Token Selection Module"): before the LLM prefill,
+ * every visual token is scored by the softmax attention it receives from the
+ * request's text tokens in the first decoder layer (FastV-style attention-score
+ * pruning, Related Work), the top-k tokens of each request are kept (ratio r,
+ * Results section, "Visual Token Compression"; Table 1 token counts), and the
+ * kept hidden / K / V rows are gathered, in their original order, into a
+ * shorter ragged sequence for the prefill.
+ *
+ * Score definition (for request b with N_b visual and T_b text tokens, Hq query
+ * heads, Hkv key heads, G = Hq / Hkv, head dimension d):
+ *     s[h][i][j] = q_scale * k_scale * (q[i,h,:] . k[j, h / G, :]) / sqrt(d)
+ *     score[j]   = (1 / (Hq * T_b)) * sum_h sum_i softmax_j(s[h][i][:])[j]
+ * The softmax runs over the request's visual tokens only; every text token of
+ * the request is a query; no causal mask (text follows the image).
+ * Top-k order: score descending, then token index ascending (the lower index
+ * wins a tie); NaN ranks below every number, -0 equals +0.
+ * k_b = keep_k[b], or floor((double)keep_ratio * N_b) when no keep_k is given.
+ *
+ * Conventions for every call:
+ *   - Pointers named *_d and all tensor pointers are DEVICE pointers; *_h are
+ *     HOST pointers. The caller owns all of them; the library keeps none after
+ *     the call returns.
+ *   - Layouts are row-major and contiguous:
+ *       q        [sum_b T_b, Hq,  d]   bf16, or e4m3 codes (uint8)
+ *       k        [sum_b N_b, Hkv, d]   same element type as q
+ *       offsets  int32 [batch + 1], offsets[0] = 0, non-decreasing
+ *   - Work is enqueued on `stream` (a cudaStream_t) and runs asynchronously;
+ *     a call returns after enqueueing. Host-side validation happens before any
+ *     work is enqueued; on error nothing is enqueued.
+ *   - The *_h offset arrays must hold the same values as their *_d mirrors;
+ *     they are read on the host for validation and sizing only. Mirrors that
+ *     disagree are undefined behaviour.
+ *   - Every function returns a status and never aborts the process. The text
+ *     of the last error of a handle is available from litevlm_select_last_error.
+ *   - A handle is used by one host thread and one stream at a time.
+ *   - Hot calls (score, topk, compact) allocate nothing; the workspace is
+ *     allocated once by create and freed by destroy.
+ */
+#ifndef LITEVLM_SELECT_H
+#define LITEVLM_SELECT_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* litevlm_stream_t;
+
+typedef enum {
+    LITEVLM_OK = 0,
+    LITEVLM_ERR_INVALID_ARG = 1,  /* bad pointer, size, offsets, k, ratio or scale */
+    LITEVLM_ERR_UNSUPPORTED = 2,  /* valid but outside what the kernels implement */
+    LITEVLM_ERR_WORKSPACE = 3,    /* batch or totals beyond the maxima given to create */
+    LITEVLM_ERR_CUDA = 4,         /* a CUDA runtime/driver call failed */
+    LITEVLM_ERR_TIMEOUT = 5,      /* a device-side bounded wait gave up (from check_device) */
+    LITEVLM_ERR_DEVICE_BOUNDS = 6 /* a kernel found an index outside its buffer and skipped it */
+} litevlm_status_t;
+
+typedef enum {
+    LITEVLM_BF16 = 0,     /* q and k are bfloat16 */
+    LITEVLM_FP8_E4M3 = 1  /* q and k are OCP e4m3 codes with one float scale per tensor */
+} litevlm_dtype_t;
+
+typedef struct {
+    int32_t max_batch;         /* largest batch any call will pass */
+    int64_t max_total_visual;  /* largest sum_b N_b */
+    int64_t max_total_text;    /* largest sum_b T_b */
+    int32_t num_q_heads;       /* Hq */
+    int32_t num_kv_heads;      /* Hkv, Hq % Hkv == 0 */
+    int32_t head_dim;          /* d: 64 or 128 for bf16, 128 for e4m3 */
+    litevlm_dtype_t qk_dtype;
+    int32_t flags;             /* reserved, must be 0 */
+} litevlm_select_config_t;
+
+typedef struct litevlm_select* litevlm_select_t;
+
+/*
+ * Creates a handle on the current CUDA device and allocates its workspace
+ * (partial-score buffer, error word). Limits: T_b <= 128 text tokens per request,
+ * N_b <= 65536 visual tokens per request (both checked per call).
+ * Errors: INVALID_ARG for a NULL pointer or an inconsistent config (non-positive
+ * sizes, Hq % Hkv != 0, flags != 0); UNSUPPORTED for a head_dim / dtype pair
+ * without a kernel; CUDA when the device cannot be used. *out is NULL on error.
+ */
+litevlm_status_t litevlm_select_create(const litevlm_select_config_t* config, litevlm_select_t* out);
+
+/* Frees the workspace and the handle. NULL is accepted. Not stream-ordered:
+ * the caller makes sure no work using the handle is still running. */
+litevlm_status_t litevlm_select_destroy(litevlm_select_t handle);
+
+/* Message of the last failed call on this handle ("" if none). Owned by the
+ * handle, valid until the next call on it. NULL handle: message of the last
+ * failed create in this thread. */
+const char* litevlm_select_last_error(litevlm_select_t handle);
+
+/* Static description of a status code. */
+const char* litevlm_status_string(litevlm_status_t status);
+
+/*
+ * Visual-token importance scores (steps: logits, per-row softmax statistics,
+ * head/query reduction; Design section, Token Selection Module).
+ *   batch            number of requests, 0 <= batch <= max_batch
+ *   q_text           device, [sum T_b, Hq, d] text-query rows
+ *   text_offsets_d/h int32 [batch+1] prefix of T_b
+ *   k_vis            device, [sum N_b, Hkv, d] visual key rows
+ *   seq_offsets_d/h  int32 [batch+1] prefix of N_b
+ *   q_scale, k_scale per-tensor dequantisation scales for e4m3 (> 0, finite);
+ *                    must be 1 for bf16
+ *   scores           device, float [sum N_b], written for every visual token
+ * Requirements: T_b >= 1 whenever N_b >= 1; T_b <= 128; N_b <= 65536;
+ * q_text and k_vis 16-byte aligned. The score matrix is never written to memory;
+ * a request with N_b = 0 writes nothing.
+ */
+litevlm_status_t litevlm_select_score(litevlm_select_t handle, int32_t batch,
+                                      const void* q_text, const int32_t* text_offsets_d,
+                                      const int32_t* text_offsets_h,
+                                      const void* k_vis, const int32_t* seq_offsets_d,
+                                      const int32_t* seq_offsets_h,
+                                      float q_scale, float k_scale, float* scores,
+                                      litevlm_stream_t stream);
+
+/*
+ * Per-request top-k (Results section, ratio r of visual tokens kept; Table 1).
+ *   scores           device, float [sum N_b]
+ *   keep_k_d/h       int32 [batch] tokens to keep per request, 0 <= k_b <= N_b;
+ *                    both NULL selects keep_ratio (then k_b = floor((double)keep_ratio * N_b));
+ *                    when keep_k_d is given keep_k_h must be given too
+ *   keep_ratio       0 <= r <= 1, used only when keep_k is NULL
+ *   kept_idx         device, int32 [sum k_b]: global row indices (into the
+ *                    sum N_b rows), ascending within each request
+ *   out_offsets_d    device, int32 [batch+1] prefix of k_b
+ *   out_offsets_h    optional host int32 [batch+1]; filled synchronously from
+ *                    the host mirrors before the call returns (sizes the gather)
+ * Ties are broken by the lower token index; the result is unique.
+ */
+litevlm_status_t litevlm_select_topk(litevlm_select_t handle, int32_t batch, const float* scores,
+                                     const int32_t* seq_offsets_d, const int32_t* seq_offsets_h,
+                                     const int32_t* keep_k_d, const int32_t* keep_k_h, float keep_ratio,
+                                     int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
+                                     litevlm_stream_t stream);
+
+/*
+ * Gather of the kept rows into the compacted sequence (the LLM prefill input;
+ * Design section: the module shortens the LLM input sequence; Speculative
+ * Decoding Head: K/V rows feed the KV cache).
+ *   kept_idx     device, int32 [total_kept], each in [0, src_rows)
+ *   total_kept   rows to copy (out_offsets_h[batch] from topk)
+ *   src_rows     rows of every source tensor (sum N_b)
+ *   num_tensors  1..8 tensors gathered with the same index list
+ *   src, dst     HOST arrays of num_tensors DEVICE pointers; src[t] is
+ *                [src_rows, row_bytes[t]], dst[t] is [total_kept, row_bytes[t]]
+ *   row_bytes    HOST array of num_tensors row sizes in bytes (> 0)
+ * dst[t][r] = src[t][kept_idx[r]] byte for byte. Rows whose size and pointers are
+ * 16-byte aligned move with 128-bit loads and stores; others byte by byte.
+ * An index outside [0, src_rows) is skipped on the device and reported by
+ * litevlm_select_check_device as LITEVLM_ERR_DEVICE_BOUNDS.
+ */
+litevlm_status_t litevlm_select_compact(litevlm_select_t handle, int64_t total_kept, const int32_t* kept_idx,
+                                        int64_t src_rows, int32_t num_tensors,
+                                        const void* const* src, void* const* dst, const int64_t* row_bytes,
+                                        litevlm_stream_t stream);
+
+/*
+ * Synchronises `stream`, then reads and clears the handle's device error word.
+ * Returns OK, TIMEOUT (a kernel's bounded wait gave up; its outputs are not
+ * valid), DEVICE_BOUNDS, or CUDA.
+ */
+litevlm_status_t litevlm_select_check_device(litevlm_select_t handle, litevlm_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LITEVLM_SELECT_H */

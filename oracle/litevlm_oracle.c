@@ -124,18 +124,22 @@ int litevlm_oracle_score(int32_t batch, const int32_t* seq_offsets, const int32_
         }
         double* acc = (double*)calloc((size_t)nb, sizeof(double));
         double* s = (double*)malloc((size_t)nb * sizeof(double));
-        if (!acc || !s) { free(acc); free(s); return OR_ERR_NOMEM; }
+        /* step 1: decode this request's q and k rows exactly into doubles */
+        double* qd = (double*)malloc((size_t)(tb * hq * head_dim) * sizeof(double));
+        double* kd = (double*)malloc((size_t)(nb * hkv * head_dim) * sizeof(double));
+        if (!acc || !s || !qd || !kd) { free(acc); free(s); free(qd); free(kd); return OR_ERR_NOMEM; }
+        for (int64_t x = 0; x < tb * hq * head_dim; ++x) qd[x] = litevlm_oracle_decode(dtype, q, t0 * hq * head_dim + x);
+        for (int64_t x = 0; x < nb * hkv * head_dim; ++x) kd[x] = litevlm_oracle_decode(dtype, k, n0 * hkv * head_dim + x);
 
         for (int32_t h = 0; h < hq; ++h) {
             const int32_t g = h / group;
             for (int64_t i = 0; i < tb; ++i) {
-                const int64_t qrow = ((t0 + i) * hq + h) * head_dim;
+                const int64_t qrow = (i * hq + h) * head_dim;
                 double m = -INFINITY, l = 0.0, psum = 0.0;
                 for (int64_t j = 0; j < nb; ++j) {
-                    const int64_t krow = ((n0 + j) * hkv + g) * head_dim;
+                    const int64_t krow = (j * hkv + g) * head_dim;
                     double dot = 0.0;
-                    for (int32_t c = 0; c < head_dim; ++c)
-                        dot += litevlm_oracle_decode(dtype, q, qrow + c) * litevlm_oracle_decode(dtype, k, krow + c);
+                    for (int32_t c = 0; c < head_dim; ++c) dot += qd[qrow + c] * kd[krow + c];
                     s[j] = dot * scale;
                     if (s[j] > m) m = s[j];
                 }
@@ -158,6 +162,8 @@ int litevlm_oracle_score(int32_t batch, const int32_t* seq_offsets, const int32_
         }
         free(acc);
         free(s);
+        free(qd);
+        free(kd);
     }
     return OR_OK;
 }

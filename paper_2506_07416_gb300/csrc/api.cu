@@ -1,0 +1,343 @@
+// C-ABI of the token-selection library: handle and workspace management,
+// host-side validation from the host offset mirrors, TMA descriptor encoding
+// and the kernel launches. See include/litevlm_select.h for the contract.
+
+#include <cudaTypedefs.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <cstdio>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/litevlm_select.h"
+#include "internal.h"
+
+struct litevlm_select {
+    litevlm_select_config_t cfg;
+    int device = 0;
+    int num_sms = 0;
+    float* partials = nullptr;  // [Hq][max_total_visual]: per-head-group partial scores
+    int32_t* err_d = nullptr;   // device error word (bits lvs::kErr*)
+    PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    std::string last_error;
+};
+
+namespace {
+
+thread_local std::string g_create_error;
+
+litevlm_status_t fail(litevlm_select_t h, litevlm_status_t s, const std::string& msg)
+{
+    if (h) h->last_error = msg;
+    else g_create_error = msg;
+    return s;
+}
+
+litevlm_status_t cuda_fail(litevlm_select_t h, cudaError_t e, const char* where)
+{
+    return fail(h, LITEVLM_ERR_CUDA, std::string(where) + ": " + cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Checks an offsets mirror: offs[0] = 0, non-decreasing, total within `max_total`.
+litevlm_status_t check_offsets(litevlm_select_t h, const int32_t* offs, int32_t batch, int64_t max_total,
+                               const char* name, int64_t* total)
+{
+    if (!offs) return fail(h, LITEVLM_ERR_INVALID_ARG, std::string(name) + " host mirror is NULL");
+    if (offs[0] != 0) return fail(h, LITEVLM_ERR_INVALID_ARG, std::string(name) + "[0] must be 0");
+    for (int32_t b = 0; b < batch; ++b)
+        if (offs[b + 1] < offs[b])
+            return fail(h, LITEVLM_ERR_INVALID_ARG, std::string(name) + " must be non-decreasing (request " +
+                                                        std::to_string(b) + ")");
+    *total = offs[batch];
+    if (*total > max_total)
+        return fail(h, LITEVLM_ERR_WORKSPACE, std::string(name) + " total " + std::to_string(*total) +
+                                                  " exceeds the handle maximum " + std::to_string(max_total));
+    return LITEVLM_OK;
+}
+
+int64_t keep_count_host(int32_t n, float ratio)
+{
+    double kd = floor((double)ratio * (double)n);
+    if (kd < 0) kd = 0;
+    if (kd > n) kd = n;
+    return (int64_t)kd;
+}
+
+litevlm_status_t encode_rows_map(litevlm_select_t h, CUtensorMap* map, const void* base, int32_t head_dim,
+                                 int32_t heads, int64_t rows, bool fp8, const char* what)
+{
+    const int esize = fp8 ? 1 : 2;
+    const cuuint64_t dims[3] = {(cuuint64_t)head_dim, (cuuint64_t)heads, (cuuint64_t)rows};
+    const cuuint64_t strides[2] = {(cuuint64_t)head_dim * esize, (cuuint64_t)heads * head_dim * esize};
+    const cuuint32_t box[3] = {(cuuint32_t)(128 / esize), 1u, 128u};
+    const cuuint32_t estride[3] = {1u, 1u, 1u};
+    const CUresult r = h->encode(map, fp8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                                 const_cast<void*>(base), dims, strides, box, estride,
+                                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(h, LITEVLM_ERR_CUDA, std::string("cuTensorMapEncodeTiled failed for ") + what + " (" +
+                                             std::to_string((int)r) + ")");
+    return LITEVLM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* litevlm_status_string(litevlm_status_t s)
+{
+    switch (s) {
+    case LITEVLM_OK: return "ok";
+    case LITEVLM_ERR_INVALID_ARG: return "invalid argument";
+    case LITEVLM_ERR_UNSUPPORTED: return "unsupported shape or type";
+    case LITEVLM_ERR_WORKSPACE: return "beyond the handle's configured maxima";
+    case LITEVLM_ERR_CUDA: return "CUDA error";
+    case LITEVLM_ERR_TIMEOUT: return "device-side wait timed out";
+    case LITEVLM_ERR_DEVICE_BOUNDS: return "device-side index out of bounds";
+    }
+    return "unknown status";
+}
+
+const char* litevlm_select_last_error(litevlm_select_t h)
+{
+    return h ? h->last_error.c_str() : g_create_error.c_str();
+}
+
+litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm_select_t* out)
+{
+    g_create_error.clear();
+    if (!out) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (!c) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "config is NULL");
+    if (c->max_batch <= 0 || c->max_total_visual <= 0 || c->max_total_text <= 0)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "max_batch, max_total_visual, max_total_text must be > 0");
+    if (c->max_total_visual > INT32_MAX || c->max_total_text > INT32_MAX)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "totals must fit in int32 row indices");
+    if (c->num_q_heads <= 0 || c->num_kv_heads <= 0 || c->num_q_heads % c->num_kv_heads != 0)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
+    if (c->qk_dtype != LITEVLM_BF16 && c->qk_dtype != LITEVLM_FP8_E4M3)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "qk_dtype must be LITEVLM_BF16 or LITEVLM_FP8_E4M3");
+    if (c->flags != 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "flags must be 0");
+    if (c->head_dim <= 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "head_dim must be > 0");
+    if (!lvs::score_shape_supported(c->head_dim, c->qk_dtype == LITEVLM_FP8_E4M3))
+        return fail(nullptr, LITEVLM_ERR_UNSUPPORTED,
+                    "head_dim " + std::to_string(c->head_dim) + " has no kernel for this dtype (bf16: 64, 128; e4m3: 128)");
+
+    litevlm_select* h = new (std::nothrow) litevlm_select();
+    if (!h) return fail(nullptr, LITEVLM_ERR_CUDA, "out of host memory");
+    h->cfg = *c;
+    cudaError_t e = cudaGetDevice(&h->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+    if (e == cudaSuccess) {
+        int major = 0, minor = 0;
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, h->device);
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, h->device);
+        if (major != 10) {
+            delete h;
+            return fail(nullptr, LITEVLM_ERR_UNSUPPORTED,
+                        "needs a Blackwell (sm_10x) GPU, found sm_" + std::to_string(major) + std::to_string(minor));
+        }
+    }
+    if (e == cudaSuccess) {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e == cudaSuccess && (q != cudaDriverEntryPointSuccess || !fn)) e = cudaErrorNotSupported;
+        h->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    if (e == cudaSuccess) e = cudaMalloc(&h->err_d, sizeof(int32_t));
+    if (e == cudaSuccess) e = cudaMemset(h->err_d, 0, sizeof(int32_t));
+    if (e == cudaSuccess && c->num_q_heads > 1)
+        e = cudaMalloc(&h->partials, sizeof(float) * (size_t)c->num_q_heads * (size_t)c->max_total_visual);
+    if (e != cudaSuccess) {
+        const std::string msg = std::string("create: ") + cudaGetErrorString(e);
+        if (h->err_d) cudaFree(h->err_d);
+        if (h->partials) cudaFree(h->partials);
+        delete h;
+        cudaGetLastError();
+        return fail(nullptr, LITEVLM_ERR_CUDA, msg);
+    }
+    *out = h;
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_destroy(litevlm_select_t h)
+{
+    if (!h) return LITEVLM_OK;
+    if (h->partials) cudaFree(h->partials);
+    if (h->err_d) cudaFree(h->err_d);
+    delete h;
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const void* q_text,
+                                      const int32_t* text_offsets_d, const int32_t* text_offsets_h,
+                                      const void* k_vis, const int32_t* seq_offsets_d,
+                                      const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
+                                      litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    const litevlm_select_config_t& c = h->cfg;
+    const bool fp8 = c.qk_dtype == LITEVLM_FP8_E4M3;
+    if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
+    if (batch > c.max_batch) return fail(h, LITEVLM_ERR_WORKSPACE, "batch exceeds max_batch");
+    if (batch == 0) return LITEVLM_OK;
+    int64_t tot_n = 0, tot_t = 0;
+    litevlm_status_t s = check_offsets(h, seq_offsets_h, batch, c.max_total_visual, "seq_offsets", &tot_n);
+    if (s != LITEVLM_OK) return s;
+    s = check_offsets(h, text_offsets_h, batch, c.max_total_text, "text_offsets", &tot_t);
+    if (s != LITEVLM_OK) return s;
+    int max_tiles = 0, max_n = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int32_t n = seq_offsets_h[b + 1] - seq_offsets_h[b];
+        const int32_t t = text_offsets_h[b + 1] - text_offsets_h[b];
+        if (n > 0 && t == 0)
+            return fail(h, LITEVLM_ERR_INVALID_ARG,
+                        "request " + std::to_string(b) + " has visual tokens but no text query token");
+        if (t > lvs::kMaxText)
+            return fail(h, LITEVLM_ERR_UNSUPPORTED, "request " + std::to_string(b) + " has " + std::to_string(t) +
+                                                        " text tokens; the score kernel handles at most 128");
+        if (n > 65536)
+            return fail(h, LITEVLM_ERR_UNSUPPORTED,
+                        "request " + std::to_string(b) + " has more than 65536 visual tokens");
+        const int tiles = (n + lvs::kTileRows - 1) / lvs::kTileRows;
+        if (tiles > max_tiles) max_tiles = tiles;
+        if (n > max_n) max_n = n;
+    }
+    if (tot_n == 0) return LITEVLM_OK;
+    if (!q_text || !k_vis || !scores || !text_offsets_d || !seq_offsets_d)
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
+    if (!aligned16(q_text) || !aligned16(k_vis))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "q_text and k_vis must be 16-byte aligned");
+    if (fp8) {
+        if (!(q_scale > 0.f) || !(k_scale > 0.f) || isinf(q_scale) || isinf(k_scale))
+            return fail(h, LITEVLM_ERR_INVALID_ARG, "e4m3 scales must be finite and > 0");
+    } else if (q_scale != 1.f || k_scale != 1.f) {
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "q_scale and k_scale must be 1 for bf16 inputs");
+    }
+    const lvs::ScorePlan plan = lvs::plan_score(batch, max_tiles, c.num_q_heads, h->num_sms);
+    if (plan.tiles_per_cta > lvs::kMaxTilesPerCta)
+        return fail(h, LITEVLM_ERR_UNSUPPORTED, "request too long for one cluster");
+
+    CUtensorMap tm_q, tm_k;
+    s = encode_rows_map(h, &tm_q, q_text, c.head_dim, c.num_q_heads, tot_t, fp8, "q_text");
+    if (s != LITEVLM_OK) return s;
+    s = encode_rows_map(h, &tm_k, k_vis, c.head_dim, c.num_kv_heads, tot_n, fp8, "k_vis");
+    if (s != LITEVLM_OK) return s;
+
+    lvs::ScoreLaunch p{};
+    p.seq_off = seq_offsets_d;
+    p.text_off = text_offsets_d;
+    p.err = h->err_d;
+    p.total_vis = tot_n;
+    p.hq = c.num_q_heads;
+    p.hkv = c.num_kv_heads;
+    p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
+    p.wait_budget = lvs::kWaitBudgetCycles;
+    const int row_bytes = c.head_dim * (fp8 ? 1 : 2);
+    const cudaError_t e = lvs::launch_score(tm_q, tm_k, p, plan, batch, row_bytes, fp8, h->partials, scores, max_n,
+                                            (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "score launch");
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const float* scores,
+                                     const int32_t* seq_offsets_d, const int32_t* seq_offsets_h,
+                                     const int32_t* keep_k_d, const int32_t* keep_k_h, float keep_ratio,
+                                     int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
+                                     litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
+    if (batch > h->cfg.max_batch) return fail(h, LITEVLM_ERR_WORKSPACE, "batch exceeds max_batch");
+    if ((keep_k_d == nullptr) != (keep_k_h == nullptr))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "keep_k_d and keep_k_h must be both given or both NULL");
+    if (!keep_k_h && !(keep_ratio >= 0.f && keep_ratio <= 1.f))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "keep_ratio must be in [0, 1]");
+    if (batch == 0) {
+        if (out_offsets_h) out_offsets_h[0] = 0;
+        return LITEVLM_OK;
+    }
+    int64_t tot_n = 0;
+    litevlm_status_t s = check_offsets(h, seq_offsets_h, batch, h->cfg.max_total_visual, "seq_offsets", &tot_n);
+    if (s != LITEVLM_OK) return s;
+    int64_t total_k = 0;
+    int max_n = 0;
+    std::vector<int32_t> off((size_t)batch + 1, 0);
+    for (int32_t b = 0; b < batch; ++b) {
+        const int32_t n = seq_offsets_h[b + 1] - seq_offsets_h[b];
+        if (n > max_n) max_n = n;
+        int64_t k;
+        if (keep_k_h) {
+            k = keep_k_h[b];
+            if (k < 0 || k > n)
+                return fail(h, LITEVLM_ERR_INVALID_ARG, "keep_k[" + std::to_string(b) + "] = " + std::to_string(k) +
+                                                            " outside [0, " + std::to_string(n) + "]");
+        } else {
+            k = keep_count_host(n, keep_ratio);
+        }
+        total_k += k;
+        off[(size_t)b + 1] = (int32_t)total_k;
+    }
+    if (!out_offsets_d || !seq_offsets_d) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
+    if (total_k > 0 && (!kept_idx || !scores)) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
+    if (out_offsets_h)
+        for (int32_t b = 0; b <= batch; ++b) out_offsets_h[b] = off[(size_t)b];
+    const cudaError_t e = lvs::launch_topk(batch, scores, seq_offsets_d, keep_k_d, keep_ratio, kept_idx,
+                                           out_offsets_d, max_n, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "topk launch");
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_compact(litevlm_select_t h, int64_t total_kept, const int32_t* kept_idx,
+                                        int64_t src_rows, int32_t num_tensors, const void* const* src,
+                                        void* const* dst, const int64_t* row_bytes, litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (total_kept < 0 || src_rows < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "sizes must be >= 0");
+    if (num_tensors < 1 || num_tensors > lvs::kMaxGatherTensors)
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "num_tensors must be in [1, 8]");
+    if (!src || !dst || !row_bytes) return fail(h, LITEVLM_ERR_INVALID_ARG, "src, dst and row_bytes are required");
+    lvs::GatherArgs g{};
+    g.n = num_tensors;
+    bool vec16 = true;
+    for (int t = 0; t < num_tensors; ++t) {
+        if (row_bytes[t] <= 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "row_bytes must be > 0");
+        if (total_kept > 0 && (!src[t] || !dst[t]))
+            return fail(h, LITEVLM_ERR_INVALID_ARG, "tensor " + std::to_string(t) + " pointer is NULL");
+        g.src[t] = static_cast<const uint8_t*>(src[t]);
+        g.dst[t] = static_cast<uint8_t*>(dst[t]);
+        g.row_bytes[t] = row_bytes[t];
+        vec16 = vec16 && (row_bytes[t] % 16 == 0) && aligned16(src[t]) && aligned16(dst[t]);
+    }
+    if (total_kept == 0) return LITEVLM_OK;
+    if (!kept_idx) return fail(h, LITEVLM_ERR_INVALID_ARG, "kept_idx is NULL");
+    const cudaError_t e =
+        lvs::launch_compact(total_kept, kept_idx, src_rows, g, vec16, h->err_d, h->num_sms, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "compact launch");
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    int32_t word = 0;
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e == cudaSuccess) e = cudaMemcpy(&word, h->err_d, sizeof(word), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && word) e = cudaMemset(h->err_d, 0, sizeof(int32_t));
+    if (e != cudaSuccess) return cuda_fail(h, e, "check_device");
+    if (word & lvs::kErrTimeout) return fail(h, LITEVLM_ERR_TIMEOUT, "a device-side wait timed out");
+    if (word & lvs::kErrBounds) return fail(h, LITEVLM_ERR_DEVICE_BOUNDS, "a gather index was out of bounds");
+    if (word & lvs::kErrShape) return fail(h, LITEVLM_ERR_UNSUPPORTED, "a request shape reached the kernel unchecked");
+    return LITEVLM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,209 @@
+// Per-request top-k of the visual-token scores (Results section, "Visual Token
+// Compression": a ratio r of the visual tokens is kept; Table 1 token counts).
+//
+// One CTA per request. Scores become order-preserving 32-bit keys (NaN -> 0,
+// the lowest key; -0 and +0 the same key), an MSB-first radix select (4 passes
+// of 8 bits, warp-aggregated shared-memory histograms) finds the k-th largest
+// key K* and how many keys equal to K* must be taken, then one pass over the
+// tokens in index order keeps every key > K* and the first keys == K* (lower
+// index wins a tie). Two block-wide exclusive scans give each thread its place
+// in the output, so the kept indices come out ascending, as global rows.
+// k_b = keep_k[b], or floor((double)ratio * N_b) clamped to [0, N_b];
+// out_offsets[b+1] = sum of k over requests 0..b.
+
+#include <math.h>
+
+#include "internal.h"
+
+namespace lvs {
+
+namespace {
+
+constexpr int kTopkThreads = 512;
+constexpr int kTopkWarps = kTopkThreads / 32;
+
+__device__ __forceinline__ uint32_t order_key(float f)
+{
+    uint32_t u = __float_as_uint(f);
+    if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0u;  // NaN ranks below everything
+    if (u == 0x80000000u) u = 0u;                     // -0 equals +0
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ int keep_count(const int32_t* seq_off, const int32_t* keep_k, float ratio, int b)
+{
+    const int n = seq_off[b + 1] - seq_off[b];
+    if (keep_k) return keep_k[b];
+    double kd = floor((double)ratio * (double)n);
+    kd = kd < 0.0 ? 0.0 : (kd > (double)n ? (double)n : kd);
+    return (int)kd;
+}
+
+// exclusive scan over the block; `total` receives the block sum
+__device__ __forceinline__ int block_exclusive_scan(int v, int* warp_sums, int& total)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_sums[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = lane < kTopkWarps ? warp_sums[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        if (lane < kTopkWarps) warp_sums[lane] = w;  // inclusive
+    }
+    __syncthreads();
+    const int before = (warp > 0 ? warp_sums[warp - 1] : 0) + x - v;
+    total = warp_sums[kTopkWarps - 1];
+    __syncthreads();
+    return before;
+}
+
+__global__ void __launch_bounds__(kTopkThreads)
+    topk_kernel(const float* __restrict__ scores, const int32_t* __restrict__ seq_off,
+                const int32_t* __restrict__ keep_k, float ratio, int32_t* __restrict__ kept_idx,
+                int32_t* __restrict__ out_off, int smem_keys)
+{
+    extern __shared__ uint32_t keys_s[];
+    __shared__ uint32_t hist[257];
+    __shared__ int warp_sums[kTopkWarps];
+    __shared__ uint32_t s_digit, s_above;
+    __shared__ long long s_base;
+
+    const int b = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int n0 = seq_off[b];
+    const int N = seq_off[b + 1] - n0;
+
+    // output base = sum of k over earlier requests
+    long long part = 0;
+    for (int bb = tid; bb < b; bb += kTopkThreads) part += keep_count(seq_off, keep_k, ratio, bb);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
+    if (tid == 0) s_base = 0;
+    __syncthreads();
+    if (lane == 0 && part) atomicAdd(reinterpret_cast<unsigned long long*>(&s_base), (unsigned long long)part);
+    __syncthreads();
+    const long long out_base = s_base;
+    const int k = keep_count(seq_off, keep_k, ratio, b);
+    if (tid == 0) {
+        out_off[b + 1] = (int32_t)(out_base + k);
+        if (b == 0) out_off[0] = 0;
+    }
+    if (k <= 0 || N <= 0) return;
+    int32_t* dst = kept_idx + out_base;
+    if (k >= N) {
+        for (int j = tid; j < N; j += kTopkThreads) dst[j] = n0 + j;
+        return;
+    }
+
+    const bool in_smem = N <= smem_keys;
+    if (in_smem) {
+        for (int j = tid; j < N; j += kTopkThreads) keys_s[j] = order_key(scores[n0 + j]);
+        __syncthreads();
+    }
+    auto key_at = [&](int j) -> uint32_t { return in_smem ? keys_s[j] : order_key(scores[n0 + j]); };
+
+    // ---- radix select of the k-th largest key
+    uint32_t prefix = 0u, mask = 0u;
+    int remaining = k;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        for (int i = tid; i < 257; i += kTopkThreads) hist[i] = 0u;
+        __syncthreads();
+        for (int base = warp * 32; base < N; base += kTopkThreads) {
+            const int j = base + lane;
+            uint32_t bin = 256u;
+            if (j < N) {
+                const uint32_t u = key_at(j);
+                if ((u & mask) == prefix) bin = (u >> shift) & 0xFFu;
+            }
+            const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+            if (lane == __ffs(peers) - 1) atomicAdd(&hist[bin], (uint32_t)__popc(peers));
+        }
+        __syncthreads();
+        if (warp == 0) {
+            uint32_t c[8], tot = 0;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                c[e] = hist[lane * 8 + e];
+                tot += c[e];
+            }
+            uint32_t suf = tot;  // sum over lanes >= this lane
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t y = __shfl_down_sync(0xffffffffu, suf, o);
+                if (lane + o < 32) suf += y;
+            }
+            uint32_t above = suf - tot;
+            if (above < (uint32_t)remaining && (uint32_t)remaining <= suf) {
+#pragma unroll
+                for (int e = 7; e >= 0; --e) {
+                    if (above + c[e] >= (uint32_t)remaining) {
+                        s_digit = (uint32_t)(lane * 8 + e);
+                        s_above = above;
+                        break;
+                    }
+                    above += c[e];
+                }
+            }
+        }
+        __syncthreads();
+        prefix |= s_digit << shift;
+        mask |= 0xFFu << shift;
+        remaining -= (int)s_above;
+        __syncthreads();
+    }
+
+    // ---- keep keys > prefix and the first `remaining` keys == prefix (index order)
+    const int ipt = (N + kTopkThreads - 1) / kTopkThreads;
+    const int j0 = min(N, tid * ipt), j1 = min(N, j0 + ipt);
+    int n_eq = 0;
+    for (int j = j0; j < j1; ++j) n_eq += key_at(j) == prefix;
+    int total;
+    const int eq_before = block_exclusive_scan(n_eq, warp_sums, total);
+    int n_keep = 0;
+    {
+        int e = eq_before;
+        for (int j = j0; j < j1; ++j) {
+            const uint32_t u = key_at(j);
+            if (u > prefix) ++n_keep;
+            else if (u == prefix) n_keep += (e++ < remaining);
+        }
+    }
+    int pos = block_exclusive_scan(n_keep, warp_sums, total);
+    {
+        int e = eq_before;
+        for (int j = j0; j < j1; ++j) {
+            const uint32_t u = key_at(j);
+            const bool keep = u > prefix || (u == prefix && e++ < remaining);
+            if (keep) dst[pos++] = n0 + j;
+        }
+    }
+}
+
+}  // namespace
+
+constexpr int kTopkSmemKeys = 40 * 1024;  // keys staged in shared memory (160 KB)
+
+cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,
+                        float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, cudaStream_t stream)
+{
+    if (batch <= 0) return cudaSuccess;
+    const int keys = max_n < kTopkSmemKeys ? max_n : kTopkSmemKeys;
+    const size_t smem = (size_t)(keys > 0 ? keys : 1) * 4;
+    cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    topk_kernel<<<batch, kTopkThreads, smem, stream>>>(scores, seq_off, keep_k, keep_ratio, kept_idx, out_off,
+                                                       keys);
+    return cudaGetLastError();
+}
+
+}  // namespace lvs

@@ -1,0 +1,227 @@
+"""Thin ctypes binding of the C-ABI in include/litevlm_select.h.
+
+Argument marshalling only: torch tensors give device pointers and the current
+CUDA stream; every step of the path runs in liblitevlm_select.so. There is no
+CPU fallback: if the library is missing the import of this module fails.
+
+Names follow the C functions: create / destroy / score / topk / compact /
+check_device (litevlm_select_*), plus ``Selector``, a small object that owns
+a handle and allocates outputs with torch.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "liblitevlm_select.so")
+
+STATUS = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "WORKSPACE", 4: "CUDA", 5: "TIMEOUT",
+          6: "DEVICE_BOUNDS"}
+DTYPES = {"bf16": 0, "e4m3": 1}
+
+
+class LitevlmError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS.get(status, status)}: {message}")
+        self.status = status
+        self.name = STATUS.get(status, str(status))
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("max_batch", ctypes.c_int32), ("max_total_visual", ctypes.c_int64),
+                ("max_total_text", ctypes.c_int64), ("num_q_heads", ctypes.c_int32),
+                ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("qk_dtype", ctypes.c_int32),
+                ("flags", ctypes.c_int32)]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is not built; run __graft_entry__.build() (needs nvcc)")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, i32, i64, f32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float
+    lib.litevlm_select_create.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(P)]
+    lib.litevlm_select_destroy.argtypes = [P]
+    lib.litevlm_select_last_error.argtypes = [P]
+    lib.litevlm_select_last_error.restype = ctypes.c_char_p
+    lib.litevlm_status_string.argtypes = [ctypes.c_int]
+    lib.litevlm_status_string.restype = ctypes.c_char_p
+    lib.litevlm_select_score.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P]
+    lib.litevlm_select_topk.argtypes = [P, i32, P, P, P, P, P, f32, P, P, P, P]
+    lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
+    lib.litevlm_select_check_device.argtypes = [P, P]
+    for fn in ("create", "destroy", "score", "topk", "compact", "check_device"):
+        getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
+    return lib
+
+
+LIB = _load()
+
+# every symbol declared in include/litevlm_select.h
+EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
+           "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
+           "litevlm_select_check_device"]
+
+
+def _check(rc: int, handle) -> None:
+    if rc != 0:
+        msg = LIB.litevlm_select_last_error(handle)
+        raise LitevlmError(rc, (msg or b"").decode())
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _host_i32(a) -> Optional[np.ndarray]:
+    if a is None:
+        return None
+    if isinstance(a, np.ndarray):
+        return np.ascontiguousarray(a, dtype=np.int32)
+    try:
+        import torch
+        if isinstance(a, torch.Tensor):
+            return np.ascontiguousarray(a.detach().cpu().numpy(), dtype=np.int32)
+    except ImportError:
+        pass
+    return np.ascontiguousarray(np.asarray(a), dtype=np.int32)
+
+
+def _stream_ptr(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+# ----------------------------------------------------------------------------
+# C functions, one to one
+# ----------------------------------------------------------------------------
+
+def create(max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int, num_kv_heads: int,
+           head_dim: int, qk_dtype: str = "bf16") -> int:
+    cfg = Config(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
+                 DTYPES[qk_dtype], 0)
+    h = ctypes.c_void_p()
+    _check(LIB.litevlm_select_create(ctypes.byref(cfg), ctypes.byref(h)), None)
+    return h.value
+
+
+def destroy(handle: int) -> None:
+    _check(LIB.litevlm_select_destroy(handle), handle)
+
+
+def score(handle: int, batch: int, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h,
+          q_scale: float, k_scale: float, scores, stream=None) -> None:
+    to_h, so_h = _host_i32(text_offsets_h), _host_i32(seq_offsets_h)
+    _check(LIB.litevlm_select_score(handle, batch, _ptr(q_text), _ptr(text_offsets_d), _ptr(to_h), _ptr(k_vis),
+                                    _ptr(seq_offsets_d), _ptr(so_h), q_scale, k_scale, _ptr(scores),
+                                    _stream_ptr(stream)), handle)
+
+
+def topk(handle: int, batch: int, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h, keep_ratio: float,
+         kept_idx, out_offsets_d, out_offsets_h: Optional[np.ndarray] = None, stream=None) -> None:
+    so_h, kk_h = _host_i32(seq_offsets_h), _host_i32(keep_k_h)
+    _check(LIB.litevlm_select_topk(handle, batch, _ptr(scores), _ptr(seq_offsets_d), _ptr(so_h), _ptr(keep_k_d),
+                                   _ptr(kk_h), keep_ratio, _ptr(kept_idx), _ptr(out_offsets_d),
+                                   _ptr(out_offsets_h), _stream_ptr(stream)), handle)
+
+
+def compact(handle: int, total_kept: int, kept_idx, src_rows: int, srcs: Sequence, dsts: Sequence,
+            row_bytes: Sequence[int], stream=None) -> None:
+    n = len(srcs)
+    src_arr = (ctypes.c_void_p * n)(*[_ptr(s) for s in srcs])
+    dst_arr = (ctypes.c_void_p * n)(*[_ptr(d) for d in dsts])
+    rb_arr = (ctypes.c_int64 * n)(*[int(r) for r in row_bytes])
+    _check(LIB.litevlm_select_compact(handle, total_kept, _ptr(kept_idx), src_rows, n, src_arr, dst_arr, rb_arr,
+                                      _stream_ptr(stream)), handle)
+
+
+def check_device(handle: int, stream=None) -> None:
+    _check(LIB.litevlm_select_check_device(handle, _stream_ptr(stream)), handle)
+
+
+# ----------------------------------------------------------------------------
+# convenience object (allocates outputs with torch; still marshalling only)
+# ----------------------------------------------------------------------------
+
+class Selector:
+    """Owns one handle. Tensors are torch CUDA tensors laid out as in the C header."""
+
+    def __init__(self, max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int,
+                 num_kv_heads: int, head_dim: int, qk_dtype: str = "bf16"):
+        self.handle = create(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
+                             qk_dtype)
+        self.qk_dtype = qk_dtype
+
+    def close(self) -> None:
+        if self.handle:
+            destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def score(self, q, text_offsets, k, seq_offsets, q_scale=1.0, k_scale=1.0, out=None, text_offsets_h=None,
+              seq_offsets_h=None, stream=None):
+        import torch
+        so_h = _host_i32(seq_offsets if seq_offsets_h is None else seq_offsets_h)
+        to_h = _host_i32(text_offsets if text_offsets_h is None else text_offsets_h)
+        if out is None:
+            out = torch.empty(int(so_h[-1]), dtype=torch.float32, device=k.device)
+        score(self.handle, len(so_h) - 1, q, text_offsets, to_h, k, seq_offsets, so_h, q_scale, k_scale, out,
+              stream)
+        return out
+
+    def topk(self, scores, seq_offsets, keep_k=None, keep_ratio: float = 0.0, seq_offsets_h=None, kept_idx=None,
+             out_offsets=None, stream=None):
+        """Returns (kept_idx, out_offsets device tensor, out_offsets host numpy)."""
+        import torch
+        so_h = _host_i32(seq_offsets if seq_offsets_h is None else seq_offsets_h)
+        batch = len(so_h) - 1
+        kk_h = _host_i32(keep_k)
+        kk_d = None
+        if kk_h is not None:
+            kk_d = keep_k if isinstance(keep_k, torch.Tensor) and keep_k.is_cuda else \
+                torch.from_numpy(kk_h).to(scores.device)
+        off_h = np.zeros(batch + 1, dtype=np.int32)
+        if kk_h is not None:
+            total = int(kk_h.sum())
+        else:
+            r = float(np.float32(keep_ratio))
+            total = int(sum(min(n, max(0, int(np.floor(r * n)))) for n in np.diff(so_h)))
+        if kept_idx is None:
+            kept_idx = torch.empty(max(total, 1), dtype=torch.int32, device=scores.device)
+        if out_offsets is None:
+            out_offsets = torch.empty(batch + 1, dtype=torch.int32, device=scores.device)
+        topk(self.handle, batch, scores, seq_offsets, so_h, kk_d, kk_h, keep_ratio, kept_idx, out_offsets, off_h,
+             stream)
+        self._keep_alive = kk_d
+        return kept_idx[:int(off_h[-1])], out_offsets, off_h
+
+    def compact(self, kept_idx, total_kept: int, srcs: Sequence, dsts: Optional[List] = None, stream=None):
+        import torch
+        rows = [s.shape[0] for s in srcs]
+        if dsts is None:
+            dsts = [torch.empty((max(total_kept, 0),) + tuple(s.shape[1:]), dtype=s.dtype, device=s.device)
+                    for s in srcs]
+        rb = [s[0].numel() * s.element_size() if s.shape[0] else 1 for s in srcs]
+        compact(self.handle, total_kept, kept_idx, min(rows) if rows else 0, srcs, dsts, rb, stream)
+        return dsts
+
+    def check_device(self, stream=None) -> None:
+        check_device(self.handle, stream)

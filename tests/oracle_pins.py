@@ -155,6 +155,22 @@ def pin_row_and_total_sums(lib):
             assert abs(s64[so[b]:so[b + 1]].sum() - 1.0) < 1e-13
 
 
+def pin_batch_equals_single_requests(lib):
+    """Requests are independent: scoring a ragged batch gives, for each request,
+    the scores of that request scored alone."""
+    hq, hkv, d = 4, 2, 16
+    n_vis, n_txt = [13, 0, 40, 9], [3, 2, 5, 1]
+    q, k, so, to = _ragged(22, hq, hkv, d, n_vis, n_txt)
+    _, whole, _, _ = oracle.score(q, k, so, to, hq, hkv, d, "f32", lib=lib, details=True)
+    for b in range(len(n_vis)):
+        if n_vis[b] == 0:
+            continue
+        qb, kb = q[to[b]:to[b + 1]], k[so[b]:so[b + 1]]
+        _, alone, _, _ = oracle.score(qb, kb, [0, n_vis[b]], [0, n_txt[b]], hq, hkv, d, "f32", lib=lib,
+                                      details=True)
+        np.testing.assert_array_equal(whole[so[b]:so[b + 1]], alone)
+
+
 def pin_permutation_equivariance(lib):
     q, k, so, to = _ragged(14, 4, 4, 16, [41], [6])
     perm = np.random.Generator(np.random.PCG64(15)).permutation(41)
@@ -273,6 +289,6 @@ def pin_compact(lib):
 
 
 ALL_PINS = [pin_bf16_decode, pin_e4m3_decode, pin_worked_example, pin_uniform_keys, pin_single_query_is_softmax,
-            pin_row_and_total_sums, pin_permutation_equivariance, pin_gqa_replication, pin_scale_placement,
+            pin_row_and_total_sums, pin_batch_equals_single_requests, pin_permutation_equivariance, pin_gqa_replication, pin_scale_placement,
             pin_e4m3_scores, pin_salient_tokens_rank_first, pin_topk_bruteforce, pin_topk_batch_and_ratio,
             pin_table1_token_counts, pin_compact]

@@ -14,8 +14,12 @@ SRC = os.path.join(os.path.dirname(oracle.__file__), "litevlm_oracle.c")
 # (name, original text, planted text)
 MUTANTS = [
     ("gqa_head_map_modulo", "const int32_t g = h / group;", "const int32_t g = h % hkv;"),
-    ("key_head_always_zero", "const int64_t krow = ((n0 + j) * hkv + g) * head_dim;",
-     "const int64_t krow = ((n0 + j) * hkv + 0) * head_dim;"),
+    ("key_head_always_zero", "const int64_t krow = (j * hkv + g) * head_dim;",
+     "const int64_t krow = (j * hkv + 0) * head_dim;"),
+    ("key_rows_of_first_request", "kd[x] = litevlm_oracle_decode(dtype, k, n0 * hkv * head_dim + x);",
+     "kd[x] = litevlm_oracle_decode(dtype, k, x);"),
+    ("query_rows_of_first_request", "qd[x] = litevlm_oracle_decode(dtype, q, t0 * hq * head_dim + x);",
+     "qd[x] = litevlm_oracle_decode(dtype, q, x);"),
     ("scale_1_over_d", "/ sqrt((double)head_dim)", "/ (double)head_dim"),
     ("logit_sign", "s[j] = dot * scale;", "s[j] = -dot * scale;"),
     ("no_mean_over_queries", "const double denom = (double)hq * (double)tb;", "const double denom = (double)hq;"),
