@@ -1,0 +1,305 @@
+"""Parity of the CUDA path (through the C-ABI) with the CPU oracle.
+
+Bar: scores within a relative tolerance of 2e-3 (bf16) / 3e-2 (e4m3) per
+element; top-k indices and gathered rows bit-exact when top-k and the gather
+are fed the oracle's scores / indices. Small cases span several 128-token
+tiles and ragged tails; the full-size workloads run in the launch
+configuration the benchmark times and are checked on sampled requests (and by
+invariants on all of them)."""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+from gpu_util import (RTOL, assert_scores_close, gather_rows, rel_err, sub_offsets, to_device, to_host)
+from paper_2506_07416_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def sel():
+    if not torch.cuda.is_available():
+        pytest.fail("the GPU tests need a CUDA device")
+    from paper_2506_07416_gb300 import select
+    return select
+
+
+def _case(name, hq, hkv, d, dtype, n_vis, n_txt, sigma=None, seed=7):
+    return inputs.Workload(name, len(n_vis), list(n_vis), list(n_txt), hq, hkv, d, 256, dtype, keep_ratio=0.3,
+                           sigma=(1.0 / math.sqrt(d)) if sigma is None else sigma, seed=seed)
+
+
+SCORE_CASES = [
+    inputs.workload("tiny"),
+    _case("mha_ragged_tails", 16, 16, 128, "bf16", [1, 127, 128, 129, 700, 0, 1536], [64, 1, 16, 33, 128, 5, 64]),
+    _case("gqa_7to1", 28, 4, 128, "bf16", [1000, 2049], [128, 77]),
+    _case("d64", 4, 4, 64, "bf16", [300, 5, 64], [16, 3, 1]),
+    _case("e4m3_ragged", 8, 8, 128, "e4m3", [576, 1152, 100], [32, 128, 50]),
+    _case("many_tiles_one_request", 2, 1, 128, "bf16", [9000], [40]),
+    _case("sharp_logits", 4, 4, 128, "bf16", [513], [17], sigma=3.0),
+]
+
+
+def _selector(sel, w, max_batch=None):
+    return sel.Selector(max_batch or max(1, w.batch), max(1, w.total_vis), max(1, w.total_txt), w.hq, w.hkv,
+                        w.head_dim, w.dtype)
+
+
+def _gpu_scores(sel, s, w, x, xd):
+    out = s.score(xd["q"], xd["text_offsets"], xd["k"], xd["seq_offsets"], xd["q_scale"], xd["k_scale"],
+                  seq_offsets_h=x["seq_offsets"], text_offsets_h=x["text_offsets"])
+    s.check_device()
+    return out.cpu().numpy()
+
+
+@pytest.mark.parametrize("w", SCORE_CASES, ids=lambda w: w.name)
+def test_scores_match_oracle(sel, w):
+    x = inputs.make_numpy(w)
+    xd = to_device(x, w)
+    s = _selector(sel, w)
+    g = _gpu_scores(sel, s, w, x, xd)
+    o = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, w.dtype,
+                     x["q_scale"], x["k_scale"])
+    assert_scores_close(g, o, w.dtype)
+    # deterministic: a second call gives the same bits
+    g2 = _gpu_scores(sel, s, w, x, xd)
+    np.testing.assert_array_equal(g, g2)
+    so = x["seq_offsets"]
+    for b in range(w.batch):
+        if so[b + 1] > so[b]:
+            assert abs(float(np.sum(g[so[b]:so[b + 1]], dtype=np.float64)) - 1.0) < 1e-4
+
+
+def test_empty_and_zero_length_requests(sel):
+    w = _case("zeros", 4, 2, 128, "bf16", [0, 0, 3, 0], [1, 4, 2, 0])
+    x = inputs.make_numpy(w)
+    xd = to_device(x, w)
+    s = _selector(sel, w)
+    g = _gpu_scores(sel, s, w, x, xd)
+    o = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, "bf16")
+    assert_scores_close(g, o, "bf16")
+    # batch 0 is a no-op
+    sel.score(s.handle, 0, xd["q"], xd["text_offsets"], np.zeros(1, np.int32), xd["k"], xd["seq_offsets"],
+              np.zeros(1, np.int32), 1.0, 1.0, torch.empty(1, device="cuda"))
+    s.check_device()
+
+
+def test_score_argument_errors(sel):
+    w = _case("errs", 4, 4, 128, "bf16", [10, 5], [3, 0])
+    x = inputs.make_numpy(w)
+    xd = to_device(x, w)
+    s = _selector(sel, w)
+    with pytest.raises(sel.LitevlmError) as e:  # visual tokens without text
+        s.score(xd["q"], xd["text_offsets"], xd["k"], xd["seq_offsets"], seq_offsets_h=x["seq_offsets"],
+                text_offsets_h=x["text_offsets"])
+    assert e.value.name == "INVALID_ARG"
+    w2 = _case("long_text", 4, 4, 128, "bf16", [10], [129])
+    x2 = inputs.make_numpy(w2)
+    xd2 = to_device(x2, w2)
+    s2 = _selector(sel, w2)
+    with pytest.raises(sel.LitevlmError) as e:
+        s2.score(xd2["q"], xd2["text_offsets"], xd2["k"], xd2["seq_offsets"], seq_offsets_h=x2["seq_offsets"],
+                 text_offsets_h=x2["text_offsets"])
+    assert e.value.name == "UNSUPPORTED"
+    with pytest.raises(sel.LitevlmError) as e:  # bf16 takes no scales
+        s2.score(xd2["q"], xd2["text_offsets"], xd2["k"], xd2["seq_offsets"], q_scale=2.0,
+                 seq_offsets_h=x2["seq_offsets"], text_offsets_h=x2["text_offsets"])
+
+
+# ----------------------------------------------------------------------------- top-k
+
+def _topk_gpu(sel, s, scores_np, so, keep_k=None, ratio=0.0):
+    d = torch.from_numpy(np.ascontiguousarray(scores_np, dtype=np.float32)).cuda()
+    so_d = torch.from_numpy(np.ascontiguousarray(so, dtype=np.int32)).cuda()
+    kept, off_d, off_h = s.topk(d, so_d, keep_k=keep_k, keep_ratio=ratio, seq_offsets_h=so)
+    s.check_device()
+    return kept.cpu().numpy(), off_d.cpu().numpy(), off_h
+
+
+@pytest.mark.parametrize("w", SCORE_CASES[:5], ids=lambda w: w.name)
+def test_topk_on_oracle_scores_is_bit_exact(sel, w):
+    x = inputs.make_numpy(w)
+    o = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, w.dtype,
+                     x["q_scale"], x["k_scale"])
+    s = _selector(sel, w)
+    so = x["seq_offsets"]
+    for ratio in (0.0, 0.1, 0.3, 0.5, 0.9, 1.0):
+        kept, off_d, off_h = _topk_gpu(sel, s, o, so, ratio=ratio)
+        ok, ooff = oracle.topk(so, o, keep_ratio=ratio)
+        np.testing.assert_array_equal(kept, ok)
+        np.testing.assert_array_equal(off_d, ooff)
+        np.testing.assert_array_equal(off_h, ooff)
+    keep = [max(0, n // 3 - 1) for n in np.diff(so)]
+    kept, off_d, _ = _topk_gpu(sel, s, o, so, keep_k=keep)
+    ok, ooff = oracle.topk(so, o, keep_k=keep)
+    np.testing.assert_array_equal(kept, ok)
+    np.testing.assert_array_equal(off_d, ooff)
+
+
+def test_topk_ties_nan_signed_zero(sel):
+    rng = np.random.Generator(np.random.PCG64(5))
+    n_vis = [1, 2, 37, 0, 128, 129, 1000, 4097]
+    so = np.concatenate([[0], np.cumsum(n_vis)]).astype(np.int32)
+    vals = np.array([0.0, -0.0, np.nan, np.inf, -np.inf, 1.0, 0.5, 0.5, -1e-30, 3.4e38], np.float32)
+    scores = rng.choice(vals, size=so[-1]).astype(np.float32)
+    w = _case("ties", 1, 1, 128, "bf16", n_vis, [1] * len(n_vis))
+    s = _selector(sel, w)
+    for trial in range(4):
+        keep = [int(rng.integers(0, n + 1)) for n in n_vis]
+        kept, off_d, _ = _topk_gpu(sel, s, scores, so, keep_k=keep)
+        ok, ooff = oracle.topk(so, scores, keep_k=keep)
+        np.testing.assert_array_equal(kept, ok)
+        np.testing.assert_array_equal(off_d, ooff)
+    # all equal: the first k indices
+    flat = np.full(so[-1], 0.25, np.float32)
+    kept, _, _ = _topk_gpu(sel, s, flat, so, ratio=0.5)
+    ok, _ = oracle.topk(so, flat, keep_ratio=0.5)
+    np.testing.assert_array_equal(kept, ok)
+
+
+def test_topk_request_larger_than_shared_memory_stage(sel):
+    rng = np.random.Generator(np.random.PCG64(6))
+    n_vis = [50000, 300]
+    so = np.concatenate([[0], np.cumsum(n_vis)]).astype(np.int32)
+    scores = np.round(rng.standard_normal(so[-1]), 2).astype(np.float32)  # many ties
+    w = _case("big", 1, 1, 128, "bf16", n_vis, [1, 1])
+    s = _selector(sel, w)
+    keep = [12345, 150]
+    kept, off_d, _ = _topk_gpu(sel, s, scores, so, keep_k=keep)
+    ok, ooff = oracle.topk(so, scores, keep_k=keep)
+    np.testing.assert_array_equal(kept, ok)
+    np.testing.assert_array_equal(off_d, ooff)
+
+
+def test_topk_argument_errors(sel):
+    w = _case("e", 1, 1, 128, "bf16", [10], [1])
+    s = _selector(sel, w)
+    so = np.array([0, 10], np.int32)
+    with pytest.raises(sel.LitevlmError):
+        _topk_gpu(sel, s, np.zeros(10, np.float32), so, keep_k=[11])
+    with pytest.raises(sel.LitevlmError):
+        _topk_gpu(sel, s, np.zeros(10, np.float32), so, ratio=1.5)
+
+
+# ----------------------------------------------------------------------------- gather
+
+def test_compact_bit_exact(sel):
+    rng = np.random.Generator(np.random.PCG64(8))
+    rows = 777
+    w = _case("g", 1, 1, 128, "bf16", [rows], [1])
+    s = _selector(sel, w)
+    idx = np.sort(rng.choice(rows, size=311, replace=False)).astype(np.int32)
+    tensors = [rng.integers(0, 256, size=(rows, 4096), dtype=np.uint8),   # hidden-sized rows
+               rng.integers(0, 256, size=(rows, 2048), dtype=np.uint8),   # K rows
+               rng.integers(0, 256, size=(rows, 48), dtype=np.uint8),     # short rows
+               rng.integers(0, 256, size=(rows, 6), dtype=np.uint8)]      # unaligned rows (byte path)
+    for group in (tensors[:3], tensors[3:]):
+        srcs = [torch.from_numpy(t).cuda() for t in group]
+        dsts = s.compact(torch.from_numpy(idx).cuda(), len(idx), srcs)
+        s.check_device()
+        for t, d in zip(group, dsts):
+            np.testing.assert_array_equal(d.cpu().numpy(), oracle.compact(idx, t))
+    assert s.compact(torch.from_numpy(idx).cuda(), 0, [torch.from_numpy(tensors[0]).cuda()])[0].numel() == 0
+
+
+def test_compact_out_of_range_index_is_reported(sel):
+    w = _case("g", 1, 1, 128, "bf16", [8], [1])
+    s = _selector(sel, w)
+    src = torch.arange(8 * 16, dtype=torch.uint8, device="cuda").view(8, 16)
+    idx = torch.tensor([1, 8, 3], dtype=torch.int32, device="cuda")  # 8 is outside [0, 8)
+    dst = s.compact(idx, 3, [src])[0]
+    with pytest.raises(sel.LitevlmError) as e:
+        s.check_device()
+    assert e.value.name == "DEVICE_BOUNDS"
+    assert torch.equal(dst[0], src[1]) and torch.equal(dst[2], src[3])
+    s.check_device()  # the word was cleared
+
+
+# ----------------------------------------------------------------------------- whole path
+
+def test_tiny_whole_path(sel):
+    w = inputs.workload("tiny")
+    x = inputs.make_numpy(w)
+    xd = to_device(x, w)
+    s = _selector(sel, w)
+    g = _gpu_scores(sel, s, w, x, xd)
+    o, okept, ooff, orows = oracle.select(x, w.hq, w.hkv, w.head_dim, "bf16", keep_k=w.keep_k)
+    assert_scores_close(g, o, "bf16")
+    kept, off_d, off_h = s.topk(torch.from_numpy(g).cuda(), xd["seq_offsets"], keep_k=w.keep_k,
+                                seq_offsets_h=x["seq_offsets"])
+    # the GPU's selection is the exact top-k of the GPU's scores
+    gk, _ = oracle.topk(x["seq_offsets"], g, keep_k=w.keep_k)
+    np.testing.assert_array_equal(kept.cpu().numpy(), gk)
+    # with the oracle's scores it is the oracle's selection
+    k2, _, _ = s.topk(torch.from_numpy(o).cuda(), xd["seq_offsets"], keep_k=w.keep_k, seq_offsets_h=x["seq_offsets"])
+    np.testing.assert_array_equal(k2.cpu().numpy(), okept)
+    rows = s.compact(k2, int(off_h[-1]), [xd["hidden"]])[0]
+    s.check_device()
+    np.testing.assert_array_equal(rows.view(torch.int16).cpu().numpy().view(np.uint16), orows["hidden"])
+    # the 8 salient tokens are among the kept ones
+    assert set((x["salient"][0]).tolist()) <= set(gk.tolist())
+
+
+# ----------------------------------------------------------------------------- full size
+
+FULL = [("single", [0]), ("highres", [0]), ("fp8_ragged", None), ("sweep", [0, 77, 127])]
+
+
+@pytest.mark.parametrize("name,sample", FULL, ids=[f[0] for f in FULL])
+def test_full_size_workload(sel, name, sample):
+    w = inputs.workload(name)
+    xd = inputs.make_torch(w, "cuda")
+    so, to = w.seq_offsets(), w.text_offsets()
+    s = _selector(sel, w)
+    g_t = s.score(xd["q"], xd["text_offsets"], xd["k"], xd["seq_offsets"], xd["q_scale"], xd["k_scale"],
+                  seq_offsets_h=so, text_offsets_h=to)
+    s.check_device()
+    g = g_t.cpu().numpy()
+    # invariant on every request: the scores of a request sum to 1
+    sums = np.add.reduceat(g.astype(np.float64), so[:-1]) if w.batch > 1 else np.array([g.sum(dtype=np.float64)])
+    assert np.max(np.abs(sums - 1.0)) < 1e-4
+    if sample is None:  # smallest, largest and a middle request
+        order = np.argsort(np.diff(so), kind="stable")
+        sample = sorted({int(order[0]), int(order[-1]), int(order[len(order) // 2])})
+    # sampled requests against the oracle
+    qh = to_host({"q": xd["q"], "k": xd["k"]})
+    sq = gather_rows(qh["q"], to, sample)
+    sk = gather_rows(qh["k"], so, sample)
+    sso, sto = sub_offsets(so, sample), sub_offsets(to, sample)
+    o = oracle.score(sq, sk, sso, sto, w.hq, w.hkv, w.head_dim, w.dtype, xd["q_scale"], xd["k_scale"])
+    gs = np.concatenate([g[so[b]:so[b + 1]] for b in sample])
+    err = assert_scores_close(gs, o, w.dtype)
+    print(f"{name}: max rel err {err:.2e} on requests {sample}")
+    # top-k fed the oracle's scores: bit-exact on the sampled requests
+    ss = _selector(sel, inputs.sub_batch(w, sample))
+    ratios = [0.1, 0.2, 0.3, 0.5] if name == "sweep" else [None]
+    for r in ratios:
+        kk = None if w.keep_k is None else [w.keep_k[b] for b in sample]
+        rr = w.keep_ratio if r is None else r
+        kept, off_d, _ = _topk_gpu(sel, ss, o, sso, keep_k=kk, ratio=rr or 0.0)
+        ok, ooff = oracle.topk(sso, o, keep_k=kk, keep_ratio=rr or 0.0)
+        np.testing.assert_array_equal(kept, ok)
+        np.testing.assert_array_equal(off_d, ooff)
+    # top-k on the GPU scores of every request is the exact top-k of those scores,
+    # and the gather moves exactly those rows
+    for r in ratios:
+        rr = w.keep_ratio if r is None else r
+        kept_t, off_d, off_h = s.topk(g_t, xd["seq_offsets"], keep_k=w.keep_k if r is None else None,
+                                      keep_ratio=rr or 0.0, seq_offsets_h=so)
+        ok, ooff = oracle.topk(so, g, keep_k=w.keep_k if r is None else None, keep_ratio=rr or 0.0)
+        np.testing.assert_array_equal(kept_t.cpu().numpy(), ok)
+        np.testing.assert_array_equal(off_h, ooff)
+        srcs = [xd[n] for n in w.gather]
+        outs = s.compact(kept_t, int(off_h[-1]), srcs)
+        s.check_device()
+        idx = kept_t.long()
+        for src, dst in zip(srcs, outs):
+            assert torch.equal(dst.view(torch.uint8) if dst.dtype != torch.uint8 else dst,
+                               src.index_select(0, idx).view(torch.uint8) if src.dtype != torch.uint8
+                               else src.index_select(0, idx))
+    del xd
+    torch.cuda.empty_cache()
