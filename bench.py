@@ -46,6 +46,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=None)
     ap.add_argument("--workload", default="single", choices=["single", "highres", "fp8_ragged", "sweep"])
     ap.add_argument("--ratio", type=float, default=None, help="keep ratio override (sweep: 0.1/0.2/0.3/0.5)")
+    ap.add_argument("--batch", type=int, default=None, help="use only the first B requests (profiling)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="bounded CPU work for the oracle baseline")
@@ -61,6 +62,8 @@ def workload_for(args):
     if args.ratio is not None:
         from dataclasses import replace
         w = replace(w, keep_ratio=args.ratio, keep_k=None)
+    if args.batch is not None and args.batch < w.batch:
+        w = inputs.sub_batch(w, list(range(args.batch)))
     return w
 
 

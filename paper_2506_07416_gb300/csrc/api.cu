@@ -19,6 +19,7 @@ struct litevlm_select {
     int device = 0;
     int num_sms = 0;
     float* partials = nullptr;  // [Hq][max_total_visual]: per-head-group partial scores
+    int32_t* counters = nullptr;  // [max_batch]: fold tickets of the score kernel
     int32_t* err_d = nullptr;   // device error word (bits lvs::kErr*)
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     std::string last_error;
@@ -68,12 +69,12 @@ int64_t keep_count_host(int32_t n, float ratio)
 }
 
 litevlm_status_t encode_rows_map(litevlm_select_t h, CUtensorMap* map, const void* base, int32_t head_dim,
-                                 int32_t heads, int64_t rows, bool fp8, const char* what)
+                                 int32_t heads, int64_t rows, int box_rows, bool fp8, const char* what)
 {
     const int esize = fp8 ? 1 : 2;
     const cuuint64_t dims[3] = {(cuuint64_t)head_dim, (cuuint64_t)heads, (cuuint64_t)rows};
     const cuuint64_t strides[2] = {(cuuint64_t)head_dim * esize, (cuuint64_t)heads * head_dim * esize};
-    const cuuint32_t box[3] = {(cuuint32_t)(128 / esize), 1u, 128u};
+    const cuuint32_t box[3] = {(cuuint32_t)(128 / esize), 1u, (cuuint32_t)box_rows};
     const cuuint32_t estride[3] = {1u, 1u, 1u};
     const CUresult r = h->encode(map, fp8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
                                  const_cast<void*>(base), dims, strides, box, estride,
@@ -154,8 +155,12 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
     if (e == cudaSuccess) e = cudaMemset(h->err_d, 0, sizeof(int32_t));
     if (e == cudaSuccess && c->num_q_heads > 1)
         e = cudaMalloc(&h->partials, sizeof(float) * (size_t)c->num_q_heads * (size_t)c->max_total_visual);
+    if (e == cudaSuccess) e = cudaMalloc(&h->counters, sizeof(int32_t) * (size_t)c->max_batch);
+    if (e == cudaSuccess) e = cudaMemset(h->counters, 0, sizeof(int32_t) * (size_t)c->max_batch);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         const std::string msg = std::string("create: ") + cudaGetErrorString(e);
+        if (h->counters) cudaFree(h->counters);
         if (h->err_d) cudaFree(h->err_d);
         if (h->partials) cudaFree(h->partials);
         delete h;
@@ -170,6 +175,7 @@ litevlm_status_t litevlm_select_destroy(litevlm_select_t h)
 {
     if (!h) return LITEVLM_OK;
     if (h->partials) cudaFree(h->partials);
+    if (h->counters) cudaFree(h->counters);
     if (h->err_d) cudaFree(h->err_d);
     delete h;
     return LITEVLM_OK;
@@ -193,7 +199,7 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
     if (s != LITEVLM_OK) return s;
     s = check_offsets(h, text_offsets_h, batch, c.max_total_text, "text_offsets", &tot_t);
     if (s != LITEVLM_OK) return s;
-    int max_tiles = 0, max_n = 0;
+    int max_tiles = 0, max_n = 0, max_t = 0;
     for (int32_t b = 0; b < batch; ++b) {
         const int32_t n = seq_offsets_h[b + 1] - seq_offsets_h[b];
         const int32_t t = text_offsets_h[b + 1] - text_offsets_h[b];
@@ -209,6 +215,7 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
         const int tiles = (n + lvs::kTileRows - 1) / lvs::kTileRows;
         if (tiles > max_tiles) max_tiles = tiles;
         if (n > max_n) max_n = n;
+        if (n > 0 && t > max_t) max_t = t;
     }
     if (tot_n == 0) return LITEVLM_OK;
     if (!q_text || !k_vis || !scores || !text_offsets_d || !seq_offsets_d)
@@ -221,28 +228,32 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
     } else if (q_scale != 1.f || k_scale != 1.f) {
         return fail(h, LITEVLM_ERR_INVALID_ARG, "q_scale and k_scale must be 1 for bf16 inputs");
     }
-    const lvs::ScorePlan plan = lvs::plan_score(batch, max_tiles, c.num_q_heads, h->num_sms);
+    const int row_bytes = c.head_dim * (fp8 ? 1 : 2);
+    const lvs::ScorePlan plan = lvs::plan_score(batch, max_tiles, c.num_q_heads, c.num_kv_heads,
+                                                lvs::kTileRows * row_bytes, h->num_sms);
     if (plan.tiles_per_cta > lvs::kMaxTilesPerCta)
         return fail(h, LITEVLM_ERR_UNSUPPORTED, "request too long for one cluster");
+    const int mrows = max_t <= 64 ? 64 : 128;  // text rows of the pass-1 MMA
 
     CUtensorMap tm_q, tm_k;
-    s = encode_rows_map(h, &tm_q, q_text, c.head_dim, c.num_q_heads, tot_t, fp8, "q_text");
+    s = encode_rows_map(h, &tm_q, q_text, c.head_dim, c.num_q_heads, tot_t, mrows, fp8, "q_text");
     if (s != LITEVLM_OK) return s;
-    s = encode_rows_map(h, &tm_k, k_vis, c.head_dim, c.num_kv_heads, tot_n, fp8, "k_vis");
+    s = encode_rows_map(h, &tm_k, k_vis, c.head_dim, c.num_kv_heads, tot_n, lvs::kTileRows, fp8, "k_vis");
     if (s != LITEVLM_OK) return s;
 
     lvs::ScoreLaunch p{};
     p.seq_off = seq_offsets_d;
     p.text_off = text_offsets_d;
+    p.out = scores;
+    p.partials = h->partials;
+    p.counters = h->counters;
     p.err = h->err_d;
     p.total_vis = tot_n;
     p.hq = c.num_q_heads;
     p.hkv = c.num_kv_heads;
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
     p.wait_budget = lvs::kWaitBudgetCycles;
-    const int row_bytes = c.head_dim * (fp8 ? 1 : 2);
-    const cudaError_t e = lvs::launch_score(tm_q, tm_k, p, plan, batch, row_bytes, fp8, h->partials, scores, max_n,
-                                            (cudaStream_t)stream);
+    const cudaError_t e = lvs::launch_score(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "score launch");
     return LITEVLM_OK;
 }

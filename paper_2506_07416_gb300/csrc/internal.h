@@ -21,15 +21,17 @@ constexpr int kMaxCluster = 16;
 constexpr long long kWaitBudgetCycles = 4000000000LL;
 
 struct ScoreLaunch {
-    // device inputs
-    const int32_t* seq_off;
-    const int32_t* text_off;
-    float* out;               // scores [sum N] (one head group) or partials [groups][sum N]
+    const int32_t* seq_off;   // device [batch+1]
+    const int32_t* text_off;  // device [batch+1]
+    float* out;               // scores [sum N]
+    float* partials;          // [groups][sum N] when groups > 1 (workspace)
+    int32_t* counters;        // [batch] fold tickets, zero between launches (workspace)
     int32_t* err;
     int64_t total_vis;        // partial-row stride
     int32_t hq, hkv;
     int32_t heads_per_group;
     int32_t groups;
+    int32_t ctas_per_request; // cluster size * groups
     float c_log2;             // q_scale * k_scale / sqrt(d) * log2(e)
     long long wait_budget;
 };
@@ -41,12 +43,10 @@ struct ScorePlan {
 };
 
 // Host helpers (score_tc.cu)
-ScorePlan plan_score(int batch, int max_tiles, int hq, int num_sms);
+ScorePlan plan_score(int batch, int max_tiles, int hq, int hkv, int tile_bytes, int num_sms);
 cudaError_t launch_score(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
-                         const ScorePlan& plan, int batch, int row_bytes, bool fp8, float* partials,
-                         float* scores, int max_n, cudaStream_t stream);
+                         const ScorePlan& plan, int batch, int row_bytes, bool fp8, int mrows, cudaStream_t stream);
 bool score_shape_supported(int head_dim, bool fp8);
-size_t score_smem_bytes(int row_bytes);
 
 // topk.cu
 cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,

@@ -9,21 +9,25 @@
 //
 // Work decomposition. One thread-block cluster of C CTAs serves one (request,
 // head group); CTA r of the cluster owns a contiguous range of 128-token tiles
-// of the request. For each query head h of the group, the CTA
-//   pass 1: D1 = Q_h * K_tile^T on tcgen05 (M = 128 text rows, N = 128 visual
-//           columns) into TMEM; one epilogue thread per text row keeps an online
-//           (max, sum of exp) over the columns of all its tiles;
+// of the request. For every query head h of the group:
+//   pass 1: D1 = Q_h * K_tile^T on tcgen05 (M = 64 or 128 text rows, N = 128
+//           visual columns) into TMEM; one or two epilogue threads per text row
+//           keep an online (max, sum of 2^x) over the columns of all the CTA's
+//           tiles;
 //   exchange: each CTA publishes its per-row (m, l) in shared memory and
-//           signals every CTA of the cluster through remote mbarrier arrivals;
-//           every CTA merges the C partials in rank order (deterministic) into
-//           b_hi = m_hi*log2(e)*scale + log2(l_hi);
+//           signals every CTA of the cluster by remote mbarrier arrivals; each
+//           CTA merges the C partials in rank order (deterministic) into
+//           b_hi = m_hi * c + log2(l_hi), c = scale * log2(e);
 //   pass 2: D2 = K_tile * Q_h^T (M = 128 visual rows, N = T rounded up to 16)
 //           into TMEM; one epilogue thread per visual token adds
-//           sum_i 2^(s_ij*c - b_hi) to its running score.
-// The K tiles stream through a TMA ring twice per head (the second pass reads
-// the CTA's few tiles again, normally from L2). Scores sum over the heads of
-// the group in shared memory; one head group writes final scores, several
-// write partial rows that a fold kernel adds in a fixed order.
+//           sum_i 2^(s_ij * c - b_hi) to its running score.
+// Software pipeline with one head of look-ahead: pass 1 of head s+1 runs while
+// the statistics of head s travel across the cluster, then pass 2 of head s.
+// The K tiles stream through a TMA ring for both passes (the pass-2 re-read of
+// a CTA's few tiles is normally served by L2). Scores are summed over the heads
+// of the group in shared memory; with one head group they are final, with
+// several the CTAs write partial rows and the last CTA of the request to finish
+// (atomic ticket) adds them in a fixed order.
 //
 // Warp roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
 // MMA issuer, warps 2..5 = epilogue (TMEM lane quadrant = warp % 4).
@@ -40,25 +44,33 @@ namespace lvs {
 namespace {
 
 constexpr int kThreads = 192;
+constexpr int kStatSlots = 4;  // stats of heads s-3..s may be live across the cluster
 
-// Ring depth: 4 x 32 KB tiles for 256-byte rows, 8 x 16 KB for 128-byte rows.
-// Both layouts need more than half of the SM's shared memory, so a single CTA
-// (and a single 512-column TMEM allocation) lives on an SM at a time.
-template <int ROW_BYTES>
+// Shared-memory plan. The ring gets whatever is left of the 227 KB after the
+// Q double buffer and the bookkeeping; every variant needs more than half of
+// the SM's shared memory, so a single CTA (and a single 512-column TMEM
+// allocation) lives on an SM at a time.
+template <int ROW_BYTES, int MROWS>
 struct SmemLayout {
-    static constexpr int kStages = ROW_BYTES == 256 ? 4 : 8;
     static constexpr int KB = ROW_BYTES / 128;             // 128-byte swizzle blocks along d
     static constexpr int TILE_BYTES = kTileRows * ROW_BYTES;
-    static constexpr int Q_BYTES = kMaxText * ROW_BYTES;   // Q tile: 128 text rows
+    static constexpr int Q_BYTES = MROWS * ROW_BYTES;
+    // Q(s) lives from pass 1 of head s to pass 2 of head s; a third buffer lets
+    // Q(s+2) load while pass 2 of head s is still reading Q(s).
+    static constexpr int QBUF = MROWS == 64 ? 3 : 2;
+    static constexpr int FIXED = QBUF * Q_BYTES + kMaxTilesPerCta * kTileRows * 4 + kStatSlots * kMaxText * 8 +
+                                 2 * kMaxText * 4 + 512 + 64 + 1024;
+    static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
+    static constexpr int kStages = STAGES_FIT > 10 ? 10 : STAGES_FIT;
     static constexpr int OFF_K = 0;
     static constexpr int OFF_Q = OFF_K + kStages * TILE_BYTES;
-    static constexpr int OFF_ACC = OFF_Q + 2 * Q_BYTES;
+    static constexpr int OFF_ACC = OFF_Q + QBUF * Q_BYTES;
     static constexpr int OFF_STATS = OFF_ACC + kMaxTilesPerCta * kTileRows * 4;
-    static constexpr int OFF_B2 = OFF_STATS + 2 * kMaxText * 8;
-    static constexpr int OFF_BAR = OFF_B2 + kMaxText * 4;
-    // barriers: k_full[S], k_empty[S], q_full[2], q_empty[2], t1_full[2], t1_empty[2],
-    //           t2_full[2], t2_empty[2], stats[2], drain
-    static constexpr int NBAR = 2 * kStages + 2 * 2 * 4 + 2 + 1;
+    static constexpr int OFF_B2 = OFF_STATS + kStatSlots * kMaxText * 8;
+    static constexpr int OFF_BAR = OFF_B2 + 2 * kMaxText * 4;
+    // k_full[S], k_empty[S], q_full[QBUF], q_empty[QBUF], t1_full[2], t1_empty[2],
+    // t2_full[2], t2_empty[2], stats[4], drain
+    static constexpr int NBAR = 2 * kStages + 2 * QBUF + 2 * 4 + kStatSlots + 1;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
     static constexpr int BYTES = OFF_MISC + 16;
     static constexpr int ALLOC = BYTES + 1024;  // slack for 1024-byte alignment
@@ -100,16 +112,65 @@ __device__ __forceinline__ bool wait_phase_cluster(uint32_t bar, uint32_t parity
     }
 }
 
-template <int ROW_BYTES, bool FP8>
+// Online (max, sum 2^(x*c - max*c)) update of one row over NV columns.
+template <int NV>
+__device__ __forceinline__ void row_stats_update(const float* v, int valid, float cl, float& m, float& l)
+{
+    float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+    if (valid >= NV) {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            mx0 = fmaxf(mx0, v[c]);
+            mx1 = fmaxf(mx1, v[c + 1]);
+            mx2 = fmaxf(mx2, v[c + 2]);
+            mx3 = fmaxf(mx3, v[c + 3]);
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            mx0 = fmaxf(mx0, c < valid ? v[c] : -INFINITY);
+            mx1 = fmaxf(mx1, c + 1 < valid ? v[c + 1] : -INFINITY);
+            mx2 = fmaxf(mx2, c + 2 < valid ? v[c + 2] : -INFINITY);
+            mx3 = fmaxf(mx3, c + 3 < valid ? v[c + 3] : -INFINITY);
+        }
+    }
+    const float m_new = fmaxf(m, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)));
+    if (m_new == -INFINITY) return;  // no valid column yet
+    const float mc = m_new * cl;
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    if (valid >= NV) {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            s0 += ex2(fmaf(v[c], cl, -mc));
+            s1 += ex2(fmaf(v[c + 1], cl, -mc));
+            s2 += ex2(fmaf(v[c + 2], cl, -mc));
+            s3 += ex2(fmaf(v[c + 3], cl, -mc));
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            s0 += c < valid ? ex2(fmaf(v[c], cl, -mc)) : 0.f;
+            s1 += c + 1 < valid ? ex2(fmaf(v[c + 1], cl, -mc)) : 0.f;
+            s2 += c + 2 < valid ? ex2(fmaf(v[c + 2], cl, -mc)) : 0.f;
+            s3 += c + 3 < valid ? ex2(fmaf(v[c + 3], cl, -mc)) : 0.f;
+        }
+    }
+    l = l * ex2((m - m_new) * cl) + ((s0 + s1) + (s2 + s3));
+    m = m_new;
+}
+
+template <int ROW_BYTES, bool FP8, int MROWS>
 __global__ void __launch_bounds__(kThreads, 1)
     score_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const ScoreLaunch p)
 {
-    using L = SmemLayout<ROW_BYTES>;
+    using L = SmemLayout<ROW_BYTES, MROWS>;
     constexpr int KSTEPS = ROW_BYTES / 32;                 // one MMA consumes 32 bytes of d
     constexpr int ELEMS_PER_KB = FP8 ? 128 : 64;           // elements in 128 bytes
     constexpr uint32_t FMT = FP8 ? 0u : 1u;
     constexpr int kStages = L::kStages;
+    constexpr int QBUF = L::QBUF;
+    static_assert(kStages >= 3, "ring depth");
     static_assert(L::ALLOC > 116 * 1024, "one CTA per SM");
     static_assert(L::ALLOC <= 227 * 1024, "shared memory per CTA");
 
@@ -127,11 +188,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int N = p.seq_off[b + 1] - n0;
     const int t0 = p.text_off[b];
     const int T = p.text_off[b + 1] - t0;
-    // Uniform for the whole cluster (same request): nothing touched yet.
-    if (N <= 0 || T <= 0 || T > kMaxText) {
-        if (N > 0 && threadIdx.x == 0 && rank == 0) atomicOr(p.err, kErrShape);
+    const bool multi = p.groups > 1;
+    // Uniform for the whole cluster (same request). With several head groups
+    // every CTA must still take its fold ticket, so only shape errors return.
+    if (T > MROWS || (N > 0 && T <= 0)) {
+        if (threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
         return;
     }
+    if (N <= 0) return;
     const int n_tiles = (N + kTileRows - 1) / kTileRows;
     const int tpc = (n_tiles + (int)csize - 1) / (int)csize;
     const int tile_begin = min(n_tiles, (int)rank * tpc);
@@ -142,14 +206,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int hpg = p.heads_per_group;
     const float cl = p.c_log2;
 
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::OFF_BAR);
     const uint32_t bar0 = base + L::OFF_BAR;
     auto BAR = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
-    const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + 2, T1_FULL = Q_EMPTY + 2,
+    const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + QBUF, T1_FULL = Q_EMPTY + QBUF,
               T1_EMPTY = T1_FULL + 2, T2_FULL = T1_EMPTY + 2, T2_EMPTY = T2_FULL + 2, STATS = T2_EMPTY + 2,
-              DRAIN = STATS + 2;
+              DRAIN = STATS + kStatSlots;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
+    volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 8);
     float* acc_s = reinterpret_cast<float*>(smem + L::OFF_ACC);
     float2* stats_s = reinterpret_cast<float2*>(smem + L::OFF_STATS);
     float* b2_s = reinterpret_cast<float*>(smem + L::OFF_B2);
@@ -159,17 +223,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(BAR(K_FULL + s), 1);
             mbar_init(BAR(K_EMPTY + s), 1);
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < QBUF; ++i) {
             mbar_init(BAR(Q_FULL + i), 1);
             mbar_init(BAR(Q_EMPTY + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(BAR(T1_FULL + i), 1);
             mbar_init(BAR(T1_EMPTY + i), 128);
             mbar_init(BAR(T2_FULL + i), 1);
             mbar_init(BAR(T2_EMPTY + i), 128);
-            mbar_init(BAR(STATS + i), csize);
         }
+        for (int i = 0; i < kStatSlots; ++i) mbar_init(BAR(STATS + i), csize);
         mbar_init(BAR(DRAIN), 1);
         *abort_flag = 0;
+        *last_flag = 0;
         fence_mbar_init_cluster();
     }
     if (warp == 0 && lane == 0) {
@@ -185,64 +252,75 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     cluster_sync_all();  // every CTA's barriers exist before any remote arrival
     const uint32_t tmem = *tmem_slot;
-    (void)bars;
-
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
+    // Pipeline step s (0..hpg): pass 1 of head s (s < hpg), then pass 2 of head s-1 (s >= 1).
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0 && mt > 0) {
             uint32_t ks = 0, kph = 0;
             int k_issued[kStages];
-            int q_issued[2] = {0, 0};
+            int q_issued[QBUF];
+            for (int s = 0; s < QBUF; ++s) q_issued[s] = 0;
             for (int s = 0; s < kStages; ++s) k_issued[s] = 0;
             bool ok = true;
-            for (int hi = 0; hi < hpg && ok; ++hi) {
-                const int h = hg * hpg + hi;
-                const int g = h / G;
-                const int qb = hi & 1;
-                if (!wait_phase(BAR(Q_EMPTY + qb), ((hi >> 1) & 1) ^ 1, ctl)) { ok = false; break; }
-                mbar_arrive_expect_tx(BAR(Q_FULL + qb), L::Q_BYTES);
-                const uint32_t qdst = base + L::OFF_Q + qb * L::Q_BYTES;
+            auto load_tiles = [&](int g) {
+                for (int t = tile_begin; t < tile_end && ok; ++t) {
+                    if (!wait_phase(BAR(K_EMPTY + ks), kph ^ 1, ctl)) { ok = false; break; }
+                    mbar_arrive_expect_tx(BAR(K_FULL + ks), L::TILE_BYTES);
+                    const uint32_t kdst = base + L::OFF_K + ks * L::TILE_BYTES;
 #pragma unroll
-                for (int kb = 0; kb < L::KB; ++kb)
-                    tma_load_3d(qdst + kb * kMaxText * 128, &tm_q, BAR(Q_FULL + qb), kb * ELEMS_PER_KB, h, t0);
-                ++q_issued[qb];
-                for (int pass = 0; pass < 2 && ok; ++pass) {
-                    for (int t = tile_begin; t < tile_end; ++t) {
-                        if (!wait_phase(BAR(K_EMPTY + ks), kph ^ 1, ctl)) { ok = false; break; }
-                        mbar_arrive_expect_tx(BAR(K_FULL + ks), L::TILE_BYTES);
-                        const uint32_t kdst = base + L::OFF_K + ks * L::TILE_BYTES;
-#pragma unroll
-                        for (int kb = 0; kb < L::KB; ++kb)
-                            tma_load_3d(kdst + kb * kTileRows * 128, &tm_k, BAR(K_FULL + ks), kb * ELEMS_PER_KB, g,
-                                        n0 + t * kTileRows);
-                        ++k_issued[ks];
-                        if (++ks == kStages) { ks = 0; kph ^= 1; }
-                    }
+                    for (int kb = 0; kb < L::KB; ++kb)
+                        tma_load_3d(kdst + kb * kTileRows * 128, &tm_k, BAR(K_FULL + ks), kb * ELEMS_PER_KB, g,
+                                    n0 + t * kTileRows);
+                    ++k_issued[ks];
+                    if (++ks == kStages) { ks = 0; kph ^= 1; }
                 }
+            };
+            for (int s = 0; s <= hpg && ok; ++s) {
+                if (s < hpg) {
+                    const int h = hg * hpg + s;
+                    const int qb = s % QBUF;
+                    if (!wait_phase(BAR(Q_EMPTY + qb), ((s / QBUF) & 1) ^ 1, ctl)) break;
+                    mbar_arrive_expect_tx(BAR(Q_FULL + qb), L::Q_BYTES);
+                    const uint32_t qdst = base + L::OFF_Q + qb * L::Q_BYTES;
+#pragma unroll
+                    for (int kb = 0; kb < L::KB; ++kb)
+                        tma_load_3d(qdst + kb * MROWS * 128, &tm_q, BAR(Q_FULL + qb), kb * ELEMS_PER_KB, h, t0);
+                    ++q_issued[qb];
+                    load_tiles(h / G);
+                }
+                if (s >= 1 && ok) load_tiles((hg * hpg + s - 1) / G);
             }
-            // drain: the last load of every slot must land before the CTA leaves
+            // drain: the last load of every slot lands before the CTA leaves
+            // (these waits ignore the abort flag)
+            volatile int no_abort = 0;
+            const Ctl drain_ctl{&no_abort, p.err, kWaitBudgetCycles};
             for (int s = 0; s < kStages; ++s)
-                if (k_issued[s] > 0) wait_phase(BAR(K_FULL + s), (uint32_t)(k_issued[s] - 1) & 1u, ctl);
-            for (int s = 0; s < 2; ++s)
-                if (q_issued[s] > 0) wait_phase(BAR(Q_FULL + s), (uint32_t)(q_issued[s] - 1) & 1u, ctl);
+                if (k_issued[s] > 0) wait_phase(BAR(K_FULL + s), (uint32_t)(k_issued[s] - 1) & 1u, drain_ctl);
+            for (int s = 0; s < QBUF; ++s)
+                if (q_issued[s] > 0) wait_phase(BAR(Q_FULL + s), (uint32_t)(q_issued[s] - 1) & 1u, drain_ctl);
         }
         __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             if (mt > 0) {
-                const uint32_t idesc1 = idesc_make(128, 128, FMT);
+                const uint32_t idesc1 = idesc_make(MROWS, 128, FMT);
                 const uint32_t idesc2 = idesc_make(128, (uint32_t)n2, FMT);
                 uint32_t ks = 0, kph = 0, t1i = 0, t2i = 0;
                 bool ok = true;
-                for (int hi = 0; hi < hpg && ok; ++hi) {
-                    const int qb = hi & 1;
-                    if (!wait_phase(BAR(Q_FULL + qb), (hi >> 1) & 1, ctl)) break;
-                    tc_fence_after();
-                    const uint32_t qaddr = base + L::OFF_Q + qb * L::Q_BYTES;
+                for (int s = 0; s <= hpg && ok; ++s) {
                     for (int pass = 0; pass < 2 && ok; ++pass) {
+                        if (pass == 0 && s >= hpg) continue;
+                        if (pass == 1 && s < 1) continue;
+                        const int hs = pass == 0 ? s : s - 1;  // head of this unit
+                        const int qb = hs % QBUF;
+                        if (pass == 0) {
+                            if (!wait_phase(BAR(Q_FULL + qb), (hs / QBUF) & 1, ctl)) { ok = false; break; }
+                            tc_fence_after();
+                        }
+                        const uint32_t qaddr = base + L::OFF_Q + qb * L::Q_BYTES;
                         for (int t = tile_begin; t < tile_end; ++t) {
                             if (!wait_phase(BAR(K_FULL + ks), kph, ctl)) { ok = false; break; }
                             const uint32_t tb = pass == 0 ? (t1i & 1) : (t2i & 1);
@@ -256,9 +334,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                             const uint32_t d = tmem + (pass == 0 ? 0u : 256u) + tb * 128u;
 #pragma unroll
                             for (int st = 0; st < KSTEPS; ++st) {
-                                const uint32_t off = (st >> 2) * (kTileRows * 128) + (st & 3) * 32;
-                                const uint64_t qd = sdesc_k_sw128(qaddr + off);
-                                const uint64_t kd = sdesc_k_sw128(kaddr + off);
+                                const uint32_t koff = (st >> 2) * (kTileRows * 128) + (st & 3) * 32;
+                                const uint32_t qoff = (st >> 2) * (MROWS * 128) + (st & 3) * 32;
+                                const uint64_t qd = sdesc_k_sw128(qaddr + qoff);
+                                const uint64_t kd = sdesc_k_sw128(kaddr + koff);
                                 if (pass == 0) {
                                     if (FP8) mma_f8(d, qd, kd, idesc1, st > 0);
                                     else mma_f16(d, qd, kd, idesc1, st > 0);
@@ -272,137 +351,183 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (pass == 0) ++t1i; else ++t2i;
                             if (++ks == kStages) { ks = 0; kph ^= 1; }
                         }
+                        if (pass == 1 && ok) mma_commit(BAR(Q_EMPTY + qb));  // last reader of Q(hs)
                     }
-                    mma_commit(BAR(Q_EMPTY + qb));
                 }
             }
             // drain: every MMA issued by this thread has completed
             mma_commit(BAR(DRAIN));
-            wait_phase(BAR(DRAIN), 0, ctl);
+            volatile int no_abort = 0;
+            const Ctl drain_ctl{&no_abort, p.err, kWaitBudgetCycles};
+            wait_phase(BAR(DRAIN), 0, drain_ctl);
         }
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        const int quad = warp & 3;
-        const int row = quad * 32 + lane;                     // TMEM lane of this thread
-        const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-        for (int tl = 0; tl < mt; ++tl) acc_s[tl * kTileRows + row] = 0.f;
-        uint32_t t1i = 0, t2i = 0;
         // Control flow here is identical for all 128 threads (named barriers);
-        // after an abort every wait returns at once and the loop runs out.
-        for (int hi = 0; hi < hpg; ++hi) {
-            const int par = hi & 1;
-            // ---- pass 1: online row statistics over this CTA's tiles
-            float m = -INFINITY, l = 0.f;
-            const bool warp_live = quad * 32 < T;
-            for (int t = tile_begin; t < tile_end; ++t) {
-                const uint32_t tb = t1i & 1;
-                wait_phase(BAR(T1_FULL + tb), (t1i >> 1) & 1, ctl);
-                tc_fence_after();
-                float v[128];
-                if (warp_live) {
+        // after an abort every wait returns at once and the steps run out.
+        const int quad = warp & 3;
+        const int et = threadIdx.x - 64;                      // 0..127
+        const int vrow = quad * 32 + lane;                    // pass 2: TMEM lane = visual token in tile
+        const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+        // pass 1 row of this thread: M=128 -> lane; M=64 -> lanes 16q..16q+15, two column halves
+        const int prow = MROWS == 128 ? quad * 32 + lane : quad * 16 + (lane & 15);
+        const int phalf = MROWS == 128 ? 0 : (lane >> 4);
+        const bool p1_live = MROWS == 128 ? (quad * 32 < T) : (quad * 16 < T);
+        for (int tl = 0; tl < mt; ++tl) acc_s[tl * kTileRows + vrow] = 0.f;
+        uint32_t t1i = 0, t2i = 0;
+        for (int s = 0; s <= hpg; ++s) {
+            if (s < hpg) {
+                // ---- pass 1 of head s: online row statistics over this CTA's tiles
+                float m = -INFINITY, l = 0.f;
+                for (int t = tile_begin; t < tile_end; ++t) {
+                    const uint32_t tb = t1i & 1;
+                    wait_phase(BAR(T1_FULL + tb), (t1i >> 1) & 1, ctl);
+                    tc_fence_after();
                     const uint32_t ta = tmem + lane_off + tb * 128u;
-                    tmem_ld32(ta + 0, v);
-                    tmem_ld32(ta + 32, v + 32);
-                    tmem_ld32(ta + 64, v + 64);
-                    tmem_ld32(ta + 96, v + 96);
-                    tmem_wait_ld();
-                }
-                tc_fence_before();
-                mbar_arrive(BAR(T1_EMPTY + tb));
-                ++t1i;
-                if (warp_live) {
-                    const int valid = N - t * kTileRows;
-                    if (valid < kTileRows) {
+                    // 64 columns at a time: M = 64 -> this thread's half of the row;
+                    // M = 128 -> the row's two halves one after the other
+                    constexpr int NH = MROWS == 128 ? 2 : 1;
 #pragma unroll
-                        for (int c = 0; c < 128; ++c)
-                            if (c >= valid) v[c] = -INFINITY;
-                    }
-                    float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
-#pragma unroll
-                    for (int c = 4; c < 128; c += 4) {
-                        mx0 = fmaxf(mx0, v[c]);
-                        mx1 = fmaxf(mx1, v[c + 1]);
-                        mx2 = fmaxf(mx2, v[c + 2]);
-                        mx3 = fmaxf(mx3, v[c + 3]);
-                    }
-                    const float m_new = fmaxf(m, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)));
-                    const float mc = m_new * cl;
-                    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-                    for (int c = 0; c < 128; c += 4) {
-                        s0 += ex2(fmaf(v[c], cl, -mc));
-                        s1 += ex2(fmaf(v[c + 1], cl, -mc));
-                        s2 += ex2(fmaf(v[c + 2], cl, -mc));
-                        s3 += ex2(fmaf(v[c + 3], cl, -mc));
-                    }
-                    l = l * ex2((m - m_new) * cl) + ((s0 + s1) + (s2 + s3));
-                    m = m_new;
-                }
-            }
-            // ---- exchange (m, l) across the cluster
-            stats_s[par * kMaxText + row] = make_float2(m, l);
-            fence_acq_rel_cluster();
-            named_bar_sync(1, 128);
-            if (row == 0) {
-                const uint32_t sb = BAR(STATS + par);
-                for (uint32_t r = 0; r < csize; ++r) mbar_arrive_remote(mapa_shared(sb, r));
-            }
-            wait_phase_cluster(BAR(STATS + par), (hi >> 1) & 1, ctl);
-            {
-                const uint32_t my = base + L::OFF_STATS + (uint32_t)(par * kMaxText + row) * 8u;
-                float M = -INFINITY;
-                for (uint32_t r = 0; r < csize; ++r) M = fmaxf(M, ld_shared_cluster_f2(mapa_shared(my, r)).x);
-                float Lsum = 0.f;
-                for (uint32_t r = 0; r < csize; ++r) {
-                    const float2 st = ld_shared_cluster_f2(mapa_shared(my, r));
-                    if (st.y > 0.f) Lsum += st.y * ex2((st.x - M) * cl);
-                }
-                b2_s[row] = (row < T) ? fmaf(M, cl, __log2f(Lsum)) : INFINITY;
-            }
-            named_bar_sync(1, 128);
-            // ---- pass 2: per-visual-token sums of probabilities
-            for (int t = tile_begin; t < tile_end; ++t) {
-                const uint32_t tb = t2i & 1;
-                wait_phase(BAR(T2_FULL + tb), (t2i >> 1) & 1, ctl);
-                tc_fence_after();
-                float v[128];
-                const uint32_t ta = tmem + lane_off + 256u + tb * 128u;
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    if (k * 32 + 32 <= n2) tmem_ld32(ta + k * 32, v + k * 32);
-                    else if (k * 32 + 16 <= n2) tmem_ld16(ta + k * 32, v + k * 32);
-                }
-                tmem_wait_ld();
-                tc_fence_before();
-                mbar_arrive(BAR(T2_EMPTY + tb));
-                ++t2i;
-                float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    if (k * 16 < n2) {
-#pragma unroll
-                        for (int e = 0; e < 16; e += 4) {
-                            const float4 bb = *reinterpret_cast<const float4*>(b2_s + k * 16 + e);
-                            a0 += ex2(fmaf(v[k * 16 + e], cl, -bb.x));
-                            a1 += ex2(fmaf(v[k * 16 + e + 1], cl, -bb.y));
-                            a2 += ex2(fmaf(v[k * 16 + e + 2], cl, -bb.z));
-                            a3 += ex2(fmaf(v[k * 16 + e + 3], cl, -bb.w));
+                    for (int hh = 0; hh < NH; ++hh) {
+                        float v[64];
+                        if (p1_live) {
+                            if constexpr (MROWS == 128) {
+                                tmem_ld32(ta + hh * 64, v);
+                                tmem_ld32(ta + hh * 64 + 32, v + 32);
+                            } else {
+                                tmem_ld16x2_32(ta + 0, v);
+                                tmem_ld16x2_32(ta + 32, v + 32);
+                            }
+                            tmem_wait_ld();
+                        }
+                        if (hh == NH - 1) {
+                            tc_fence_before();
+                            mbar_arrive(BAR(T1_EMPTY + tb));
+                        }
+                        if (p1_live) {
+                            const int valid = N - t * kTileRows - (MROWS == 128 ? hh : phalf) * 64;
+                            row_stats_update<64>(v, valid, cl, m, l);
                         }
                     }
+                    ++t1i;
                 }
-                acc_s[(t - tile_begin) * kTileRows + row] += (a0 + a1) + (a2 + a3);
+                if (MROWS == 64) {
+                    // merge the two column halves of each row (threads t and t ^ 16)
+                    const float mo = __shfl_xor_sync(0xffffffffu, m, 16);
+                    const float lo = __shfl_xor_sync(0xffffffffu, l, 16);
+                    const float mm = fmaxf(m, mo);
+                    if (mm != -INFINITY) {
+                        l = (l > 0.f ? l * ex2((m - mm) * cl) : 0.f) + (lo > 0.f ? lo * ex2((mo - mm) * cl) : 0.f);
+                        m = mm;
+                    }
+                }
+                // ---- publish (m, l) of head s to the cluster
+                const int slot = s % kStatSlots;
+                if (MROWS == 128 || lane < 16) stats_s[slot * kMaxText + prow] = make_float2(m, l);
+                fence_acq_rel_cluster();
+                named_bar_sync(1, 128);
+                if (et == 0) {
+                    const uint32_t sb = BAR(STATS + slot);
+                    for (uint32_t r = 0; r < csize; ++r) mbar_arrive_remote(mapa_shared(sb, r));
+                }
+            }
+            if (s >= 1) {
+                // ---- merge the cluster's statistics of head s-1
+                const int hs = s - 1;
+                const int slot = hs % kStatSlots;
+                float* b2 = b2_s + (hs & 1) * kMaxText;
+                wait_phase_cluster(BAR(STATS + slot), (uint32_t)(hs / kStatSlots) & 1u, ctl);
+                {
+                    const uint32_t my = base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u;
+                    float M = -INFINITY;
+                    for (uint32_t r = 0; r < csize; ++r) M = fmaxf(M, ld_shared_cluster_f2(mapa_shared(my, r)).x);
+                    float Lsum = 0.f;
+                    for (uint32_t r = 0; r < csize; ++r) {
+                        const float2 st = ld_shared_cluster_f2(mapa_shared(my, r));
+                        if (st.y > 0.f) Lsum += st.y * ex2((st.x - M) * cl);
+                    }
+                    b2[et] = (et < T) ? fmaf(M, cl, __log2f(Lsum)) : INFINITY;
+                }
+                named_bar_sync(1, 128);
+                // ---- pass 2 of head s-1: per-visual-token sums of probabilities
+                for (int t = tile_begin; t < tile_end; ++t) {
+                    const uint32_t tb = t2i & 1;
+                    wait_phase(BAR(T2_FULL + tb), (t2i >> 1) & 1, ctl);
+                    tc_fence_after();
+                    const uint32_t ta = tmem + lane_off + 256u + tb * 128u;
+                    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+                    for (int hh = 0; hh < MROWS / 64; ++hh) {
+                        if (hh * 64 < n2) {
+                            float v[64];
+#pragma unroll
+                            for (int k = 0; k < 2; ++k) {
+                                const int c0 = hh * 64 + k * 32;
+                                if (c0 + 32 <= n2) tmem_ld32(ta + c0, v + k * 32);
+                                else if (c0 + 16 <= n2) tmem_ld16(ta + c0, v + k * 32);
+                            }
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) {
+                                if (hh * 64 + k * 16 < n2) {
+#pragma unroll
+                                    for (int e = 0; e < 16; e += 4) {
+                                        const float4 bb = *reinterpret_cast<const float4*>(b2 + hh * 64 + k * 16 + e);
+                                        a0 += ex2(fmaf(v[k * 16 + e], cl, -bb.x));
+                                        a1 += ex2(fmaf(v[k * 16 + e + 1], cl, -bb.y));
+                                        a2 += ex2(fmaf(v[k * 16 + e + 2], cl, -bb.z));
+                                        a3 += ex2(fmaf(v[k * 16 + e + 3], cl, -bb.w));
+                                    }
+                                }
+                            }
+                        }
+                    }
+                    tc_fence_before();
+                    mbar_arrive(BAR(T2_EMPTY + tb));
+                    ++t2i;
+                    acc_s[(t - tile_begin) * kTileRows + vrow] += (a0 + a1) + (a2 + a3);
+                }
+            }
+        }
+        // ---- results
+        const float denom = (float)p.hq * (float)T;
+        for (int tl = 0; tl < mt; ++tl) {
+            const int j = (tile_begin + tl) * kTileRows + vrow;
+            if (j < N) {
+                const float a = acc_s[tl * kTileRows + vrow];
+                if (!multi) p.out[n0 + j] = a / denom;
+                else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
+            }
+        }
+        if (multi) {
+            // last CTA of the request (over all head groups) adds the partial rows
+            __threadfence();
+            named_bar_sync(1, 128);
+            if (et == 0) {
+                const int ticket = atomicAdd(p.counters + b, 1);
+                if (ticket == p.ctas_per_request - 1) {
+                    *last_flag = 1;
+                    p.counters[b] = 0;  // ready for the next launch
+                }
             }
             named_bar_sync(1, 128);
-        }
-        if (!*abort_flag) {
-            const float denom = (float)p.hq * (float)T;
-            for (int tl = 0; tl < mt; ++tl) {
-                const int j = (tile_begin + tl) * kTileRows + row;
-                if (j < N) {
-                    const float a = acc_s[tl * kTileRows + row];
-                    if (p.groups == 1) p.out[n0 + j] = a / denom;
-                    else p.out[(int64_t)hg * p.total_vis + n0 + j] = a;
+            if (*last_flag) {
+                __threadfence();
+                for (int j = et; j < N; j += 128) {
+                    // groups are added in index order; loads issued 8 at a time
+                    const float* src = p.partials + n0 + j;
+                    float sum = 0.f;
+                    int g = 0;
+                    for (; g + 8 <= p.groups; g += 8) {
+                        float x[8];
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) x[u] = __ldcg(src + (int64_t)(g + u) * p.total_vis);
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) sum += x[u];
+                    }
+                    for (; g < p.groups; ++g) sum += __ldcg(src + (int64_t)g * p.total_vis);
+                    p.out[n0 + j] = sum / denom;
                 }
             }
         }
@@ -418,28 +543,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     cluster_sync_all();  // peers are done reading this CTA's statistics
 }
 
-// scores[j] = (sum over head groups of partial[g][j]) / (Hq * T_b), fixed order
-__global__ void fold_groups_kernel(const float* __restrict__ partials, int groups, int64_t total_vis,
-                                   const int32_t* __restrict__ seq_off, const int32_t* __restrict__ text_off,
-                                   int hq, float* __restrict__ scores)
-{
-    const int b = blockIdx.y;
-    const int n0 = seq_off[b], N = seq_off[b + 1] - n0;
-    const int T = text_off[b + 1] - text_off[b];
-    const float denom = (float)hq * (float)T;
-    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < N; j += gridDim.x * blockDim.x) {
-        float s = 0.f;
-        for (int g = 0; g < groups; ++g) s += partials[(int64_t)g * total_vis + n0 + j];
-        scores[n0 + j] = s / denom;
-    }
-}
-
-template <int ROW_BYTES, bool FP8>
+template <int ROW_BYTES, bool FP8, int MROWS>
 cudaError_t launch_variant(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
                            const ScorePlan& plan, int batch, cudaStream_t stream)
 {
-    auto kern = score_tc_kernel<ROW_BYTES, FP8>;
-    const int smem = SmemLayout<ROW_BYTES>::ALLOC;
+    auto kern = score_tc_kernel<ROW_BYTES, FP8, MROWS>;
+    const int smem = SmemLayout<ROW_BYTES, MROWS>::ALLOC;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     if (plan.cluster > 8) {
@@ -469,50 +578,76 @@ bool score_shape_supported(int head_dim, bool fp8)
     return head_dim == 64 || head_dim == 128;
 }
 
-size_t score_smem_bytes(int row_bytes)
+// CTAs of one cluster size that run at once with one CTA per SM (GPC packing
+// on a 152-SM GB300: 1, 2 -> 152; 4 -> 144; 8 -> 120; 16 -> 112).
+static int cluster_capacity(int c, int num_sms)
 {
-    return row_bytes == 256 ? SmemLayout<256>::ALLOC : SmemLayout<128>::ALLOC;
+    switch (c) {
+    case 1:
+    case 2: return num_sms;
+    case 4: return num_sms * 144 / 152;
+    case 8: return num_sms * 120 / 152;
+    default: return num_sms * 112 / 152;
+    }
 }
 
-ScorePlan plan_score(int batch, int max_tiles, int hq, int num_sms)
+ScorePlan plan_score(int batch, int max_tiles, int hq, int hkv, int tile_bytes, int num_sms)
 {
-    ScorePlan pl{1, 1, 1};
-    if (max_tiles <= 0) return pl;
-    int tpc = (max_tiles + 7) / 8;
-    int c = (max_tiles + tpc - 1) / tpc;
-    if (tpc > kMaxTilesPerCta) {
-        tpc = (max_tiles + kMaxCluster - 1) / kMaxCluster;
-        c = (max_tiles + tpc - 1) / tpc;
+    ScorePlan best{1, 1, 1};
+    if (max_tiles <= 0) return best;
+    double best_cost = 1e300;
+    const int G = hq / hkv;
+    for (int pass = 0; pass < 2 && best_cost >= 1e299; ++pass) {
+        for (int c = 1; c <= kMaxCluster; c *= 2) {
+            const int tpc = (max_tiles + c - 1) / c;
+            if (tpc > kMaxTilesPerCta) continue;
+            if (c > 1 && (c / 2) >= max_tiles) break;  // idle ranks only
+            const int cap = cluster_capacity(c, num_sms);
+            for (int g = 1; g <= hq; ++g) {
+                if (hq % g) continue;
+                const long long ctas = (long long)batch * c * g;
+                const long long waves = (ctas + cap - 1) / cap;
+                const int hpg = hq / g;
+                // L2 window of the pass-2 re-read: while a CTA streams up to two
+                // slices (pass 1 of the next head, rest of the current one) the
+                // tiles it re-reads must survive in L2. Groups that split a GQA
+                // key head share its tiles.
+                const long long active = ctas < cap ? ctas : cap;
+                const int share = hpg >= G ? 1 : G / hpg;
+                const double window = 2.0 * tpc * tile_bytes * (double)active / share;
+                if (pass == 0 && window > 80.0 * 1024 * 1024) continue;
+                // per CTA: one tile-head of work per tile and head, plus a fixed
+                // launch / pipeline fill cost of about 6 tile-heads and a cluster
+                // exchange of about 1 tile-head per head; a fold when g > 1
+                const double per_cta = (double)tpc * hpg + 6.0 + (c > 1 ? 1.0 : 0.25) * hpg + (g > 1 ? 2.0 : 0.0);
+                const double cost = (double)waves * per_cta;
+                if (cost < best_cost - 1e-9) {
+                    best_cost = cost;
+                    best = ScorePlan{c, tpc, g};
+                }
+            }
+        }
     }
-    pl.cluster = c;
-    pl.tiles_per_cta = tpc;
-    int groups = hq;
-    for (int g = 1; g <= hq; ++g) {
-        if (hq % g) continue;
-        if ((long long)batch * c * g >= num_sms) { groups = g; break; }
-    }
-    pl.groups = groups;
-    return pl;
+    return best;
 }
 
 cudaError_t launch_score(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
-                         const ScorePlan& plan, int batch, int row_bytes, bool fp8, float* partials,
-                         float* scores, int max_n, cudaStream_t stream)
+                         const ScorePlan& plan, int batch, int row_bytes, bool fp8, int mrows, cudaStream_t stream)
 {
     ScoreLaunch q = p;
     q.groups = plan.groups;
     q.heads_per_group = p.hq / plan.groups;
-    q.out = plan.groups == 1 ? scores : partials;
-    cudaError_t e;
-    if (fp8) e = launch_variant<128, true>(tm_q, tm_k, q, plan, batch, stream);
-    else if (row_bytes == 256) e = launch_variant<256, false>(tm_q, tm_k, q, plan, batch, stream);
-    else e = launch_variant<128, false>(tm_q, tm_k, q, plan, batch, stream);
-    if (e != cudaSuccess || plan.groups == 1) return e;
-    const int threads = 256;
-    const int gx = (max_n + threads - 1) / threads;
-    fold_groups_kernel<<<dim3(gx > 0 ? gx : 1, batch), threads, 0, stream>>>(partials, plan.groups, p.total_vis,
-                                                                              p.seq_off, p.text_off, p.hq, scores);
-    return cudaGetLastError();
+    q.ctas_per_request = plan.cluster * plan.groups;
+    if (fp8) {
+        return mrows == 64 ? launch_variant<128, true, 64>(tm_q, tm_k, q, plan, batch, stream)
+                           : launch_variant<128, true, 128>(tm_q, tm_k, q, plan, batch, stream);
+    }
+    if (row_bytes == 256) {
+        return mrows == 64 ? launch_variant<256, false, 64>(tm_q, tm_k, q, plan, batch, stream)
+                           : launch_variant<256, false, 128>(tm_q, tm_k, q, plan, batch, stream);
+    }
+    return mrows == 64 ? launch_variant<128, false, 64>(tm_q, tm_k, q, plan, batch, stream)
+                       : launch_variant<128, false, 128>(tm_q, tm_k, q, plan, batch, stream);
 }
 
 }  // namespace lvs
