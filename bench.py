@@ -305,7 +305,8 @@ def run_ours(args):
     if step_bytes < 2 * l2:
         flush = torch.empty(max(8 * l2, 1 << 30) // 4, dtype=torch.int32, device=dev)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
-    launches_per_step = 3 + (1 if sel_groups(w, dev) > 1 else 0)
+    plan = sel.score_plan(to_h, so_h)
+    launches_per_step = 3  # score (fold inside), top-k, gather
 
     if world > 1:
         dist.barrier()
@@ -352,13 +353,13 @@ def run_ours(args):
         achieved = alg["score_bytes"] / (score_us * 1e-6) / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
                 "frac": achieved / pk["hbm_gbs"], "traffic": committed_traffic(w.name),
-                "kernel": "score (score_tc_kernel" + (" + fold_groups_kernel)" if launches_per_step > 3 else ")"),
+                "kernel": select.KERNELS.get(plan[0], "score"),
                 "algorithmic_bytes_per_launch": alg["score_bytes"], "peak_source": pk["source"] + " (burst copy)"}
     else:
         achieved = alg["score_flops"] / (score_us * 1e-6) / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
                 "frac": achieved / pk["bf16_tflops"], "traffic": committed_traffic(w.name),
-                "kernel": "score", "algorithmic_flops_per_launch": alg["score_flops"],
+                "kernel": select.KERNELS.get(plan[0], "score"), "algorithmic_flops_per_launch": alg["score_flops"],
                 "peak_source": pk["source"] + " (burst cuBLAS bf16)"}
 
     # end to end through the public API with host buffers
@@ -380,7 +381,9 @@ def run_ours(args):
                        "kept_tokens": total_kept, "gather": list(w.gather),
                        "l2": ("flushed between timed steps (write of %d MB)" % (flush.numel() * 4 >> 20))
                        if flush is not None else "inputs larger than L2, no flush",
-                       "parallelism": f"replicas x{world}, one batch per GPU, no collective"},
+                       "parallelism": f"replicas x{world}, one batch per GPU, no collective",
+                       "score_launch": {"kernel": select.KERNELS.get(plan[0]), "cluster": plan[1],
+                                        "tiles_per_cta": plan[2], "head_groups": plan[3]}},
             "stages_p50_us": stage_us,
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches_per_step * steps, "clocks": clocks,
@@ -391,22 +394,6 @@ def run_ours(args):
         dist.destroy_process_group()
     sel.close()
     return 0
-
-
-def sel_groups(w, dev):
-    """Head groups the score launch uses (mirrors the library's plan) to count launches."""
-    import torch
-    sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    max_tiles = max((n + 127) // 128 for n in w.n_vis)
-    tpc = (max_tiles + 7) // 8
-    c = (max_tiles + tpc - 1) // tpc
-    if tpc > 32:
-        tpc = (max_tiles + 15) // 16
-        c = (max_tiles + tpc - 1) // tpc
-    for g in range(1, w.hq + 1):
-        if w.hq % g == 0 and w.batch * c * g >= sms:
-            return g
-    return w.hq
 
 
 def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept):

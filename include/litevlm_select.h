@@ -67,6 +67,11 @@ typedef enum {
     LITEVLM_FP8_E4M3 = 1  /* q and k are OCP e4m3 codes with one float scale per tensor */
 } litevlm_dtype_t;
 
+/* Score-kernel selection (litevlm_select_config_t.flags). By default the
+ * library picks the kernel and launch shape from the batch's sizes. */
+#define LITEVLM_FLAG_SCORE_REREAD 1   /* always use the kernel that streams K twice per head */
+#define LITEVLM_FLAG_SCORE_RESIDENT 2 /* use the TMEM-resident kernel whenever the shapes allow it */
+
 typedef struct {
     int32_t max_batch;         /* largest batch any call will pass */
     int64_t max_total_visual;  /* largest sum_b N_b */
@@ -75,7 +80,7 @@ typedef struct {
     int32_t num_kv_heads;      /* Hkv, Hq % Hkv == 0 */
     int32_t head_dim;          /* d: 64 or 128 for bf16, 128 for e4m3 */
     litevlm_dtype_t qk_dtype;
-    int32_t flags;             /* reserved, must be 0 */
+    int32_t flags;             /* 0, LITEVLM_FLAG_SCORE_REREAD or LITEVLM_FLAG_SCORE_RESIDENT */
 } litevlm_select_config_t;
 
 typedef struct litevlm_select* litevlm_select_t;
@@ -85,7 +90,7 @@ typedef struct litevlm_select* litevlm_select_t;
  * (partial-score buffer, error word). Limits: T_b <= 128 text tokens per request,
  * N_b <= 65536 visual tokens per request (both checked per call).
  * Errors: INVALID_ARG for a NULL pointer or an inconsistent config (non-positive
- * sizes, Hq % Hkv != 0, flags != 0); UNSUPPORTED for a head_dim / dtype pair
+ * sizes, Hq % Hkv != 0, unknown flags); UNSUPPORTED for a head_dim / dtype pair
  * without a kernel; CUDA when the device cannot be used. *out is NULL on error.
  */
 litevlm_status_t litevlm_select_create(const litevlm_select_config_t* config, litevlm_select_t* out);
@@ -165,6 +170,17 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t handle, int64_t total_k
                                         int64_t src_rows, int32_t num_tensors,
                                         const void* const* src, void* const* dst, const int64_t* row_bytes,
                                         litevlm_stream_t stream);
+
+/*
+ * Launch shape litevlm_select_score would use for this batch (host only, no
+ * device work; the occupancy of a kernel variant is queried once per handle).
+ * plan[0] = kernel (1: K re-read per pass, 2: pass-2 products resident in
+ * tensor memory), plan[1] = CTAs per thread-block cluster, plan[2] = 128-token
+ * tiles per CTA, plan[3] = query-head groups (grid y). plan holds 4 int32.
+ * Errors as for litevlm_select_score's host-side checks.
+ */
+litevlm_status_t litevlm_select_score_plan(litevlm_select_t handle, int32_t batch, const int32_t* text_offsets_h,
+                                           const int32_t* seq_offsets_h, int32_t* plan);
 
 /*
  * Synchronises `stream`, then reads and clears the handle's device error word.

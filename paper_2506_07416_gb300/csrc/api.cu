@@ -19,9 +19,10 @@ struct litevlm_select {
     int device = 0;
     int num_sms = 0;
     float* partials = nullptr;  // [Hq][max_total_visual]: per-head-group partial scores
-    int32_t* counters = nullptr;  // [max_batch]: fold tickets of the score kernel
+    int32_t* counters = nullptr;  // fold tickets of the score kernels, one per 128-token tile
     int32_t* err_d = nullptr;   // device error word (bits lvs::kErr*)
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    int res_capacity[2][17];  // resident score kernel: CTAs at once per cluster size, by pass-1 rows (64/128); -1 unknown
     std::string last_error;
 };
 
@@ -86,6 +87,60 @@ litevlm_status_t encode_rows_map(litevlm_select_t h, CUtensorMap* map, const voi
     return LITEVLM_OK;
 }
 
+struct ScoreChoice {
+    bool resident;
+    lvs::ScorePlan plan;
+};
+
+// Picks the score kernel and its launch shape. Cost unit: one tile-head of
+// epilogue work; a CTA also pays a fixed ~6 units (launch, TMEM, pipeline
+// fill) and ~1 unit per head for the cluster exchange; waves of CTAs are
+// counted from the cluster occupancy of the kernel. The re-read kernel streams
+// every K tile twice, so its cost is weighted by 1.6.
+ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, int max_tiles, int max_t, int row_bytes, bool fp8)
+{
+    const litevlm_select_config_t& c = h->cfg;
+    const int hq = c.num_q_heads, G = c.num_q_heads / c.num_kv_heads;
+    const int mrows = max_t <= 64 ? 64 : 128;
+    const int slot_cols = (max_t + 15) & ~15;
+    const int R = lvs::res_max_tiles(slot_cols);
+    const int cmax = lvs::res_max_cluster(row_bytes, slot_cols);
+    ScoreChoice best{false, lvs::plan_score(batch, max_tiles, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, h->num_sms)};
+    double best_cost = 1e300;
+    {
+        const lvs::ScorePlan& pl = best.plan;
+        const int hpg = hq / pl.groups;
+        int cap = pl.cluster <= 2 ? h->num_sms : (pl.cluster <= 4 ? h->num_sms * 144 / 152 : h->num_sms * 112 / 152);
+        const long long ctas = (long long)batch * pl.cluster * pl.groups;
+        const long long waves = (ctas + cap - 1) / cap;
+        best_cost = 1.6 * waves * ((double)pl.tiles_per_cta * hpg + 6.0 + hpg + (pl.groups > 1 ? 2.0 : 0.0));
+    }
+    if (c.flags == LITEVLM_FLAG_SCORE_REREAD) return best;
+    if (c.flags == LITEVLM_FLAG_SCORE_RESIDENT) best_cost = 1e300;
+    for (int cl = 1; cl <= cmax; ++cl) {
+        const int tpc = (max_tiles + cl - 1) / cl;
+        if (tpc > R) continue;
+        if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;  // an idle rank
+        int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
+        if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
+        if (cap <= 0) continue;
+        for (int g = 1; g <= hq; ++g) {
+            if (hq % g) continue;
+            const int hpg = hq / g;
+            const long long ctas = (long long)batch * cl * g;
+            const long long waves = (ctas + cap - 1) / cap;
+            const double per = (double)tpc * hpg + 6.0 + (cl > 1 ? 1.0 : 0.25) * hpg + (g > 1 ? 2.0 : 0.0);
+            const double cost = (double)waves * per;
+            if (cost < best_cost - 1e-9) {
+                best_cost = cost;
+                best = ScoreChoice{true, lvs::ScorePlan{cl, tpc, g}};
+            }
+        }
+    }
+    (void)G;
+    return best;
+}
+
 }  // namespace
 
 extern "C" {
@@ -123,7 +178,8 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
     if (c->qk_dtype != LITEVLM_BF16 && c->qk_dtype != LITEVLM_FP8_E4M3)
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "qk_dtype must be LITEVLM_BF16 or LITEVLM_FP8_E4M3");
-    if (c->flags != 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "flags must be 0");
+    if (c->flags != 0 && c->flags != LITEVLM_FLAG_SCORE_REREAD && c->flags != LITEVLM_FLAG_SCORE_RESIDENT)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "flags must be 0 or one LITEVLM_FLAG_SCORE_* value");
     if (c->head_dim <= 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "head_dim must be > 0");
     if (!lvs::score_shape_supported(c->head_dim, c->qk_dtype == LITEVLM_FP8_E4M3))
         return fail(nullptr, LITEVLM_ERR_UNSUPPORTED,
@@ -132,6 +188,8 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
     litevlm_select* h = new (std::nothrow) litevlm_select();
     if (!h) return fail(nullptr, LITEVLM_ERR_CUDA, "out of host memory");
     h->cfg = *c;
+    for (auto& row : h->res_capacity)
+        for (int& v : row) v = -1;
     cudaError_t e = cudaGetDevice(&h->device);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
     if (e == cudaSuccess) {
@@ -155,8 +213,10 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
     if (e == cudaSuccess) e = cudaMemset(h->err_d, 0, sizeof(int32_t));
     if (e == cudaSuccess && c->num_q_heads > 1)
         e = cudaMalloc(&h->partials, sizeof(float) * (size_t)c->num_q_heads * (size_t)c->max_total_visual);
-    if (e == cudaSuccess) e = cudaMalloc(&h->counters, sizeof(int32_t) * (size_t)c->max_batch);
-    if (e == cudaSuccess) e = cudaMemset(h->counters, 0, sizeof(int32_t) * (size_t)c->max_batch);
+    // one fold ticket per 128-token tile: index floor(n0 / 128) + t + b < total / 128 + 2 * batch + 1
+    const size_t n_counters = (size_t)(c->max_total_visual / lvs::kTileRows) + 2 * (size_t)c->max_batch + 2;
+    if (e == cudaSuccess) e = cudaMalloc(&h->counters, sizeof(int32_t) * n_counters);
+    if (e == cudaSuccess) e = cudaMemset(h->counters, 0, sizeof(int32_t) * n_counters);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         const std::string msg = std::string("create: ") + cudaGetErrorString(e);
@@ -181,25 +241,23 @@ litevlm_status_t litevlm_select_destroy(litevlm_select_t h)
     return LITEVLM_OK;
 }
 
-litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const void* q_text,
-                                      const int32_t* text_offsets_d, const int32_t* text_offsets_h,
-                                      const void* k_vis, const int32_t* seq_offsets_d,
-                                      const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
-                                      litevlm_stream_t stream)
+namespace {
+struct ScoreShape {
+    int64_t tot_n = 0, tot_t = 0;
+    int max_tiles = 0, max_n = 0, max_t = 0;
+};
+
+litevlm_status_t check_score_shape(litevlm_select_t h, int32_t batch, const int32_t* text_offsets_h,
+                                   const int32_t* seq_offsets_h, ScoreShape* sh)
 {
-    if (!h) return LITEVLM_ERR_INVALID_ARG;
-    h->last_error.clear();
     const litevlm_select_config_t& c = h->cfg;
-    const bool fp8 = c.qk_dtype == LITEVLM_FP8_E4M3;
     if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
     if (batch > c.max_batch) return fail(h, LITEVLM_ERR_WORKSPACE, "batch exceeds max_batch");
     if (batch == 0) return LITEVLM_OK;
-    int64_t tot_n = 0, tot_t = 0;
-    litevlm_status_t s = check_offsets(h, seq_offsets_h, batch, c.max_total_visual, "seq_offsets", &tot_n);
+    litevlm_status_t s = check_offsets(h, seq_offsets_h, batch, c.max_total_visual, "seq_offsets", &sh->tot_n);
     if (s != LITEVLM_OK) return s;
-    s = check_offsets(h, text_offsets_h, batch, c.max_total_text, "text_offsets", &tot_t);
+    s = check_offsets(h, text_offsets_h, batch, c.max_total_text, "text_offsets", &sh->tot_t);
     if (s != LITEVLM_OK) return s;
-    int max_tiles = 0, max_n = 0, max_t = 0;
     for (int32_t b = 0; b < batch; ++b) {
         const int32_t n = seq_offsets_h[b + 1] - seq_offsets_h[b];
         const int32_t t = text_offsets_h[b + 1] - text_offsets_h[b];
@@ -213,10 +271,49 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
             return fail(h, LITEVLM_ERR_UNSUPPORTED,
                         "request " + std::to_string(b) + " has more than 65536 visual tokens");
         const int tiles = (n + lvs::kTileRows - 1) / lvs::kTileRows;
-        if (tiles > max_tiles) max_tiles = tiles;
-        if (n > max_n) max_n = n;
-        if (n > 0 && t > max_t) max_t = t;
+        if (tiles > sh->max_tiles) sh->max_tiles = tiles;
+        if (n > sh->max_n) sh->max_n = n;
+        if (n > 0 && t > sh->max_t) sh->max_t = t;
     }
+    return LITEVLM_OK;
+}
+}  // namespace
+
+litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, const int32_t* text_offsets_h,
+                                           const int32_t* seq_offsets_h, int32_t* plan)
+{
+    if (!h || !plan) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    ScoreShape sh;
+    const litevlm_status_t s = check_score_shape(h, batch, text_offsets_h, seq_offsets_h, &sh);
+    if (s != LITEVLM_OK) return s;
+    plan[0] = plan[1] = plan[2] = plan[3] = 0;
+    if (batch == 0 || sh.tot_n == 0) return LITEVLM_OK;
+    const bool fp8 = h->cfg.qk_dtype == LITEVLM_FP8_E4M3;
+    const ScoreChoice ch = choose_score_kernel(h, batch, sh.max_tiles, sh.max_t, h->cfg.head_dim * (fp8 ? 1 : 2), fp8);
+    plan[0] = ch.resident ? 2 : 1;
+    plan[1] = ch.plan.cluster;
+    plan[2] = ch.plan.tiles_per_cta;
+    plan[3] = ch.plan.groups;
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const void* q_text,
+                                      const int32_t* text_offsets_d, const int32_t* text_offsets_h,
+                                      const void* k_vis, const int32_t* seq_offsets_d,
+                                      const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
+                                      litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    const litevlm_select_config_t& c = h->cfg;
+    const bool fp8 = c.qk_dtype == LITEVLM_FP8_E4M3;
+    ScoreShape sh;
+    litevlm_status_t s = check_score_shape(h, batch, text_offsets_h, seq_offsets_h, &sh);
+    if (s != LITEVLM_OK) return s;
+    if (batch == 0) return LITEVLM_OK;
+    const int64_t tot_n = sh.tot_n, tot_t = sh.tot_t;
+    const int max_tiles = sh.max_tiles, max_t = sh.max_t;
     if (tot_n == 0) return LITEVLM_OK;
     if (!q_text || !k_vis || !scores || !text_offsets_d || !seq_offsets_d)
         return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
@@ -229,8 +326,8 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
         return fail(h, LITEVLM_ERR_INVALID_ARG, "q_scale and k_scale must be 1 for bf16 inputs");
     }
     const int row_bytes = c.head_dim * (fp8 ? 1 : 2);
-    const lvs::ScorePlan plan = lvs::plan_score(batch, max_tiles, c.num_q_heads, c.num_kv_heads,
-                                                lvs::kTileRows * row_bytes, h->num_sms);
+    const ScoreChoice choice = choose_score_kernel(h, batch, max_tiles, max_t, row_bytes, fp8);
+    const lvs::ScorePlan& plan = choice.plan;
     if (plan.tiles_per_cta > lvs::kMaxTilesPerCta)
         return fail(h, LITEVLM_ERR_UNSUPPORTED, "request too long for one cluster");
     const int mrows = max_t <= 64 ? 64 : 128;  // text rows of the pass-1 MMA
@@ -253,7 +350,11 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
     p.hkv = c.num_kv_heads;
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
     p.wait_budget = lvs::kWaitBudgetCycles;
-    const cudaError_t e = lvs::launch_score(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream);
+    p.slot_cols = (max_t + 15) & ~15;
+    const cudaError_t e =
+        choice.resident
+            ? lvs::launch_score_resident(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream)
+            : lvs::launch_score(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "score launch");
     return LITEVLM_OK;
 }

@@ -25,13 +25,14 @@ struct ScoreLaunch {
     const int32_t* text_off;  // device [batch+1]
     float* out;               // scores [sum N]
     float* partials;          // [groups][sum N] when groups > 1 (workspace)
-    int32_t* counters;        // [batch] fold tickets, zero between launches (workspace)
+    int32_t* counters;        // one fold ticket per 128-token tile, zero between launches (workspace)
     int32_t* err;
     int64_t total_vis;        // partial-row stride
     int32_t hq, hkv;
     int32_t heads_per_group;
     int32_t groups;
     int32_t ctas_per_request; // cluster size * groups
+    int32_t slot_cols;        // resident kernel: TMEM columns per pass-2 slot (T rounded up to 16, max over batch)
     float c_log2;             // q_scale * k_scale / sqrt(d) * log2(e)
     long long wait_budget;
 };
@@ -47,6 +48,14 @@ ScorePlan plan_score(int batch, int max_tiles, int hq, int hkv, int tile_bytes, 
 cudaError_t launch_score(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
                          const ScorePlan& plan, int batch, int row_bytes, bool fp8, int mrows, cudaStream_t stream);
 bool score_shape_supported(int head_dim, bool fp8);
+
+// score_res.cu (one contraction per K tile and head, logits resident in TMEM)
+int res_max_tiles(int slot_cols);                  // tiles per CTA that fit in tensor memory
+int res_max_cluster(int row_bytes, int slot_cols); // cluster size limit of the statistics buffer
+int res_cluster_capacity(int row_bytes, bool fp8, int mrows, int cluster);
+cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
+                                  const ScorePlan& plan, int batch, int row_bytes, bool fp8, int mrows,
+                                  cudaStream_t stream);
 
 // topk.cu
 cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,

@@ -1,0 +1,161 @@
+// Pipeline helpers shared by the score kernels: bounded mbarrier waits and
+// the online row-statistics update of the softmax normaliser.
+#pragma once
+
+#include <math.h>
+#include <stdint.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace lvs {
+
+struct Ctl {
+    volatile int* abort;
+    int32_t* err;
+    long long budget;
+};
+
+__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, const Ctl& c)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*c.abort) return false;
+        if (clock64() - t0 > c.budget) {
+            *c.abort = 1;
+            atomicOr(c.err, kErrTimeout);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ bool wait_phase_cluster(uint32_t bar, uint32_t parity, const Ctl& c)
+{
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    const long long t0 = clock64();
+    for (;;) {
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (*c.abort) return false;
+        if (clock64() - t0 > c.budget) {
+            *c.abort = 1;
+            atomicOr(c.err, kErrTimeout);
+            return false;
+        }
+    }
+}
+
+// Online (max, sum 2^(x*c - max*c)) update of one row over NV columns.
+template <int NV>
+__device__ __forceinline__ void row_stats_update(const float* v, int valid, float cl, float& m, float& l)
+{
+    float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+    if (valid >= NV) {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            mx0 = fmaxf(mx0, v[c]);
+            mx1 = fmaxf(mx1, v[c + 1]);
+            mx2 = fmaxf(mx2, v[c + 2]);
+            mx3 = fmaxf(mx3, v[c + 3]);
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            mx0 = fmaxf(mx0, c < valid ? v[c] : -INFINITY);
+            mx1 = fmaxf(mx1, c + 1 < valid ? v[c + 1] : -INFINITY);
+            mx2 = fmaxf(mx2, c + 2 < valid ? v[c + 2] : -INFINITY);
+            mx3 = fmaxf(mx3, c + 3 < valid ? v[c + 3] : -INFINITY);
+        }
+    }
+    const float m_new = fmaxf(m, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)));
+    if (m_new == -INFINITY) return;  // no valid column yet
+    const float mc = m_new * cl;
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    if (valid >= NV) {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            s0 += ex2(fmaf(v[c], cl, -mc));
+            s1 += ex2(fmaf(v[c + 1], cl, -mc));
+            s2 += ex2(fmaf(v[c + 2], cl, -mc));
+            s3 += ex2(fmaf(v[c + 3], cl, -mc));
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < NV; c += 4) {
+            s0 += c < valid ? ex2(fmaf(v[c], cl, -mc)) : 0.f;
+            s1 += c + 1 < valid ? ex2(fmaf(v[c + 1], cl, -mc)) : 0.f;
+            s2 += c + 2 < valid ? ex2(fmaf(v[c + 2], cl, -mc)) : 0.f;
+            s3 += c + 3 < valid ? ex2(fmaf(v[c + 3], cl, -mc)) : 0.f;
+        }
+    }
+    l = l * ex2((m - m_new) * cl) + ((s0 + s1) + (s2 + s3));
+    m = m_new;
+}
+
+// Merges the (max, sum) partials of one row from every CTA of the cluster in
+// rank order and returns b = M * c + log2(L). All remote loads are issued
+// before any is used, so their latencies overlap.
+__device__ __forceinline__ float merge_cluster_row(uint32_t my_addr, uint32_t csize, float cl)
+{
+    float2 st[kMaxCluster];
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r)
+        if (r < (int)csize) st[r] = ld_shared_cluster_f2(mapa_shared(my_addr, (uint32_t)r));
+    float M = -INFINITY;
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r)
+        if (r < (int)csize) M = fmaxf(M, st[r].x);
+    float L = 0.f;
+#pragma unroll
+    for (int r = 0; r < kMaxCluster; ++r)
+        if (r < (int)csize && st[r].y > 0.f) L += st[r].y * ex2((st[r].x - M) * cl);
+    return fmaf(M, cl, __log2f(L));
+}
+
+// Ticket slot of tile t of the request starting at row n0 (request b): unique
+// over the batch because floor((n0 + N) / 128) - floor(n0 / 128) >= tiles - 1.
+__device__ __forceinline__ int fold_ticket_index(int b, int n0, int t) { return n0 / kTileRows + t + b; }
+
+// After a CTA wrote its partial rows (head group hg) for tiles [tile_begin,
+// tile_begin + mt): take one ticket per tile; the last of the `groups` CTAs
+// that own a tile adds the group partials of that tile in index order and
+// writes the scores. `nthreads` threads (ids 0..nthreads-1, synchronised by
+// named barrier `bar_id`) take part; `flags` is shared memory for mt ints.
+__device__ __forceinline__ void fold_tiles(const ScoreLaunch& p, int b, int n0, int N, int T, int tile_begin,
+                                           int mt, int tid, int nthreads, uint32_t bar_id, volatile int* flags)
+{
+    __threadfence();
+    named_bar_sync(bar_id, nthreads);
+    for (int tl = tid; tl < mt; tl += nthreads) {
+        int* c = p.counters + fold_ticket_index(b, n0, tile_begin + tl);
+        const int ticket = atomicAdd(c, 1);
+        const int last = ticket == p.groups - 1;
+        if (last) *c = 0;  // ready for the next launch
+        flags[tl] = last;
+    }
+    named_bar_sync(bar_id, nthreads);
+    __threadfence();
+    const float denom = (float)p.hq * (float)T;
+    for (int tl = 0; tl < mt; ++tl) {
+        if (!flags[tl]) continue;
+        for (int r = tid; r < kTileRows; r += nthreads) {
+            const int j = (tile_begin + tl) * kTileRows + r;
+            if (j >= N) break;
+            const float* src = p.partials + n0 + j;
+            float sum = 0.f;
+            int g = 0;
+            for (; g + 8 <= p.groups; g += 8) {
+                float x[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) x[q] = __ldcg(src + (int64_t)(g + q) * p.total_vis);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) sum += x[q];
+            }
+            for (; g < p.groups; ++g) sum += __ldcg(src + (int64_t)g * p.total_vis);
+            p.out[n0 + j] = sum / denom;
+        }
+    }
+}
+
+}  // namespace lvs

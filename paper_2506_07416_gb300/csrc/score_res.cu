@@ -1,0 +1,592 @@
+// Visual-token importance scores, TMEM-resident variant (sm_103a tcgen05).
+//
+// Same result as score_tc.cu (Design section, Token Selection Module:
+// score[j] = 1/(Hq*T) * sum_h sum_i softmax_j(q_i . k_j / sqrt(d))), for the
+// common case where one head's logits for all of a CTA's tiles fit in tensor
+// memory (T rounded up to 16, times the CTA's tiles, at most 512 columns).
+//
+// One tensor-core contraction per K tile and head:
+//     S^T = K_tile * Q_h^T   (M = 128 visual rows, N = T rounded up to 16, K = d)
+// into a TMEM slot that stays resident for the whole head. Visual tokens are
+// TMEM lanes, text tokens are columns. The epilogue reads each slot three times:
+//   A  the column (text-row) maximum over the CTA's visual tokens: a warp-wide
+//      max per column (redux.sync), then across the four lane-quadrant warps;
+//   B  per-thread sums of 2^(s*c - m*c) per column, reduced across lanes once
+//      per head by a 5-step shuffle transpose (lane l ends with column l);
+//   -  the per-column (m, l) go to every CTA of the cluster with st.async,
+//      which writes the pair and completes bytes on the receiver's mbarrier;
+//      each CTA merges the cluster's pairs in rank order (deterministic) into
+//      b_i = m_i * c + log2(l_i), c = scale * log2(e);
+//   C  each visual token adds sum_i 2^(s_ij * c - b_i) to its running score,
+//      and the slot is handed back to the MMA warp for the next head.
+// While the statistics travel, the producer keeps the next head's K tiles
+// streaming into the ring. The two epilogue warpgroups split each slot's text
+// columns (no cross-warpgroup merge of statistics); each keeps its own partial
+// score rows, added in a fixed order at the end. With several head groups the
+// CTAs write partial rows and a per-tile ticket lets the last writer of each
+// tile add them (fixed group order).
+//
+// Warp roles (320 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
+// MMA issuer, warps 2..5 / 6..9 = epilogue warpgroups 0 / 1. Waits are bounded
+// (clock budget) as in score_tc.cu.
+
+#include <math.h>
+
+#include "internal.h"
+#include "pipe.cuh"
+#include "ptx.cuh"
+
+namespace lvs {
+
+namespace {
+
+constexpr int kResThreads = 320;
+constexpr int kResTmemCols = 512;
+constexpr int kResMaxSlots = 16;
+
+template <int ROW_BYTES, int MROWS>
+struct ResLayout {
+    static constexpr int KB = ROW_BYTES / 128;
+    static constexpr int TILE_BYTES = kTileRows * ROW_BYTES;
+    static constexpr int Q_BYTES = MROWS * ROW_BYTES;
+    // statistics receive buffer: [2 heads][cluster rank][column] (m, l); cluster size
+    // times slot columns must fit RECV_COLS
+    static constexpr int RECV_COLS = ROW_BYTES == 256 ? 512 : 1024;
+    static constexpr int ACC_BYTES = 2 * kResMaxSlots * kTileRows * 4;  // per warpgroup partial rows
+    static constexpr int SCR_BYTES = 2 * 2 * 4 * 64 * 4;                // [max|sum][wg][warp][64 cols]
+    static constexpr int NBAR_FIXED = 2 * 2 + 2 * kResMaxSlots + 2 + 1;
+    static constexpr int FIXED = 2 * Q_BYTES + ACC_BYTES + SCR_BYTES + 2 * RECV_COLS * 8 + 2 * 64 * 4 +
+                                 kResMaxSlots * 4 + (NBAR_FIXED + 2 * 10) * 8 + 64 + 1024;
+    static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
+    static constexpr int kStages = STAGES_FIT > 10 ? 10 : STAGES_FIT;
+    static constexpr int OFF_K = 0;
+    static constexpr int OFF_Q = OFF_K + kStages * TILE_BYTES;
+    static constexpr int OFF_ACC = OFF_Q + 2 * Q_BYTES;
+    static constexpr int OFF_SCR = OFF_ACC + ACC_BYTES;
+    static constexpr int OFF_RECV = OFF_SCR + SCR_BYTES;
+    static constexpr int OFF_B2 = OFF_RECV + 2 * RECV_COLS * 8;
+    static constexpr int OFF_FLAGS = OFF_B2 + 2 * 64 * 4;  // b per warpgroup column, +inf past its columns
+    static constexpr int OFF_BAR = OFF_FLAGS + kResMaxSlots * 4;
+    static constexpr int NBAR = 2 * kStages + NBAR_FIXED;
+    static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+    static constexpr int BYTES = OFF_MISC + 16;
+    static constexpr int ALLOC = BYTES + 1024;
+};
+
+// x[c] (c < 32, one value per lane per column) -> sum over the warp's lanes of
+// column `lane`, returned in lane `lane`.
+__device__ __forceinline__ float transpose_sum32(float (&x)[32], int lane)
+{
+#pragma unroll
+    for (int step = 0; step < 5; ++step) {
+        const int o = 16 >> step;
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int k = 0; k < o; ++k) {
+            const float send = up ? x[k] : x[k + o];
+            const float keep = up ? x[k + o] : x[k];
+            x[k] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    return x[0];
+}
+
+template <int ROW_BYTES, bool FP8, int MROWS>
+__global__ void __launch_bounds__(kResThreads, 1)
+    score_res_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                     const ScoreLaunch p)
+{
+    using L = ResLayout<ROW_BYTES, MROWS>;
+    constexpr int KSTEPS = ROW_BYTES / 32;
+    constexpr int ELEMS_PER_KB = FP8 ? 128 : 64;
+    constexpr uint32_t FMT = FP8 ? 0u : 1u;
+    constexpr int kStages = L::kStages;
+    static_assert(kStages >= 3, "ring depth");
+    static_assert(L::ALLOC > 116 * 1024, "one CTA per SM");
+    static_assert(L::ALLOC <= 227 * 1024, "shared memory per CTA");
+
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t* smem = smem_raw + (base - raw);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.z, hg = blockIdx.y;
+    const uint32_t rank = cluster_ctarank();
+    const uint32_t csize = cluster_nctarank();
+
+    const int n0 = p.seq_off[b];
+    const int N = p.seq_off[b + 1] - n0;
+    const int t0 = p.text_off[b];
+    const int T = p.text_off[b + 1] - t0;
+    const bool multi = p.groups > 1;
+    const int n2 = (T + 15) & ~15;
+    const int n_tiles = (N + kTileRows - 1) / kTileRows;
+    const int tpc = N > 0 ? (n_tiles + (int)csize - 1) / (int)csize : 0;
+    // Uniform for the whole cluster (same request). Shape errors are caught on
+    // the host; this only keeps the kernel within its buffers.
+    const int span = p.slot_cols / 2 + 32 * ((p.slot_cols / 2 + 31) / 32);  // columns the epilogue reads per slot
+    if (T > MROWS || n2 > p.slot_cols || (N > 0 && T <= 0) || (tpc > 0 && (tpc - 1) * p.slot_cols + span > kResTmemCols) ||
+        tpc > kResMaxSlots || (int)csize * p.slot_cols > L::RECV_COLS) {
+        if (threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
+        return;
+    }
+    if (N <= 0) return;
+    const int tile_begin = min(n_tiles, (int)rank * tpc);
+    const int tile_end = min(n_tiles, tile_begin + tpc);
+    const int mt = tile_end - tile_begin;
+    const int G = p.hq / p.hkv;
+    const int hpg = p.heads_per_group;
+    const float cl = p.c_log2;
+    const int scols = p.slot_cols;
+
+    const uint32_t bar0 = base + L::OFF_BAR;
+    auto BAR = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
+    const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + 2, S_FULL = Q_EMPTY + 2,
+              S_EMPTY = S_FULL + kResMaxSlots, STATS = S_EMPTY + kResMaxSlots, DRAIN = STATS + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
+    float* acc_s = reinterpret_cast<float*>(smem + L::OFF_ACC);
+    float* scr_max = reinterpret_cast<float*>(smem + L::OFF_SCR);        // [wg][warp][64]
+    float* scr_sum = scr_max + 2 * 4 * 64;                                // [wg][warp][64]
+    const float2* recv = reinterpret_cast<const float2*>(smem + L::OFF_RECV);
+    float* b2_s = reinterpret_cast<float*>(smem + L::OFF_B2);
+    volatile int* fold_flags = reinterpret_cast<volatile int*>(smem + L::OFF_FLAGS);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(BAR(K_FULL + s), 1);
+            mbar_init(BAR(K_EMPTY + s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(BAR(Q_FULL + i), 1);
+            mbar_init(BAR(Q_EMPTY + i), 1);
+            mbar_init(BAR(STATS + i), 1);  // the local arm; peers complete bytes
+        }
+        for (int i = 0; i < kResMaxSlots; ++i) {
+            mbar_init(BAR(S_FULL + i), 1);
+            mbar_init(BAR(S_EMPTY + i), 256);
+        }
+        mbar_init(BAR(DRAIN), 1);
+        *abort_flag = 0;
+        fence_mbar_init_cluster();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(tmem_slot), kResTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    cluster_sync_all();
+    const uint32_t tmem = *tmem_slot;
+    const Ctl ctl{abort_flag, p.err, p.wait_budget};
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0 && mt > 0) {
+            uint32_t ks = 0, kph = 0;
+            int k_issued[kStages];
+            int q_issued[2] = {0, 0};
+            for (int s = 0; s < kStages; ++s) k_issued[s] = 0;
+            bool ok = true;
+            for (int s = 0; s < hpg && ok; ++s) {
+                const int h = hg * hpg + s;
+                const int g = h / G;
+                const int qb = s & 1;
+                if (!wait_phase(BAR(Q_EMPTY + qb), ((s >> 1) & 1) ^ 1, ctl)) break;
+                mbar_arrive_expect_tx(BAR(Q_FULL + qb), L::Q_BYTES);
+                const uint32_t qdst = base + L::OFF_Q + qb * L::Q_BYTES;
+#pragma unroll
+                for (int kb = 0; kb < L::KB; ++kb)
+                    tma_load_3d(qdst + kb * MROWS * 128, &tm_q, BAR(Q_FULL + qb), kb * ELEMS_PER_KB, h, t0);
+                ++q_issued[qb];
+                for (int t = tile_begin; t < tile_end; ++t) {
+                    if (!wait_phase(BAR(K_EMPTY + ks), kph ^ 1, ctl)) { ok = false; break; }
+                    mbar_arrive_expect_tx(BAR(K_FULL + ks), L::TILE_BYTES);
+                    const uint32_t kdst = base + L::OFF_K + ks * L::TILE_BYTES;
+#pragma unroll
+                    for (int kb = 0; kb < L::KB; ++kb)
+                        tma_load_3d(kdst + kb * kTileRows * 128, &tm_k, BAR(K_FULL + ks), kb * ELEMS_PER_KB, g,
+                                    n0 + t * kTileRows);
+                    ++k_issued[ks];
+                    if (++ks == kStages) { ks = 0; kph ^= 1; }
+                }
+            }
+            volatile int no_abort = 0;
+            const Ctl drain_ctl{&no_abort, p.err, kWaitBudgetCycles};
+            for (int s = 0; s < kStages; ++s)
+                if (k_issued[s] > 0) wait_phase(BAR(K_FULL + s), (uint32_t)(k_issued[s] - 1) & 1u, drain_ctl);
+            for (int s = 0; s < 2; ++s)
+                if (q_issued[s] > 0) wait_phase(BAR(Q_FULL + s), (uint32_t)(q_issued[s] - 1) & 1u, drain_ctl);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            if (mt > 0) {
+                const uint32_t idesc = idesc_make(128, (uint32_t)n2, FMT);
+                uint32_t ks = 0, kph = 0;
+                bool ok = true;
+                for (int s = 0; s < hpg && ok; ++s) {
+                    const int qb = s & 1;
+                    if (!wait_phase(BAR(Q_FULL + qb), (s >> 1) & 1, ctl)) break;
+                    tc_fence_after();
+                    const uint32_t qaddr = base + L::OFF_Q + qb * L::Q_BYTES;
+                    for (int tl = 0; tl < mt; ++tl) {
+                        if (!wait_phase(BAR(K_FULL + ks), kph, ctl)) { ok = false; break; }
+                        if (!wait_phase(BAR(S_EMPTY + tl), ((uint32_t)s & 1u) ^ 1u, ctl)) { ok = false; break; }
+                        tc_fence_after();
+                        const uint32_t kaddr = base + L::OFF_K + ks * L::TILE_BYTES;
+                        const uint32_t d = tmem + (uint32_t)(tl * scols);
+#pragma unroll
+                        for (int st = 0; st < KSTEPS; ++st) {
+                            const uint32_t qoff = (st >> 2) * (MROWS * 128) + (st & 3) * 32;
+                            const uint32_t koff = (st >> 2) * (kTileRows * 128) + (st & 3) * 32;
+                            if (FP8) mma_f8(d, sdesc_k_sw128(kaddr + koff), sdesc_k_sw128(qaddr + qoff), idesc, st > 0);
+                            else mma_f16(d, sdesc_k_sw128(kaddr + koff), sdesc_k_sw128(qaddr + qoff), idesc, st > 0);
+                        }
+                        mma_commit(BAR(S_FULL + tl));
+                        mma_commit(BAR(K_EMPTY + ks));
+                        if (++ks == kStages) { ks = 0; kph ^= 1; }
+                    }
+                    if (ok) mma_commit(BAR(Q_EMPTY + qb));
+                }
+            }
+            mma_commit(BAR(DRAIN));
+            volatile int no_abort = 0;
+            const Ctl drain_ctl{&no_abort, p.err, kWaitBudgetCycles};
+            wait_phase(BAR(DRAIN), 0, drain_ctl);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue (2 warpgroups)
+        // Control flow is identical for every thread of a warpgroup (named
+        // barriers); after an abort every wait returns at once. Every
+        // warp-synchronous instruction (tcgen05.ld, redux.sync, shuffles) is
+        // executed unconditionally: always 32 columns per chunk, columns past
+        // the warpgroup's range masked arithmetically.
+        const int wg = (warp - 2) >> 2;
+        const int quad = warp & 3;
+        const int et = threadIdx.x - 64;               // 0..255
+        const int wt = et - 128 * wg;                  // 0..127 within the warpgroup
+        const int vrow = quad * 32 + lane;             // visual token of this lane within a tile
+        const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+        const uint32_t wg_bar = 2u + (uint32_t)wg;
+        const int h2 = n2 >> 1;                        // this warpgroup's columns: [c_begin, c_begin + h2)
+        const int c_begin = wg * h2;
+        const int nch = (h2 + 31) >> 5;
+        float* accw = acc_s + wg * kResMaxSlots * kTileRows;
+        float* smax = scr_max + wg * 4 * 64;
+        float* ssum = scr_sum + wg * 4 * 64;
+        float* b2w = b2_s + wg * 64;                   // b of column c_begin + c, +inf for c >= h2 or >= T
+        const uint32_t recv_base = base + L::OFF_RECV;
+        const uint32_t tcol = tmem + lane_off;
+        for (int tl = 0; tl < mt; ++tl) accw[tl * kTileRows + vrow] = 0.f;
+        auto lane_valid = [&](int tl) { return tl < mt && (tile_begin + tl) * kTileRows + vrow < N; };
+
+        for (int s = 0; s < hpg; ++s) {
+            const int slot = s & 1;
+            if (et == 0) mbar_arrive_expect_tx(BAR(STATS + slot), (uint32_t)(csize * n2 * 8));
+            for (int ch = 0; ch < nch; ++ch) {
+                const int cw = min(32, h2 - 32 * ch);
+                const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
+                // ---- A: column maxima over this CTA's visual tokens (next slot prefetched)
+                float cm[32];
+#pragma unroll
+                for (int c = 0; c < 32; ++c) cm[c] = -INFINITY;
+                {
+                    float va[32], vb[32];
+                    if (ch == 0 && mt > 0) {  // a rank without tiles gets no MMA
+                        wait_phase(BAR(S_FULL + 0), (uint32_t)s & 1u, ctl);
+                        tc_fence_after();
+                    }
+                    tmem_ld32(tcol + col0, va);
+                    for (int tl = 0; tl < mt; tl += 2) {
+                        const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
+                        tmem_wait_ld();
+                        if (ch == 0 && tl + 1 < mt) {
+                            wait_phase(BAR(S_FULL + t1), (uint32_t)s & 1u, ctl);
+                            tc_fence_after();
+                        }
+                        tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
+                        const bool va_ok = lane_valid(tl);
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], warp_max_f32(va_ok ? va[c] : -INFINITY));
+                        tmem_wait_ld();
+                        if (ch == 0 && tl + 2 < mt) {
+                            wait_phase(BAR(S_FULL + t2), (uint32_t)s & 1u, ctl);
+                            tc_fence_after();
+                        }
+                        tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
+                        const bool vb_ok = lane_valid(tl + 1);
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], warp_max_f32(vb_ok ? vb[c] : -INFINITY));
+                    }
+                    tmem_wait_ld();
+                }
+                if (lane == 0) {
+#pragma unroll
+                    for (int c = 0; c < 32; c += 4)
+                        *reinterpret_cast<float4*>(smax + quad * 64 + 32 * ch + c) =
+                            make_float4(cm[c], cm[c + 1], cm[c + 2], cm[c + 3]);
+                }
+                named_bar_sync(wg_bar, 128);
+                float mc[32];  // column max * c (columns past cw hold garbage and are never used)
+#pragma unroll
+                for (int c = 0; c < 32; c += 4) {
+                    float4 m4 = *reinterpret_cast<const float4*>(smax + 32 * ch + c);
+#pragma unroll
+                    for (int q = 1; q < 4; ++q) {
+                        const float4 o = *reinterpret_cast<const float4*>(smax + q * 64 + 32 * ch + c);
+                        m4.x = fmaxf(m4.x, o.x);
+                        m4.y = fmaxf(m4.y, o.y);
+                        m4.z = fmaxf(m4.z, o.z);
+                        m4.w = fmaxf(m4.w, o.w);
+                    }
+                    mc[c] = m4.x * cl;
+                    mc[c + 1] = m4.y * cl;
+                    mc[c + 2] = m4.z * cl;
+                    mc[c + 3] = m4.w * cl;
+                }
+                // ---- B: per-thread sums of 2^(s*c - m*c), then over the warp's lanes
+                float sm[32];
+#pragma unroll
+                for (int c = 0; c < 32; ++c) sm[c] = 0.f;
+                {
+                    float va[32], vb[32];
+                    tmem_ld32(tcol + col0, va);
+                    for (int tl = 0; tl < mt; tl += 2) {
+                        const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
+                        tmem_wait_ld();
+                        tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
+                        if (lane_valid(tl)) {
+#pragma unroll
+                            for (int c = 0; c < 32; ++c) sm[c] += ex2(fmaf(va[c], cl, -mc[c]));
+                        }
+                        tmem_wait_ld();
+                        tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
+                        if (lane_valid(tl + 1)) {
+#pragma unroll
+                            for (int c = 0; c < 32; ++c) sm[c] += ex2(fmaf(vb[c], cl, -mc[c]));
+                        }
+                    }
+                    tmem_wait_ld();
+                }
+                const float colsum = transpose_sum32(sm, lane);
+                if (lane < cw) ssum[quad * 64 + 32 * ch + lane] = colsum;
+                named_bar_sync(wg_bar, 128);
+                // ---- publish (m, l) of columns col0 .. col0+cw-1 to every CTA of the cluster
+                if (quad == 2 && lane < cw) {  // the warpgroup's first warp
+                    const int c = 32 * ch + lane;
+                    float m = smax[c], l = ssum[c];
+#pragma unroll
+                    for (int q = 1; q < 4; ++q) {
+                        m = fmaxf(m, smax[q * 64 + c]);
+                        l += ssum[q * 64 + c];
+                    }
+                    const int col = c_begin + c;
+                    const uint32_t dst = recv_base + (uint32_t)(((slot * (int)csize + (int)rank) * scols + col) * 8);
+                    const uint32_t bar = BAR(STATS + slot);
+                    for (uint32_t r = 0; r < csize; ++r)
+                        st_async_f2(mapa_shared(dst, r), m, l, mapa_shared(bar, r));
+                }
+            }
+            // ---- merge the cluster's statistics of this head (rank order)
+            wait_phase_cluster(BAR(STATS + slot), (uint32_t)(s >> 1) & 1u, ctl);
+            if (wt < 64) {
+                const int col = c_begin + wt;
+                float bval = INFINITY;
+                if (wt < h2 && col < T) {
+                    float2 st[kMaxCluster];
+#pragma unroll
+                    for (int r = 0; r < kMaxCluster; ++r)
+                        if (r < (int)csize) st[r] = recv[(slot * (int)csize + r) * scols + col];
+                    float M = -INFINITY;
+#pragma unroll
+                    for (int r = 0; r < kMaxCluster; ++r)
+                        if (r < (int)csize) M = fmaxf(M, st[r].x);
+                    float Ls = 0.f;
+#pragma unroll
+                    for (int r = 0; r < kMaxCluster; ++r)
+                        if (r < (int)csize && st[r].y > 0.f) Ls += st[r].y * ex2((st[r].x - M) * cl);
+                    bval = fmaf(M, cl, __log2f(Ls));
+                }
+                b2w[wt] = bval;
+            }
+            named_bar_sync(wg_bar, 128);
+            // ---- C: per-visual-token sums of probabilities over this warpgroup's columns
+            {
+                float va[32], vb[32];
+                float acc_a = 0.f, acc_b = 0.f;
+                for (int ch = 0; ch < nch; ++ch) {
+                    const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
+                    const float* bw = b2w + 32 * ch;
+                    tmem_ld32(tcol + col0, va);
+                    for (int tl = 0; tl < mt; tl += 2) {
+                        const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
+                        tmem_wait_ld();
+                        tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
+                        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+                        for (int c = 0; c < 32; c += 4) {
+                            const float4 bb = *reinterpret_cast<const float4*>(bw + c);
+                            a0 += ex2(fmaf(va[c], cl, -bb.x));
+                            a1 += ex2(fmaf(va[c + 1], cl, -bb.y));
+                            a2 += ex2(fmaf(va[c + 2], cl, -bb.z));
+                            a3 += ex2(fmaf(va[c + 3], cl, -bb.w));
+                        }
+                        acc_a = (a0 + a1) + (a2 + a3);
+                        tmem_wait_ld();
+                        tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
+                        a0 = a1 = a2 = a3 = 0.f;
+#pragma unroll
+                        for (int c = 0; c < 32; c += 4) {
+                            const float4 bb = *reinterpret_cast<const float4*>(bw + c);
+                            a0 += ex2(fmaf(vb[c], cl, -bb.x));
+                            a1 += ex2(fmaf(vb[c + 1], cl, -bb.y));
+                            a2 += ex2(fmaf(vb[c + 2], cl, -bb.z));
+                            a3 += ex2(fmaf(vb[c + 3], cl, -bb.w));
+                        }
+                        acc_b = (a0 + a1) + (a2 + a3);
+                        accw[tl * kTileRows + vrow] += acc_a;
+                        if (tl + 1 < mt) accw[(tl + 1) * kTileRows + vrow] += acc_b;
+                    }
+                    tmem_wait_ld();
+                }
+                // every slot of this head is consumed: hand them back to the MMA warp
+                tc_fence_before();
+                for (int tl = 0; tl < mt; ++tl) mbar_arrive(BAR(S_EMPTY + tl));
+            }
+        }
+        // ---- results: the two warpgroups' partial rows, added in a fixed order
+        named_bar_sync(1, 256);
+        const float denom = (float)p.hq * (float)T;
+        for (int tl = wg; tl < mt; tl += 2) {
+            const int j = (tile_begin + tl) * kTileRows + vrow;
+            if (j < N) {
+                const float a = acc_s[tl * kTileRows + vrow] + acc_s[kResMaxSlots * kTileRows + tl * kTileRows + vrow];
+                if (!multi) p.out[n0 + j] = a / denom;
+                else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
+            }
+        }
+        if (multi) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 256, 1, fold_flags);
+        tc_fence_before();
+    }
+
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kResTmemCols);
+    }
+    cluster_sync_all();
+}
+
+template <int ROW_BYTES, bool FP8, int MROWS>
+cudaError_t res_prepare(int cluster)
+{
+    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         ResLayout<ROW_BYTES, MROWS>::ALLOC);
+    if (e == cudaSuccess && cluster > 8) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return e;
+}
+
+template <int ROW_BYTES, bool FP8, int MROWS>
+cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p, const ScorePlan& plan,
+                       int batch, cudaStream_t stream)
+{
+    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS>;
+    cudaError_t e = res_prepare<ROW_BYTES, FP8, MROWS>(plan.cluster);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(plan.cluster, plan.groups, batch);
+    cfg.blockDim = dim3(kResThreads, 1, 1);
+    cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS>::ALLOC;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = plan.cluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, tm_q, tm_k, p);
+}
+
+template <int ROW_BYTES, bool FP8, int MROWS>
+int res_capacity(int cluster)
+{
+    if (res_prepare<ROW_BYTES, FP8, MROWS>(cluster) != cudaSuccess) return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cluster, 64, 1);
+    cfg.blockDim = dim3(kResThreads, 1, 1);
+    cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS>::ALLOC;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, score_res_kernel<ROW_BYTES, FP8, MROWS>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return n * cluster;
+}
+
+}  // namespace
+
+// Tiles per CTA: the epilogue reads 32 columns per chunk, so the last slot's
+// padded read, (r - 1) * slot_cols + slot_cols / 2 + 32 * chunks, must stay
+// within the 512 TMEM columns.
+int res_max_tiles(int slot_cols)
+{
+    if (slot_cols <= 0) return 0;
+    const int h2 = slot_cols / 2, span = h2 + 32 * ((h2 + 31) / 32);
+    int r = kResMaxSlots;
+    while (r > 0 && (r - 1) * slot_cols + span > kResTmemCols) --r;
+    return r;
+}
+
+int res_max_cluster(int row_bytes, int slot_cols)
+{
+    if (slot_cols <= 0) return 0;
+    const int recv = row_bytes == 256 ? ResLayout<256, 64>::RECV_COLS : ResLayout<128, 64>::RECV_COLS;
+    const int c = recv / slot_cols;
+    return c < kMaxCluster ? c : kMaxCluster;
+}
+
+int res_cluster_capacity(int row_bytes, bool fp8, int mrows, int cluster)
+{
+    if (fp8) return mrows == 64 ? res_capacity<128, true, 64>(cluster) : res_capacity<128, true, 128>(cluster);
+    if (row_bytes == 256)
+        return mrows == 64 ? res_capacity<256, false, 64>(cluster) : res_capacity<256, false, 128>(cluster);
+    return mrows == 64 ? res_capacity<128, false, 64>(cluster) : res_capacity<128, false, 128>(cluster);
+}
+
+cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
+                                  const ScorePlan& plan, int batch, int row_bytes, bool fp8, int mrows,
+                                  cudaStream_t stream)
+{
+    ScoreLaunch q = p;
+    q.groups = plan.groups;
+    q.heads_per_group = p.hq / plan.groups;
+    q.ctas_per_request = plan.cluster * plan.groups;
+    if (fp8)
+        return mrows == 64 ? res_launch<128, true, 64>(tm_q, tm_k, q, plan, batch, stream)
+                           : res_launch<128, true, 128>(tm_q, tm_k, q, plan, batch, stream);
+    if (row_bytes == 256)
+        return mrows == 64 ? res_launch<256, false, 64>(tm_q, tm_k, q, plan, batch, stream)
+                           : res_launch<256, false, 128>(tm_q, tm_k, q, plan, batch, stream);
+    return mrows == 64 ? res_launch<128, false, 64>(tm_q, tm_k, q, plan, batch, stream)
+                       : res_launch<128, false, 128>(tm_q, tm_k, q, plan, batch, stream);
+}
+
+}  // namespace lvs

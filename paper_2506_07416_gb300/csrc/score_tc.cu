@@ -37,6 +37,7 @@
 #include <math.h>
 
 #include "internal.h"
+#include "pipe.cuh"
 #include "ptx.cuh"
 
 namespace lvs {
@@ -59,7 +60,7 @@ struct SmemLayout {
     // Q(s+2) load while pass 2 of head s is still reading Q(s).
     static constexpr int QBUF = MROWS == 64 ? 3 : 2;
     static constexpr int FIXED = QBUF * Q_BYTES + kMaxTilesPerCta * kTileRows * 4 + kStatSlots * kMaxText * 8 +
-                                 2 * kMaxText * 4 + 512 + 64 + 1024;
+                                 2 * kMaxText * 4 + kMaxTilesPerCta * 4 + 512 + 64 + 1024;
     static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
     static constexpr int kStages = STAGES_FIT > 10 ? 10 : STAGES_FIT;
     static constexpr int OFF_K = 0;
@@ -67,7 +68,8 @@ struct SmemLayout {
     static constexpr int OFF_ACC = OFF_Q + QBUF * Q_BYTES;
     static constexpr int OFF_STATS = OFF_ACC + kMaxTilesPerCta * kTileRows * 4;
     static constexpr int OFF_B2 = OFF_STATS + kStatSlots * kMaxText * 8;
-    static constexpr int OFF_BAR = OFF_B2 + 2 * kMaxText * 4;
+    static constexpr int OFF_FLAGS = OFF_B2 + 2 * kMaxText * 4;   // [32] int, fold flags
+    static constexpr int OFF_BAR = OFF_FLAGS + kMaxTilesPerCta * 4;
     // k_full[S], k_empty[S], q_full[QBUF], q_empty[QBUF], t1_full[2], t1_empty[2],
     // t2_full[2], t2_empty[2], stats[4], drain
     static constexpr int NBAR = 2 * kStages + 2 * QBUF + 2 * 4 + kStatSlots + 1;
@@ -75,89 +77,6 @@ struct SmemLayout {
     static constexpr int BYTES = OFF_MISC + 16;
     static constexpr int ALLOC = BYTES + 1024;  // slack for 1024-byte alignment
 };
-
-struct Ctl {
-    volatile int* abort;
-    int32_t* err;
-    long long budget;
-};
-
-__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, const Ctl& c)
-{
-    if (mbar_try_wait(bar, parity)) return true;
-    const long long t0 = clock64();
-    for (;;) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*c.abort) return false;
-        if (clock64() - t0 > c.budget) {
-            *c.abort = 1;
-            atomicOr(c.err, kErrTimeout);
-            return false;
-        }
-    }
-}
-
-__device__ __forceinline__ bool wait_phase_cluster(uint32_t bar, uint32_t parity, const Ctl& c)
-{
-    if (mbar_try_wait_cluster(bar, parity)) return true;
-    const long long t0 = clock64();
-    for (;;) {
-        if (mbar_try_wait_cluster(bar, parity)) return true;
-        if (*c.abort) return false;
-        if (clock64() - t0 > c.budget) {
-            *c.abort = 1;
-            atomicOr(c.err, kErrTimeout);
-            return false;
-        }
-    }
-}
-
-// Online (max, sum 2^(x*c - max*c)) update of one row over NV columns.
-template <int NV>
-__device__ __forceinline__ void row_stats_update(const float* v, int valid, float cl, float& m, float& l)
-{
-    float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
-    if (valid >= NV) {
-#pragma unroll
-        for (int c = 0; c < NV; c += 4) {
-            mx0 = fmaxf(mx0, v[c]);
-            mx1 = fmaxf(mx1, v[c + 1]);
-            mx2 = fmaxf(mx2, v[c + 2]);
-            mx3 = fmaxf(mx3, v[c + 3]);
-        }
-    } else {
-#pragma unroll
-        for (int c = 0; c < NV; c += 4) {
-            mx0 = fmaxf(mx0, c < valid ? v[c] : -INFINITY);
-            mx1 = fmaxf(mx1, c + 1 < valid ? v[c + 1] : -INFINITY);
-            mx2 = fmaxf(mx2, c + 2 < valid ? v[c + 2] : -INFINITY);
-            mx3 = fmaxf(mx3, c + 3 < valid ? v[c + 3] : -INFINITY);
-        }
-    }
-    const float m_new = fmaxf(m, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)));
-    if (m_new == -INFINITY) return;  // no valid column yet
-    const float mc = m_new * cl;
-    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-    if (valid >= NV) {
-#pragma unroll
-        for (int c = 0; c < NV; c += 4) {
-            s0 += ex2(fmaf(v[c], cl, -mc));
-            s1 += ex2(fmaf(v[c + 1], cl, -mc));
-            s2 += ex2(fmaf(v[c + 2], cl, -mc));
-            s3 += ex2(fmaf(v[c + 3], cl, -mc));
-        }
-    } else {
-#pragma unroll
-        for (int c = 0; c < NV; c += 4) {
-            s0 += c < valid ? ex2(fmaf(v[c], cl, -mc)) : 0.f;
-            s1 += c + 1 < valid ? ex2(fmaf(v[c + 1], cl, -mc)) : 0.f;
-            s2 += c + 2 < valid ? ex2(fmaf(v[c + 2], cl, -mc)) : 0.f;
-            s3 += c + 3 < valid ? ex2(fmaf(v[c + 3], cl, -mc)) : 0.f;
-        }
-    }
-    l = l * ex2((m - m_new) * cl) + ((s0 + s1) + (s2 + s3));
-    m = m_new;
-}
 
 template <int ROW_BYTES, bool FP8, int MROWS>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -213,7 +132,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               DRAIN = STATS + kStatSlots;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
-    volatile int* last_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 8);
+    volatile int* fold_flags = reinterpret_cast<volatile int*>(smem + L::OFF_FLAGS);
     float* acc_s = reinterpret_cast<float*>(smem + L::OFF_ACC);
     float2* stats_s = reinterpret_cast<float2*>(smem + L::OFF_STATS);
     float* b2_s = reinterpret_cast<float*>(smem + L::OFF_B2);
@@ -236,7 +155,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < kStatSlots; ++i) mbar_init(BAR(STATS + i), csize);
         mbar_init(BAR(DRAIN), 1);
         *abort_flag = 0;
-        *last_flag = 0;
         fence_mbar_init_cluster();
     }
     if (warp == 0 && lane == 0) {
@@ -396,8 +314,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 tmem_ld32(ta + hh * 64, v);
                                 tmem_ld32(ta + hh * 64 + 32, v + 32);
                             } else {
-                                tmem_ld16x2_32(ta + 0, v);
-                                tmem_ld16x2_32(ta + 32, v + 32);
+                                tmem_ld16x2_32<64>(ta + 0, v);
+                                tmem_ld16x2_32<64>(ta + 32, v + 32);
                             }
                             tmem_wait_ld();
                         }
@@ -425,9 +343,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // ---- publish (m, l) of head s to the cluster
                 const int slot = s % kStatSlots;
                 if (MROWS == 128 || lane < 16) stats_s[slot * kMaxText + prow] = make_float2(m, l);
-                fence_acq_rel_cluster();
                 named_bar_sync(1, 128);
                 if (et == 0) {
+                    fence_acq_rel_cluster();
                     const uint32_t sb = BAR(STATS + slot);
                     for (uint32_t r = 0; r < csize; ++r) mbar_arrive_remote(mapa_shared(sb, r));
                 }
@@ -438,17 +356,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int slot = hs % kStatSlots;
                 float* b2 = b2_s + (hs & 1) * kMaxText;
                 wait_phase_cluster(BAR(STATS + slot), (uint32_t)(hs / kStatSlots) & 1u, ctl);
-                {
-                    const uint32_t my = base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u;
-                    float M = -INFINITY;
-                    for (uint32_t r = 0; r < csize; ++r) M = fmaxf(M, ld_shared_cluster_f2(mapa_shared(my, r)).x);
-                    float Lsum = 0.f;
-                    for (uint32_t r = 0; r < csize; ++r) {
-                        const float2 st = ld_shared_cluster_f2(mapa_shared(my, r));
-                        if (st.y > 0.f) Lsum += st.y * ex2((st.x - M) * cl);
-                    }
-                    b2[et] = (et < T) ? fmaf(M, cl, __log2f(Lsum)) : INFINITY;
-                }
+                if (et < T) b2[et] = merge_cluster_row(base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u, csize, cl);
+                else b2[et] = INFINITY;
                 named_bar_sync(1, 128);
                 // ---- pass 2 of head s-1: per-visual-token sums of probabilities
                 for (int t = tile_begin; t < tile_end; ++t) {
@@ -500,37 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
             }
         }
-        if (multi) {
-            // last CTA of the request (over all head groups) adds the partial rows
-            __threadfence();
-            named_bar_sync(1, 128);
-            if (et == 0) {
-                const int ticket = atomicAdd(p.counters + b, 1);
-                if (ticket == p.ctas_per_request - 1) {
-                    *last_flag = 1;
-                    p.counters[b] = 0;  // ready for the next launch
-                }
-            }
-            named_bar_sync(1, 128);
-            if (*last_flag) {
-                __threadfence();
-                for (int j = et; j < N; j += 128) {
-                    // groups are added in index order; loads issued 8 at a time
-                    const float* src = p.partials + n0 + j;
-                    float sum = 0.f;
-                    int g = 0;
-                    for (; g + 8 <= p.groups; g += 8) {
-                        float x[8];
-#pragma unroll
-                        for (int u = 0; u < 8; ++u) x[u] = __ldcg(src + (int64_t)(g + u) * p.total_vis);
-#pragma unroll
-                        for (int u = 0; u < 8; ++u) sum += x[u];
-                    }
-                    for (; g < p.groups; ++g) sum += __ldcg(src + (int64_t)g * p.total_vis);
-                    p.out[n0 + j] = sum / denom;
-                }
-            }
-        }
+        if (multi) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 128, 1, fold_flags);
         tc_fence_before();
     }
 

@@ -53,7 +53,8 @@ def _load():
     lib.litevlm_select_topk.argtypes = [P, i32, P, P, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
-    for fn in ("create", "destroy", "score", "topk", "compact", "check_device"):
+    lib.litevlm_select_score_plan.argtypes = [P, i32, P, P, P]
+    for fn in ("create", "destroy", "score", "topk", "compact", "check_device", "score_plan"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -63,7 +64,9 @@ LIB = _load()
 # every symbol declared in include/litevlm_select.h
 EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
-           "litevlm_select_check_device"]
+           "litevlm_select_check_device", "litevlm_select_score_plan"]
+FLAGS = {"auto": 0, "reread": 1, "resident": 2}
+KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (pass-2 products resident in TMEM)"}
 
 
 def _check(rc: int, handle) -> None:
@@ -110,9 +113,9 @@ def _stream_ptr(stream) -> Optional[int]:
 # ----------------------------------------------------------------------------
 
 def create(max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int, num_kv_heads: int,
-           head_dim: int, qk_dtype: str = "bf16") -> int:
+           head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto") -> int:
     cfg = Config(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
-                 DTYPES[qk_dtype], 0)
+                 DTYPES[qk_dtype], FLAGS[score_kernel])
     h = ctypes.c_void_p()
     _check(LIB.litevlm_select_create(ctypes.byref(cfg), ctypes.byref(h)), None)
     return h.value
@@ -152,6 +155,14 @@ def check_device(handle: int, stream=None) -> None:
     _check(LIB.litevlm_select_check_device(handle, _stream_ptr(stream)), handle)
 
 
+def score_plan(handle: int, batch: int, text_offsets_h, seq_offsets_h):
+    """(kernel, cluster, tiles_per_cta, groups) litevlm_select_score would launch."""
+    to_h, so_h = _host_i32(text_offsets_h), _host_i32(seq_offsets_h)
+    out = np.zeros(4, np.int32)
+    _check(LIB.litevlm_select_score_plan(handle, batch, _ptr(to_h), _ptr(so_h), _ptr(out)), handle)
+    return tuple(int(v) for v in out)
+
+
 # ----------------------------------------------------------------------------
 # convenience object (allocates outputs with torch; still marshalling only)
 # ----------------------------------------------------------------------------
@@ -160,9 +171,9 @@ class Selector:
     """Owns one handle. Tensors are torch CUDA tensors laid out as in the C header."""
 
     def __init__(self, max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int,
-                 num_kv_heads: int, head_dim: int, qk_dtype: str = "bf16"):
+                 num_kv_heads: int, head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto"):
         self.handle = create(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
-                             qk_dtype)
+                             qk_dtype, score_kernel)
         self.qk_dtype = qk_dtype
 
     def close(self) -> None:
@@ -225,3 +236,7 @@ class Selector:
 
     def check_device(self, stream=None) -> None:
         check_device(self.handle, stream)
+
+    def score_plan(self, text_offsets_h, seq_offsets_h):
+        so = _host_i32(seq_offsets_h)
+        return score_plan(self.handle, len(so) - 1, text_offsets_h, so)

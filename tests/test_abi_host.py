@@ -70,7 +70,8 @@ def _cfg(sel, **kw):
     (dict(num_q_heads=6, num_kv_heads=4), 1),
     (dict(max_batch=0), 1),
     (dict(max_total_visual=-5), 1),
-    (dict(flags=1), 1),
+    (dict(flags=3), 1),
+    (dict(flags=-1), 1),
     (dict(qk_dtype=7), 1),
     (dict(head_dim=96), 2),
     (dict(head_dim=64, qk_dtype=1), 2),

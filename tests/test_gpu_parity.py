@@ -44,9 +44,9 @@ SCORE_CASES = [
 ]
 
 
-def _selector(sel, w, max_batch=None):
+def _selector(sel, w, max_batch=None, kernel="auto"):
     return sel.Selector(max_batch or max(1, w.batch), max(1, w.total_vis), max(1, w.total_txt), w.hq, w.hkv,
-                        w.head_dim, w.dtype)
+                        w.head_dim, w.dtype, score_kernel=kernel)
 
 
 def _gpu_scores(sel, s, w, x, xd):
@@ -56,11 +56,17 @@ def _gpu_scores(sel, s, w, x, xd):
     return out.cpu().numpy()
 
 
+@pytest.mark.parametrize("kernel", ["reread", "resident"])
 @pytest.mark.parametrize("w", SCORE_CASES, ids=lambda w: w.name)
-def test_scores_match_oracle(sel, w):
+def test_scores_match_oracle(sel, w, kernel):
     x = inputs.make_numpy(w)
     xd = to_device(x, w)
-    s = _selector(sel, w)
+    s = _selector(sel, w, kernel=kernel)
+    plan = s.score_plan(x["text_offsets"], x["seq_offsets"])
+    if kernel == "reread":
+        assert plan[0] == 1
+    elif max(w.n_txt) <= 64:
+        assert plan[0] == 2, plan  # every case with short text fits the resident kernel
     g = _gpu_scores(sel, s, w, x, xd)
     o = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, w.dtype,
                      x["q_scale"], x["k_scale"])
@@ -251,10 +257,12 @@ FULL = [("single", [0]), ("highres", [0]), ("fp8_ragged", None), ("sweep", [0, 7
 
 @pytest.mark.parametrize("name,sample", FULL, ids=[f[0] for f in FULL])
 def test_full_size_workload(sel, name, sample):
+    """Full size, in the launch configuration bench.py times (automatic kernel choice)."""
     w = inputs.workload(name)
     xd = inputs.make_torch(w, "cuda")
     so, to = w.seq_offsets(), w.text_offsets()
     s = _selector(sel, w)
+    print(f"{name}: score plan {s.score_plan(to, so)}")
     g_t = s.score(xd["q"], xd["text_offsets"], xd["k"], xd["seq_offsets"], xd["q_scale"], xd["k_scale"],
                   seq_offsets_h=so, text_offsets_h=to)
     s.check_device()
