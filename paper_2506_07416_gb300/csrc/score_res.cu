@@ -9,16 +9,19 @@
 //     S^T = K_tile * Q_h^T   (M = 128 visual rows, N = T rounded up to 16, K = d)
 // into a TMEM slot that stays resident for the whole head. Visual tokens are
 // TMEM lanes, text tokens are columns. The epilogue reads each slot three times:
-//   A  the column (text-row) maximum over the CTA's visual tokens: a warp-wide
-//      max per column (redux.sync), then across the four lane-quadrant warps;
-//   B  per-thread sums of 2^(s*c - m*c) per column, reduced across lanes once
+//   A  the column (text-row) maximum over the CTA's visual tokens: per thread
+//      over its slots, then one warp-wide max per column (redux.sync) and a
+//      max over the four lane-quadrant warps;
+//   B  e = 2^(s*c - m*c) (m: the CTA's column max) is written back over the
+//      logits; per-thread sums of e per column are reduced across lanes once
 //      per head by a 5-step shuffle transpose (lane l ends with column l);
 //   -  the per-column (m, l) go to every CTA of the cluster with st.async,
 //      which writes the pair and completes bytes on the receiver's mbarrier;
 //      each CTA merges the cluster's pairs in rank order (deterministic) into
-//      b_i = m_i * c + log2(l_i), c = scale * log2(e);
-//   C  each visual token adds sum_i 2^(s_ij * c - b_i) to its running score,
-//      and the slot is handed back to the MMA warp for the next head.
+//      b_i = M_i * c + log2(L_i), c = scale * log2(e), and the column weight
+//      w_i = 2^(m_i * c - b_i);
+//   C  each visual token adds sum_i e_ij * w_i (= sum_i 2^(s_ij * c - b_i)) to
+//      its running score, and the slot goes back to the MMA warp.
 // While the statistics travel, the producer keeps the next head's K tiles
 // streaming into the ring. The two epilogue warpgroups split each slot's text
 // columns (no cross-warpgroup merge of statistics); each keeps its own partial
@@ -283,7 +286,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         float* accw = acc_s + wg * kResMaxSlots * kTileRows;
         float* smax = scr_max + wg * 4 * 64;
         float* ssum = scr_sum + wg * 4 * 64;
-        float* b2w = b2_s + wg * 64;                   // b of column c_begin + c, +inf for c >= h2 or >= T
+        float* b2w = b2_s + wg * 64;                   // weight of column c_begin + c, 0 for c >= h2 or >= T
         const uint32_t recv_base = base + L::OFF_RECV;
         const uint32_t tcol = tmem + lane_off;
         for (int tl = 0; tl < mt; ++tl) accw[tl * kTileRows + vrow] = 0.f;
@@ -295,7 +298,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
             for (int ch = 0; ch < nch; ++ch) {
                 const int cw = min(32, h2 - 32 * ch);
                 const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
-                // ---- A: column maxima over this CTA's visual tokens (next slot prefetched)
+                // ---- A: column maxima, per thread over its slots, then over the lanes
                 float cm[32];
 #pragma unroll
                 for (int c = 0; c < 32; ++c) cm[c] = -INFINITY;
@@ -314,21 +317,25 @@ __global__ void __launch_bounds__(kResThreads, 1)
                             tc_fence_after();
                         }
                         tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
-                        const bool va_ok = lane_valid(tl);
+                        if (lane_valid(tl)) {
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], warp_max_f32(va_ok ? va[c] : -INFINITY));
+                            for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], va[c]);
+                        }
                         tmem_wait_ld();
                         if (ch == 0 && tl + 2 < mt) {
                             wait_phase(BAR(S_FULL + t2), (uint32_t)s & 1u, ctl);
                             tc_fence_after();
                         }
                         tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
-                        const bool vb_ok = lane_valid(tl + 1);
+                        if (lane_valid(tl + 1)) {
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], warp_max_f32(vb_ok ? vb[c] : -INFINITY));
+                            for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], vb[c]);
+                        }
                     }
                     tmem_wait_ld();
                 }
+#pragma unroll
+                for (int c = 0; c < 32; ++c) cm[c] = warp_max_f32(cm[c]);
                 if (lane == 0) {
 #pragma unroll
                     for (int c = 0; c < 32; c += 4)
@@ -336,7 +343,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                             make_float4(cm[c], cm[c + 1], cm[c + 2], cm[c + 3]);
                 }
                 named_bar_sync(wg_bar, 128);
-                float mc[32];  // column max * c (columns past cw hold garbage and are never used)
+                float mc[32];  // CTA-local column max * c (columns past cw: garbage, never used)
 #pragma unroll
                 for (int c = 0; c < 32; c += 4) {
                     float4 m4 = *reinterpret_cast<const float4*>(smax + 32 * ch + c);
@@ -353,29 +360,24 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     mc[c + 2] = m4.z * cl;
                     mc[c + 3] = m4.w * cl;
                 }
-                // ---- B: per-thread sums of 2^(s*c - m*c), then over the warp's lanes
+                // ---- B: e = 2^(s*c - m*c) written back over the logits (this warpgroup's
+                // columns only); per-thread column sums of e, then over the warp's lanes
                 float sm[32];
 #pragma unroll
                 for (int c = 0; c < 32; ++c) sm[c] = 0.f;
-                {
-                    float va[32], vb[32];
-                    tmem_ld32(tcol + col0, va);
-                    for (int tl = 0; tl < mt; tl += 2) {
-                        const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
-                        tmem_wait_ld();
-                        tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
-                        if (lane_valid(tl)) {
-#pragma unroll
-                            for (int c = 0; c < 32; ++c) sm[c] += ex2(fmaf(va[c], cl, -mc[c]));
-                        }
-                        tmem_wait_ld();
-                        tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
-                        if (lane_valid(tl + 1)) {
-#pragma unroll
-                            for (int c = 0; c < 32; ++c) sm[c] += ex2(fmaf(vb[c], cl, -mc[c]));
-                        }
-                    }
+                for (int tl = 0; tl < mt; ++tl) {
+                    float v[32];
+                    const uint32_t ta = tcol + (uint32_t)(tl * scols) + col0;
+                    tmem_ld32(ta, v);
                     tmem_wait_ld();
+                    const bool ok = lane_valid(tl);
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) {
+                        const float e = ok ? ex2(fmaf(v[c], cl, -mc[c])) : 0.f;
+                        v[c] = e;
+                        sm[c] += e;
+                    }
+                    tmem_st_cols(ta, v, cw);
                 }
                 const float colsum = transpose_sum32(sm, lane);
                 if (lane < cw) ssum[quad * 64 + 32 * ch + lane] = colsum;
@@ -396,11 +398,13 @@ __global__ void __launch_bounds__(kResThreads, 1)
                         st_async_f2(mapa_shared(dst, r), m, l, mapa_shared(bar, r));
                 }
             }
-            // ---- merge the cluster's statistics of this head (rank order)
+            tmem_wait_st();
+            // ---- merge the cluster's statistics of this head (rank order) into the
+            // column weights w = 2^(m_local*c - b), b = M*c + log2(L); 0 for unused columns
             wait_phase_cluster(BAR(STATS + slot), (uint32_t)(s >> 1) & 1u, ctl);
             if (wt < 64) {
                 const int col = c_begin + wt;
-                float bval = INFINITY;
+                float wval = 0.f;
                 if (wt < h2 && col < T) {
                     float2 st[kMaxCluster];
 #pragma unroll
@@ -414,54 +418,60 @@ __global__ void __launch_bounds__(kResThreads, 1)
 #pragma unroll
                     for (int r = 0; r < kMaxCluster; ++r)
                         if (r < (int)csize && st[r].y > 0.f) Ls += st[r].y * ex2((st[r].x - M) * cl);
-                    bval = fmaf(M, cl, __log2f(Ls));
+                    const float b = fmaf(M, cl, __log2f(Ls));
+                    float mloc = smax[wt];  // this CTA's column max: the e values' reference
+#pragma unroll
+                    for (int q = 1; q < 4; ++q) mloc = fmaxf(mloc, smax[q * 64 + wt]);
+                    wval = mloc == -INFINITY ? 0.f : ex2(fmaf(mloc, cl, -b));
                 }
-                b2w[wt] = bval;
+                b2w[wt] = wval;
             }
             named_bar_sync(wg_bar, 128);
-            // ---- C: per-visual-token sums of probabilities over this warpgroup's columns
-            {
-                float va[32], vb[32];
-                float acc_a = 0.f, acc_b = 0.f;
-                for (int ch = 0; ch < nch; ++ch) {
-                    const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
-                    const float* bw = b2w + 32 * ch;
-                    tmem_ld32(tcol + col0, va);
-                    for (int tl = 0; tl < mt; tl += 2) {
-                        const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
-                        tmem_wait_ld();
-                        tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
-                        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+            // ---- C: per-visual-token sums of e * w over this warpgroup's columns
+            for (int ch = 0; ch < nch; ++ch) {
+                const int cw = min(32, h2 - 32 * ch);
+                const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
+                float wv[32];
 #pragma unroll
-                        for (int c = 0; c < 32; c += 4) {
-                            const float4 bb = *reinterpret_cast<const float4*>(bw + c);
-                            a0 += ex2(fmaf(va[c], cl, -bb.x));
-                            a1 += ex2(fmaf(va[c + 1], cl, -bb.y));
-                            a2 += ex2(fmaf(va[c + 2], cl, -bb.z));
-                            a3 += ex2(fmaf(va[c + 3], cl, -bb.w));
-                        }
-                        acc_a = (a0 + a1) + (a2 + a3);
-                        tmem_wait_ld();
-                        tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
-                        a0 = a1 = a2 = a3 = 0.f;
-#pragma unroll
-                        for (int c = 0; c < 32; c += 4) {
-                            const float4 bb = *reinterpret_cast<const float4*>(bw + c);
-                            a0 += ex2(fmaf(vb[c], cl, -bb.x));
-                            a1 += ex2(fmaf(vb[c + 1], cl, -bb.y));
-                            a2 += ex2(fmaf(vb[c + 2], cl, -bb.z));
-                            a3 += ex2(fmaf(vb[c + 3], cl, -bb.w));
-                        }
-                        acc_b = (a0 + a1) + (a2 + a3);
-                        accw[tl * kTileRows + vrow] += acc_a;
-                        if (tl + 1 < mt) accw[(tl + 1) * kTileRows + vrow] += acc_b;
-                    }
-                    tmem_wait_ld();
+                for (int c = 0; c < 32; c += 4) {
+                    const float4 w4 = *reinterpret_cast<const float4*>(b2w + 32 * ch + c);
+                    wv[c] = w4.x;
+                    wv[c + 1] = w4.y;
+                    wv[c + 2] = w4.z;
+                    wv[c + 3] = w4.w;
                 }
-                // every slot of this head is consumed: hand them back to the MMA warp
-                tc_fence_before();
-                for (int tl = 0; tl < mt; ++tl) mbar_arrive(BAR(S_EMPTY + tl));
+                float va[32], vb[32];
+                tmem_ld32(tcol + col0, va);
+                for (int tl = 0; tl < mt; tl += 2) {
+                    const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
+                    tmem_wait_ld();
+                    tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
+                    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+                    for (int c = 0; c < 32; c += 2) {
+                        if (c < cw) {
+                            a0 = fmaf(va[c], wv[c], a0);
+                            a1 = fmaf(va[c + 1], wv[c + 1], a1);
+                        }
+                    }
+                    accw[tl * kTileRows + vrow] += a0 + a1;
+                    tmem_wait_ld();
+                    tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
+                    a0 = a1 = 0.f;
+#pragma unroll
+                    for (int c = 0; c < 32; c += 2) {
+                        if (c < cw) {
+                            a0 = fmaf(vb[c], wv[c], a0);
+                            a1 = fmaf(vb[c + 1], wv[c + 1], a1);
+                        }
+                    }
+                    if (tl + 1 < mt) accw[(tl + 1) * kTileRows + vrow] += a0 + a1;
+                }
+                tmem_wait_ld();
             }
+            // every slot of this head is consumed: hand them back to the MMA warp
+            tc_fence_before();
+            for (int tl = 0; tl < mt; ++tl) mbar_arrive(BAR(S_EMPTY + tl));
         }
         // ---- results: the two warpgroups' partial rows, added in a fixed order
         named_bar_sync(1, 256);
