@@ -47,6 +47,7 @@ def parse_args():
     ap.add_argument("--workload", default="single", choices=["single", "highres", "fp8_ragged", "sweep"])
     ap.add_argument("--ratio", type=float, default=None, help="keep ratio override (sweep: 0.1/0.2/0.3/0.5)")
     ap.add_argument("--batch", type=int, default=None, help="use only the first B requests (profiling)")
+    ap.add_argument("--score-kernel", default="auto", choices=["auto", "reread", "resident"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="bounded CPU work for the oracle baseline")
@@ -262,7 +263,8 @@ def run_ours(args):
     kk_d = None if kk_h is None else torch.from_numpy(kk_h).to(dev)
     ratio = float(w.keep_ratio or 0.0)
     total_kept = int(sum(alg["kept"]))
-    sel = select.Selector(w.batch, w.total_vis, w.total_txt, w.hq, w.hkv, w.head_dim, w.dtype)
+    sel = select.Selector(w.batch, w.total_vis, w.total_txt, w.hq, w.hkv, w.head_dim, w.dtype,
+                          score_kernel=args.score_kernel)
     h = sel.handle
     scores = torch.empty(w.total_vis, dtype=torch.float32, device=dev)
     kept = torch.empty(max(1, total_kept), dtype=torch.int32, device=dev)
