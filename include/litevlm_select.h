@@ -185,7 +185,8 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t handle, int32_t batc
 /*
  * Synchronises `stream`, then reads and clears the handle's device error word.
  * Returns OK, TIMEOUT (a kernel's bounded wait gave up; its outputs are not
- * valid), DEVICE_BOUNDS, or CUDA.
+ * valid, and the workspace's fold tickets are reset so the next call starts
+ * clean), DEVICE_BOUNDS, or CUDA.
  */
 litevlm_status_t litevlm_select_check_device(litevlm_select_t handle, litevlm_stream_t stream);
 

@@ -20,6 +20,7 @@ struct litevlm_select {
     int num_sms = 0;
     float* partials = nullptr;  // [Hq][max_total_visual]: per-head-group partial scores
     int32_t* counters = nullptr;  // fold tickets of the score kernels, one per 128-token tile
+    size_t n_counters = 0;
     int32_t* err_d = nullptr;   // device error word (bits lvs::kErr*)
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     int res_capacity[2][17];  // resident score kernel: CTAs at once per cluster size, by pass-1 rows (64/128); -1 unknown
@@ -214,9 +215,9 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
     if (e == cudaSuccess && c->num_q_heads > 1)
         e = cudaMalloc(&h->partials, sizeof(float) * (size_t)c->num_q_heads * (size_t)c->max_total_visual);
     // one fold ticket per 128-token tile: index floor(n0 / 128) + t + b < total / 128 + 2 * batch + 1
-    const size_t n_counters = (size_t)(c->max_total_visual / lvs::kTileRows) + 2 * (size_t)c->max_batch + 2;
-    if (e == cudaSuccess) e = cudaMalloc(&h->counters, sizeof(int32_t) * n_counters);
-    if (e == cudaSuccess) e = cudaMemset(h->counters, 0, sizeof(int32_t) * n_counters);
+    h->n_counters = (size_t)(c->max_total_visual / lvs::kTileRows) + 2 * (size_t)c->max_batch + 2;
+    if (e == cudaSuccess) e = cudaMalloc(&h->counters, sizeof(int32_t) * h->n_counters);
+    if (e == cudaSuccess) e = cudaMemset(h->counters, 0, sizeof(int32_t) * h->n_counters);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         const std::string msg = std::string("create: ") + cudaGetErrorString(e);
@@ -445,6 +446,8 @@ litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e == cudaSuccess) e = cudaMemcpy(&word, h->err_d, sizeof(word), cudaMemcpyDeviceToHost);
     if (e == cudaSuccess && word) e = cudaMemset(h->err_d, 0, sizeof(int32_t));
+    // a score kernel that gave up may have taken only some of its fold tickets
+    if (e == cudaSuccess && (word & lvs::kErrTimeout)) e = cudaMemset(h->counters, 0, sizeof(int32_t) * h->n_counters);
     if (e != cudaSuccess) return cuda_fail(h, e, "check_device");
     if (word & lvs::kErrTimeout) return fail(h, LITEVLM_ERR_TIMEOUT, "a device-side wait timed out");
     if (word & lvs::kErrBounds) return fail(h, LITEVLM_ERR_DEVICE_BOUNDS, "a gather index was out of bounds");
