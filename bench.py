@@ -54,6 +54,10 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="bounded CPU work for the oracle baseline")
     ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--events", default="score", choices=["stage", "score", "step"],
+                    help="CUDA events in the timed loop: around every stage, around the score kernel and the "
+                         "step, or at step boundaries only (an event between two kernels can keep the second "
+                         "from launching early)")
     return ap.parse_args()
 
 
@@ -326,10 +330,12 @@ def run_ours(args):
         e[0].record(stream)
         call(L.litevlm_select_score(h, w.batch, q.data_ptr(), to_d.data_ptr(), c_to_h, k.data_ptr(),
                                     so_d.data_ptr(), c_so_h, xd["q_scale"], xd["k_scale"], scores.data_ptr(), sp))
-        e[1].record(stream)
+        if args.events != "step":
+            e[1].record(stream)
         call(L.litevlm_select_topk(h, w.batch, scores.data_ptr(), so_d.data_ptr(), c_so_h, c_kk_d, c_kk_h, ratio,
                                    kept.data_ptr(), off_d.data_ptr(), off_h.ctypes.data, sp))
-        e[2].record(stream)
+        if args.events == "stage":
+            e[2].record(stream)
         call(L.litevlm_select_compact(h, total_kept, kept.data_ptr(), w.total_vis, n_t, c_src, c_dst, c_rb, sp))
         e[3].record(stream)
     torch.cuda.synchronize()
@@ -339,8 +345,12 @@ def run_ours(args):
         dist.barrier()
     sel.check_device()
 
-    st = np.array([[e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2]), e[2].elapsed_time(e[3])] for e in ev])
-    per_step_ms = st.sum(axis=1)
+    nan = float("nan")
+    st = np.array([[e[0].elapsed_time(e[1]) if args.events != "step" else nan,
+                    e[1].elapsed_time(e[2]) if args.events == "stage" else nan,
+                    e[2].elapsed_time(e[3]) if args.events == "stage" else nan,
+                    e[0].elapsed_time(e[3])] for e in ev])
+    per_step_ms = st[:, 3]
     total_ms = float(per_step_ms.sum())
     if world > 1:
         t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
@@ -374,7 +384,10 @@ def run_ours(args):
         v, desc, el, runs = time_oracle(w, args.cpu_seconds)
         cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
 
-    stage_us = {n: float(np.median(st[:, i]) * 1e3) for i, n in enumerate(("score", "topk", "compact"))}
+    stage_us = {n: (float(np.median(st[:, i]) * 1e3) if not np.isnan(st[0, i]) else None)
+                for i, n in enumerate(("score", "topk", "compact"))}
+    if args.events == "score":
+        stage_us["topk+compact"] = float(np.median(st[:, 3] - st[:, 0]) * 1e3)
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps, "warmup": warm,
             "ms_per_step": total_ms / steps, "p50_us": float(np.median(per_step_ms) * 1e3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,

@@ -9,6 +9,7 @@
 // [0, src_rows) are skipped and flagged in the error word.
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace lvs {
 
@@ -20,6 +21,8 @@ __global__ void __launch_bounds__(kGatherThreads)
     compact_vec16_kernel(int64_t total_kept, const int32_t* __restrict__ kept_idx, int64_t src_rows,
                          const GatherArgs g, int32_t* err)
 {
+    griddep_wait();
+    griddep_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int64_t w = ((int64_t)blockIdx.x * kGatherThreads + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * kGatherThreads) >> 5;
@@ -54,6 +57,8 @@ __global__ void __launch_bounds__(kGatherThreads)
     compact_bytes_kernel(int64_t total_kept, const int32_t* __restrict__ kept_idx, int64_t src_rows,
                          const GatherArgs g, int32_t* err)
 {
+    griddep_wait();
+    griddep_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int64_t w = ((int64_t)blockIdx.x * kGatherThreads + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * kGatherThreads) >> 5;
@@ -82,13 +87,15 @@ cudaError_t launch_compact(int64_t total_kept, const int32_t* kept_idx, int64_t 
     int64_t blocks = (total_kept + warps_per_block - 1) / warps_per_block;
     const int64_t cap = (int64_t)num_sms * 8;  // 2048 threads per SM
     if (blocks > cap) blocks = cap;
-    if (vec16)
-        compact_vec16_kernel<<<(unsigned)blocks, kGatherThreads, 0, stream>>>(total_kept, kept_idx, src_rows, g,
-                                                                              err);
-    else
-        compact_bytes_kernel<<<(unsigned)blocks, kGatherThreads, 0, stream>>>(total_kept, kept_idx, src_rows, g,
-                                                                              err);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks, 1, 1);
+    cfg.blockDim = dim3(kGatherThreads, 1, 1);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1] = {pdl_attribute()};
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, vec16 ? compact_vec16_kernel : compact_bytes_kernel, total_kept, kept_idx,
+                              src_rows, g, err);
 }
 
 }  // namespace lvs

@@ -20,6 +20,18 @@ constexpr int kMaxCluster = 16;
 // Wait budget for every device-side wait, in SM clock cycles (about 2 s).
 constexpr long long kWaitBudgetCycles = 4000000000LL;
 
+// Every kernel of the library is launched with programmatic dependent launch:
+// it may be scheduled while the previous kernel of the stream is finishing,
+// and it waits for that kernel to complete (griddepcontrol.wait) before its
+// first global-memory access, so stream order is kept for all memory.
+inline cudaLaunchAttribute pdl_attribute()
+{
+    cudaLaunchAttribute a;
+    a.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    a.val.programmaticStreamSerializationAllowed = 1;
+    return a;
+}
+
 struct ScoreLaunch {
     const int32_t* seq_off;   // device [batch+1]
     const int32_t* text_off;  // device [batch+1]

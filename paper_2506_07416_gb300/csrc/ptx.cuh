@@ -132,6 +132,12 @@ __device__ __forceinline__ void fence_acq_rel_cluster()
 // ----------------------------------------------------------------------------
 // TMA
 // ----------------------------------------------------------------------------
+// Programmatic dependent launch: wait until the grids this one depends on
+// have completed and their writes are visible (returns at once without one),
+// and let the next grid of the stream start launching.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map)
 {
     asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");

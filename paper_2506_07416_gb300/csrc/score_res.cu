@@ -118,6 +118,8 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const uint32_t rank = cluster_ctarank();
     const uint32_t csize = cluster_nctarank();
 
+    griddep_wait();
+    griddep_launch_dependents();
     const int n0 = p.seq_off[b];
     const int N = p.seq_off[b + 1] - n0;
     const int t0 = p.text_off[b];
@@ -518,13 +520,14 @@ cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const S
     cfg.blockDim = dim3(kResThreads, 1, 1);
     cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS>::ALLOC;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = plan.cluster;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1] = pdl_attribute();
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, tm_q, tm_k, p);
 }
 

@@ -103,6 +103,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t rank = cluster_ctarank();
     const uint32_t csize = cluster_nctarank();
 
+    griddep_wait();
+    griddep_launch_dependents();
     const int n0 = p.seq_off[b];
     const int N = p.seq_off[b + 1] - n0;
     const int t0 = p.text_off[b];
@@ -439,13 +441,14 @@ cudaError_t launch_variant(const CUtensorMap& tm_q, const CUtensorMap& tm_k, con
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = plan.cluster;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1] = pdl_attribute();
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, tm_q, tm_k, p);
 }
 

@@ -14,6 +14,7 @@
 #include <math.h>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace lvs {
 
@@ -80,6 +81,8 @@ __global__ void __launch_bounds__(kTopkThreads)
 
     const int b = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    griddep_wait();
+    griddep_launch_dependents();
     const int n0 = seq_off[b];
     const int N = seq_off[b + 1] - n0;
 
@@ -189,21 +192,244 @@ __global__ void __launch_bounds__(kTopkThreads)
     }
 }
 
+
+// ---------------------------------------------------------------------------
+// Register-resident variant for requests of at most kTopkThreads * KPT tokens.
+// Thread t holds the keys of tokens j = e * kTopkThreads + t (e < KPT), so the
+// loads are coalesced and "round e, warp w, lane l" is index order. The radix
+// select starts below the bits that every key of the request shares (one
+// min/max reduction finds them) and stops as soon as the bin holding the k-th
+// key is taken whole. Every warp finds the selected digit from the shared
+// histogram by itself, so a pass costs one barrier; histograms rotate over
+// three buffers so a buffer is cleared two passes after it was last read.
+// Output positions come from per-(round, warp) ballot counts.
+
+template <int KPT>
+__global__ void __launch_bounds__(kTopkThreads)
+    topk_reg_kernel(const float* __restrict__ scores, const int32_t* __restrict__ seq_off,
+                    const int32_t* __restrict__ keep_k, float ratio, int32_t* __restrict__ kept_idx,
+                    int32_t* __restrict__ out_off)
+{
+    __shared__ uint32_t hist[3][256];
+    __shared__ uint32_t wmin[kTopkWarps], wmax[kTopkWarps];
+    __shared__ int cnt[KPT][kTopkWarps];
+    __shared__ long long s_base;
+
+    const int b = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    griddep_wait();
+    griddep_launch_dependents();
+    const int n0 = seq_off[b];
+    const int N = seq_off[b + 1] - n0;
+
+    uint32_t key[KPT];
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) {
+        const int j = e * kTopkThreads + tid;
+        key[e] = j < N ? order_key(__ldcg(scores + n0 + j)) : 0u;
+    }
+
+    // output base = sum of k over earlier requests
+    long long part = 0;
+    for (int bb = tid; bb < b; bb += kTopkThreads) part += keep_count(seq_off, keep_k, ratio, bb);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
+    if (tid == 0) s_base = 0;
+    __syncthreads();
+    if (lane == 0 && part) atomicAdd(reinterpret_cast<unsigned long long*>(&s_base), (unsigned long long)part);
+    const int k = keep_count(seq_off, keep_k, ratio, b);
+
+    // key range of the request (padding slots take part only through valid keys)
+    uint32_t lo_k = 0xFFFFFFFFu, hi_k = 0u;
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) {
+        if (e * kTopkThreads + tid < N) {
+            lo_k = min(lo_k, key[e]);
+            hi_k = max(hi_k, key[e]);
+        }
+    }
+    lo_k = __reduce_min_sync(0xffffffffu, lo_k);
+    hi_k = __reduce_max_sync(0xffffffffu, hi_k);
+    if (lane == 0) {
+        wmin[warp] = lo_k;
+        wmax[warp] = hi_k;
+    }
+    for (int i = tid; i < 2 * 256; i += kTopkThreads) (&hist[0][0])[i] = 0u;
+    __syncthreads();
+    const long long out_base = s_base;
+    if (tid == 0) {
+        out_off[b + 1] = (int32_t)(out_base + k);
+        if (b == 0) out_off[0] = 0;
+    }
+    if (k <= 0 || N <= 0) return;
+    int32_t* dst = kept_idx + out_base;
+    if (k >= N) {
+        for (int j = tid; j < N; j += kTopkThreads) dst[j] = n0 + j;
+        return;
+    }
+    lo_k = wmin[0];
+    hi_k = wmax[0];
+#pragma unroll
+    for (int w = 1; w < kTopkWarps; ++w) {
+        lo_k = min(lo_k, wmin[w]);
+        hi_k = max(hi_k, wmax[w]);
+    }
+
+    // ---- radix select below the common high bits
+    const uint32_t diff = lo_k ^ hi_k;
+    uint32_t mask = diff ? ~((2u << (31 - __clz(diff))) - 1u) : 0xFFFFFFFFu;
+    uint32_t prefix = lo_k & mask;
+    int remaining = k;                // keys still to take from the keys matching prefix under mask
+    int n_eq = N;                     // keys matching prefix under mask
+    int top = diff ? 31 - __clz(diff) : -1;
+    int pass = 0;
+    while (top >= 0 && n_eq != remaining) {
+        const int lo = top >= 7 ? top - 7 : 0;
+        const uint32_t dmask = (2u << (top - lo)) - 1u;
+        uint32_t* h = hist[pass % 3];
+#pragma unroll
+        for (int e = 0; e < KPT; ++e) {
+            if (e * kTopkThreads + tid < N && (key[e] & mask) == prefix) atomicAdd(&h[(key[e] >> lo) & dmask], 1u);
+        }
+        if (tid < 256) hist[(pass + 1) % 3][tid] = 0u;
+        __syncthreads();
+        // every warp: the digit d with (count above d) < remaining <= (count above d) + count(d)
+        uint32_t c[8], tot = 0;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            c[e] = h[lane * 8 + e];
+            tot += c[e];
+        }
+        uint32_t suf = tot;  // sum over lanes >= this lane
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_down_sync(0xffffffffu, suf, o);
+            if (lane + o < 32) suf += y;
+        }
+        uint32_t above = suf - tot, digit = 0, cnt_d = 0, above_d = 0;
+        const bool mine = above < (uint32_t)remaining && (uint32_t)remaining <= suf;
+        if (mine) {
+#pragma unroll
+            for (int e = 7; e >= 0; --e) {
+                if (cnt_d == 0 && above + c[e] >= (uint32_t)remaining) {
+                    digit = (uint32_t)(lane * 8 + e);
+                    cnt_d = c[e];
+                    above_d = above;
+                }
+                above += c[e];
+            }
+        }
+        const int src = __ffs(__ballot_sync(0xffffffffu, mine)) - 1;
+        digit = __shfl_sync(0xffffffffu, digit, src);
+        cnt_d = __shfl_sync(0xffffffffu, cnt_d, src);
+        above_d = __shfl_sync(0xffffffffu, above_d, src);
+        prefix |= digit << lo;
+        mask |= dmask << lo;
+        remaining -= (int)above_d;
+        n_eq = (int)cnt_d;
+        top = lo - 1;
+        ++pass;
+    }
+
+    // ---- keep keys above prefix, and the first `remaining` keys equal to it in index order
+    uint32_t gt = 0, eq = 0;
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) {
+        const bool valid = e * kTopkThreads + tid < N;
+        const uint32_t m = key[e] & mask;
+        gt |= (uint32_t)(valid && m > prefix) << e;
+        eq |= (uint32_t)(valid && m == prefix) << e;
+    }
+    const uint32_t lt_mask = (1u << lane) - 1u;
+    uint32_t keep = gt | eq;
+    if (n_eq != remaining) {
+        // rank of each equal key among the equal keys (index order)
+#pragma unroll
+        for (int e = 0; e < KPT; ++e) {
+            const uint32_t bal = __ballot_sync(0xffffffffu, (eq >> e) & 1u);
+            if (lane == 0) cnt[e][warp] = __popc(bal);
+        }
+        __syncthreads();
+        int run = 0;
+        keep = gt;
+#pragma unroll
+        for (int e = 0; e < KPT; ++e) {
+            int v = lane < kTopkWarps ? cnt[e][lane] : 0;
+#pragma unroll
+            for (int o = 1; o < kTopkWarps; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, v, o);
+                if (lane >= o) v += y;
+            }
+            const int before_w = __shfl_sync(0xffffffffu, v, (warp + kTopkWarps - 1) % kTopkWarps);
+            const int tot_e = __shfl_sync(0xffffffffu, v, kTopkWarps - 1);
+            const uint32_t bal = __ballot_sync(0xffffffffu, (eq >> e) & 1u);
+            const int rank = run + (warp ? before_w : 0) + __popc(bal & lt_mask);
+            if (((eq >> e) & 1u) && rank < remaining) keep |= 1u << e;
+            run += tot_e;
+        }
+        __syncthreads();  // cnt is reused below
+    }
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) {
+        const uint32_t bal = __ballot_sync(0xffffffffu, (keep >> e) & 1u);
+        if (lane == 0) cnt[e][warp] = __popc(bal);
+    }
+    __syncthreads();
+    int run = 0;
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) {
+        int v = lane < kTopkWarps ? cnt[e][lane] : 0;
+#pragma unroll
+        for (int o = 1; o < kTopkWarps; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, v, o);
+            if (lane >= o) v += y;
+        }
+        const int before_w = __shfl_sync(0xffffffffu, v, (warp + kTopkWarps - 1) % kTopkWarps);
+        const int tot_e = __shfl_sync(0xffffffffu, v, kTopkWarps - 1);
+        const uint32_t bal = __ballot_sync(0xffffffffu, (keep >> e) & 1u);
+        if ((keep >> e) & 1u) dst[run + (warp ? before_w : 0) + __popc(bal & lt_mask)] = n0 + e * kTopkThreads + tid;
+        run += tot_e;
+    }
+}
+
 }  // namespace
 
 constexpr int kTopkSmemKeys = 40 * 1024;  // keys staged in shared memory (160 KB)
+
+template <typename... Args>
+cudaError_t launch_pdl(void (*kern)(Args...), unsigned grid, unsigned block, size_t smem, cudaStream_t stream,
+                       Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(block, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1] = {pdl_attribute()};
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
 
 cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,
                         float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, cudaStream_t stream)
 {
     if (batch <= 0) return cudaSuccess;
+    // requests up to 16 keys per thread: registers only
+    if (max_n <= 16 * kTopkThreads) {
+        auto kern = max_n <= 2 * kTopkThreads   ? topk_reg_kernel<2>
+                    : max_n <= 4 * kTopkThreads ? topk_reg_kernel<4>
+                    : max_n <= 8 * kTopkThreads ? topk_reg_kernel<8>
+                                                : topk_reg_kernel<16>;
+        return launch_pdl(kern, (unsigned)batch, kTopkThreads, 0, stream, scores, seq_off, keep_k, keep_ratio,
+                          kept_idx, out_off);
+    }
     const int keys = max_n < kTopkSmemKeys ? max_n : kTopkSmemKeys;
-    const size_t smem = (size_t)(keys > 0 ? keys : 1) * 4;
+    const size_t smem = (size_t)keys * 4;
     cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    topk_kernel<<<batch, kTopkThreads, smem, stream>>>(scores, seq_off, keep_k, keep_ratio, kept_idx, out_off,
-                                                       keys);
-    return cudaGetLastError();
+    return launch_pdl(topk_kernel, (unsigned)batch, kTopkThreads, smem, stream, scores, seq_off, keep_k, keep_ratio,
+                      kept_idx, out_off, keys);
 }
 
 }  // namespace lvs

@@ -181,6 +181,33 @@ def test_topk_request_larger_than_shared_memory_stage(sel):
     np.testing.assert_array_equal(off_d, ooff)
 
 
+@pytest.mark.parametrize("max_n", [1024, 1025, 2048, 2049, 4096, 4097, 8192, 8193])
+def test_topk_every_kernel_size_class(sel, max_n):
+    """Each request-size class of the top-k kernels (keys per thread 2/4/8/16,
+    then the shared-memory kernel) on score shapes seen in practice: softmax-
+    like values in a narrow range, coarse values with many ties, and specials."""
+    rng = np.random.Generator(np.random.PCG64(max_n))
+    n_vis = [max_n, 1, 0, int(rng.integers(1, max_n)), max_n - 1, 3]
+    so = np.concatenate([[0], np.cumsum(n_vis)]).astype(np.int32)
+    tot = int(so[-1])
+    w = _case("sizes", 1, 1, 128, "bf16", n_vis, [1] * len(n_vis))
+    s = _selector(sel, w)
+    narrow = (np.float32(1.0 / max_n) * (1 + np.float32(1e-3) * rng.standard_normal(tot))).astype(np.float32)
+    coarse = np.round(rng.standard_normal(tot), 1).astype(np.float32)
+    special = rng.choice(np.array([0.0, -0.0, np.nan, np.inf, -np.inf, 2.0, 2.0, 1e-30], np.float32), tot)
+    for scores in (narrow, coarse, special):
+        for trial in range(2):
+            keep = [int(rng.integers(0, n + 1)) for n in n_vis]
+            kept, off_d, _ = _topk_gpu(sel, s, scores, so, keep_k=keep)
+            ok, ooff = oracle.topk(so, scores, keep_k=keep)
+            np.testing.assert_array_equal(kept, ok)
+            np.testing.assert_array_equal(off_d, ooff)
+        kept, off_d, _ = _topk_gpu(sel, s, scores, so, ratio=0.3)
+        ok, ooff = oracle.topk(so, scores, keep_ratio=0.3)
+        np.testing.assert_array_equal(kept, ok)
+        np.testing.assert_array_equal(off_d, ooff)
+
+
 def test_topk_argument_errors(sel):
     w = _case("e", 1, 1, 128, "bf16", [10], [1])
     s = _selector(sel, w)
