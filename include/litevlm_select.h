@@ -190,6 +190,58 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t handle, int32_t batc
  */
 litevlm_status_t litevlm_select_check_device(litevlm_select_t handle, litevlm_stream_t stream);
 
+/*
+ * litevlm_select_score without a handle and without allocating anything.
+ * The paper has no counterpart: this is an integration entry point.
+ *
+ * Who needs it: callers that may not allocate device memory when they score,
+ * such as an inference engine that plans every buffer when a model is built
+ * and gives its plugins no allocator at run time, or a real-time pipeline that
+ * forbids allocation after start-up (cudaMalloc can block, synchronise the
+ * device, and fail on fragmented memory). These callers cannot create a handle
+ * on the hot path.
+ *
+ * Same computation, arguments and host-side checks as litevlm_select_score.
+ * A handle's config is replaced by num_q_heads, num_kv_heads, head_dim and
+ * qk_dtype, with the same rules as in litevlm_select_create. The kernel and
+ * launch shape are chosen as litevlm_select_score would choose them.
+ *
+ * Scratch: two static device arrays in this library, one per device:
+ * 4 MiB of partial scores and 64 KiB of fold tickets.
+ *   - Limit 1: total_visual / 128 + 2 * batch + 2 <= 16384.
+ *   - Limit 2: when the chosen launch splits the query heads over G > 1 CTA
+ *     groups, G * total_visual <= 1048576.
+ *   - A call beyond either limit returns LITEVLM_ERR_WORKSPACE and enqueues
+ *     nothing. Limit 1 is checked before any CUDA call.
+ *   - Each call clears the tickets it uses with cudaMemsetAsync on `stream`.
+ * Calls that overlap on one device (other streams, other host threads) share
+ * this scratch and race. Serialise them.
+ *
+ * err_d: device int32, owned by the caller. Zero it before the first call.
+ *   - Kernels OR error bits into it: 1 = a bounded wait gave up, so the scores
+ *     are not valid; 4 = a request shape reached the kernel unchecked.
+ *   - The library never reads or clears it.
+ *
+ * First call on a device: the library looks up the addresses of its static
+ * arrays with cudaGetSymbolAddress while that device is current. This may
+ * load the library's device code onto the device. The library also queries
+ * occupancy the first time it uses each kernel variant. Make this first call,
+ * with each head_dim / qk_dtype the caller will use, outside any stream
+ * capture.
+ *
+ * Errors: status codes as for litevlm_select_score (device ordinal >= 64:
+ * UNSUPPORTED). The message is available from litevlm_select_last_error(NULL)
+ * in the calling thread.
+ */
+litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                              litevlm_dtype_t qk_dtype, int32_t batch,
+                                              const void* q_text, const int32_t* text_offsets_d,
+                                              const int32_t* text_offsets_h,
+                                              const void* k_vis, const int32_t* seq_offsets_d,
+                                              const int32_t* seq_offsets_h,
+                                              float q_scale, float k_scale, float* scores, int32_t* err_d,
+                                              litevlm_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -7,6 +7,7 @@
 #include <stdint.h>
 
 #include <cstdio>
+#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -456,3 +457,166 @@ litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_
 }
 
 }  // extern "C"
+
+// ----------------------------------------------------------------------------
+// litevlm_select_score_noalloc: the score kernels with their scratch in
+// static device arrays of this library instead of a handle's workspace.
+//
+// Some callers may not allocate device memory at the moment they score: an
+// inference engine that plans every buffer of a model when it is built and
+// hands its plugins no allocator at run time, or a real-time pipeline (such
+// as an in-vehicle one) that forbids allocation after start-up because
+// cudaMalloc can block, synchronise the device and fail when memory is
+// fragmented. Such callers cannot create a handle on the hot path. This entry
+// point needs no handle: the fold partials and tickets live in the arrays
+// below (fixed size, loaded with the library's device code), the device
+// error word is the caller's, and the launch path is the one
+// litevlm_select_score takes, run on a handle built on the stack.
+// ----------------------------------------------------------------------------
+namespace {
+
+constexpr int64_t kNoAllocPartialFloats = int64_t(1) << 20;  // 4 MiB of per-head-group partial scores
+constexpr int64_t kNoAllocTickets = int64_t(1) << 14;        // 64 KiB of fold tickets
+constexpr int kNoAllocMaxDevices = 64;
+
+static __device__ __align__(256) float g_noalloc_partials[kNoAllocPartialFloats];
+static __device__ __align__(256) int32_t g_noalloc_tickets[kNoAllocTickets];
+
+struct NoAllocDevice {
+    bool ready = false;
+    int num_sms = 0;
+    float* partials = nullptr;
+    int32_t* tickets = nullptr;
+    PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    int res_capacity[3][2][17];  // by kernel family (bf16 d=128, bf16 d=64, e4m3), as in the handle
+};
+
+NoAllocDevice g_noalloc[kNoAllocMaxDevices];
+std::mutex g_noalloc_mutex;
+
+int noalloc_family(int32_t head_dim, litevlm_dtype_t dtype)
+{
+    if (dtype == LITEVLM_FP8_E4M3) return 2;
+    return head_dim == 128 ? 0 : 1;
+}
+
+// One-time setup of a device (under g_noalloc_mutex, that device current):
+// the addresses of the static arrays on it, its SM count and the TMA
+// descriptor encoder. The symbol lookup may load this library's device code
+// (and with it the arrays) onto the device.
+litevlm_status_t noalloc_setup(int dev, NoAllocDevice& d)
+{
+    if (d.ready) return LITEVLM_OK;
+    int major = 0;
+    cudaError_t e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    if (e == cudaSuccess && major != 10) return fail(nullptr, LITEVLM_ERR_UNSUPPORTED, "needs a Blackwell (sm_10x) GPU");
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
+    void* pp = nullptr;
+    void* tp = nullptr;
+    if (e == cudaSuccess) e = cudaGetSymbolAddress(&pp, g_noalloc_partials);
+    if (e == cudaSuccess) e = cudaGetSymbolAddress(&tp, g_noalloc_tickets);
+    void* fn = nullptr;
+    if (e == cudaSuccess) {
+        cudaDriverEntryPointQueryResult q;
+        e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e == cudaSuccess && (q != cudaDriverEntryPointSuccess || !fn)) e = cudaErrorNotSupported;
+    }
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(nullptr, LITEVLM_ERR_CUDA, std::string("score_noalloc setup: ") + cudaGetErrorString(e));
+    }
+    d.partials = static_cast<float*>(pp);
+    d.tickets = static_cast<int32_t*>(tp);
+    d.encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    for (auto& fam : d.res_capacity)
+        for (auto& row : fam)
+            for (int& v : row) v = -1;
+    d.ready = true;
+    return LITEVLM_OK;
+}
+
+}  // namespace
+
+extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                                         litevlm_dtype_t qk_dtype, int32_t batch, const void* q_text,
+                                                         const int32_t* text_offsets_d, const int32_t* text_offsets_h,
+                                                         const void* k_vis, const int32_t* seq_offsets_d,
+                                                         const int32_t* seq_offsets_h, float q_scale, float k_scale,
+                                                         float* scores, int32_t* err_d, litevlm_stream_t stream)
+{
+    g_create_error.clear();
+    // ---- host-only checks, before any CUDA call
+    if (num_q_heads <= 0 || num_kv_heads <= 0 || num_q_heads % num_kv_heads != 0)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
+    if (qk_dtype != LITEVLM_BF16 && qk_dtype != LITEVLM_FP8_E4M3)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "qk_dtype must be LITEVLM_BF16 or LITEVLM_FP8_E4M3");
+    if (head_dim <= 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "head_dim must be > 0");
+    if (!lvs::score_shape_supported(head_dim, qk_dtype == LITEVLM_FP8_E4M3))
+        return fail(nullptr, LITEVLM_ERR_UNSUPPORTED, "head_dim has no kernel for this dtype (bf16: 64, 128; e4m3: 128)");
+    if (batch < 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
+    if (batch == 0) return LITEVLM_OK;
+    if (!seq_offsets_h || !text_offsets_h) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "an offsets host mirror is NULL");
+    if (!err_d) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "err_d is NULL");
+    const int64_t tot_n = seq_offsets_h[batch];
+    if (seq_offsets_h[0] != 0 || tot_n < 0)
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "seq_offsets must start at 0 and be non-decreasing");
+    // fold tickets of one launch: floor(n0 / 128) + t + b < total / 128 + 2 * batch + 1
+    const int64_t n_tickets = tot_n / lvs::kTileRows + 2 * (int64_t)batch + 2;
+    if (n_tickets > kNoAllocTickets)
+        return fail(nullptr, LITEVLM_ERR_WORKSPACE,
+                    "batch too large for the static scratch: total_visual / 128 + 2 * batch + 2 must be <= 16384");
+
+    // ---- the device's static scratch
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(nullptr, LITEVLM_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(nullptr, LITEVLM_ERR_UNSUPPORTED, "device ordinal >= 64");
+    const int fam = noalloc_family(head_dim, qk_dtype);
+    litevlm_select h;
+    {
+        std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+        NoAllocDevice& d = g_noalloc[dev];
+        const litevlm_status_t s = noalloc_setup(dev, d);
+        if (s != LITEVLM_OK) return s;
+        h.device = dev;
+        h.num_sms = d.num_sms;
+        h.partials = d.partials;
+        h.counters = d.tickets;
+        h.n_counters = (size_t)kNoAllocTickets;
+        h.encode = d.encode;
+        for (int r = 0; r < 2; ++r)
+            for (int c = 0; c < 17; ++c) h.res_capacity[r][c] = d.res_capacity[fam][r][c];
+    }
+    h.err_d = err_d;
+    h.cfg.max_batch = batch;
+    h.cfg.max_total_visual = tot_n;
+    h.cfg.max_total_text = text_offsets_h[batch] > 0 ? text_offsets_h[batch] : 0;
+    h.cfg.num_q_heads = num_q_heads;
+    h.cfg.num_kv_heads = num_kv_heads;
+    h.cfg.head_dim = head_dim;
+    h.cfg.qk_dtype = qk_dtype;
+    h.cfg.flags = 0;
+
+    // ---- the plan litevlm_select_score will take, checked against the partials' size
+    int32_t plan[4];
+    litevlm_status_t s = litevlm_select_score_plan(&h, batch, text_offsets_h, seq_offsets_h, plan);
+    if (s == LITEVLM_OK && plan[3] > 1 && (int64_t)plan[3] * tot_n > kNoAllocPartialFloats)
+        s = fail(&h, LITEVLM_ERR_WORKSPACE,
+                 "head groups x total_visual exceeds the static partial-score scratch (1048576 floats)");
+    // tickets start at zero (a launch that gave up may have left some taken)
+    if (s == LITEVLM_OK && plan[3] > 1) {
+        e = cudaMemsetAsync(h.counters, 0, sizeof(int32_t) * (size_t)n_tickets, (cudaStream_t)stream);
+        if (e != cudaSuccess) s = cuda_fail(&h, e, "score_noalloc: clearing the fold tickets");
+    }
+    if (s == LITEVLM_OK)
+        s = litevlm_select_score(&h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d,
+                                 seq_offsets_h, q_scale, k_scale, scores, stream);
+    {
+        std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+        NoAllocDevice& d = g_noalloc[dev];
+        for (int r = 0; r < 2; ++r)
+            for (int c = 0; c < 17; ++c) d.res_capacity[fam][r][c] = h.res_capacity[r][c];
+    }
+    if (s != LITEVLM_OK) g_create_error = h.last_error;
+    return s;
+}

@@ -54,7 +54,8 @@ def _load():
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
     lib.litevlm_select_score_plan.argtypes = [P, i32, P, P, P]
-    for fn in ("create", "destroy", "score", "topk", "compact", "check_device", "score_plan"):
+    lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
+    for fn in ("create", "destroy", "score", "topk", "compact", "check_device", "score_plan", "score_noalloc"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -64,7 +65,7 @@ LIB = _load()
 # every symbol declared in include/litevlm_select.h
 EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
-           "litevlm_select_check_device", "litevlm_select_score_plan"]
+           "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (pass-2 products resident in TMEM)"}
 
@@ -153,6 +154,17 @@ def compact(handle: int, total_kept: int, kept_idx, src_rows: int, srcs: Sequenc
 
 def check_device(handle: int, stream=None) -> None:
     _check(LIB.litevlm_select_check_device(handle, _stream_ptr(stream)), handle)
+
+
+def score_noalloc(num_q_heads: int, num_kv_heads: int, head_dim: int, qk_dtype: str, batch: int, q_text,
+                  text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h, q_scale: float,
+                  k_scale: float, scores, err_d, stream=None) -> None:
+    """litevlm_select_score_noalloc: no handle, scratch in the library's static device arrays."""
+    to_h, so_h = _host_i32(text_offsets_h), _host_i32(seq_offsets_h)
+    _check(LIB.litevlm_select_score_noalloc(num_q_heads, num_kv_heads, head_dim, DTYPES[qk_dtype], batch,
+                                            _ptr(q_text), _ptr(text_offsets_d), _ptr(to_h), _ptr(k_vis),
+                                            _ptr(seq_offsets_d), _ptr(so_h), q_scale, k_scale, _ptr(scores),
+                                            _ptr(err_d), _stream_ptr(stream)), None)
 
 
 def score_plan(handle: int, batch: int, text_offsets_h, seq_offsets_h):
