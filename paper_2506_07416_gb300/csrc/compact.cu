@@ -4,7 +4,7 @@
 // dst[t][r] = src[t][kept_idx[r]] for every gathered tensor t, byte for byte.
 // One warp moves one kept row of every tensor: the index is read once, each
 // lane copies 16-byte vectors with streaming (evict-first) loads and stores,
-// four vectors in flight per lane. Rows whose size or pointers are not
+// up to eight vectors in flight per lane. Rows whose size or pointers are not
 // 16-byte aligned go through the byte-wise kernel. Indices outside
 // [0, src_rows) are skipped and flagged in the error word.
 
@@ -37,18 +37,16 @@ __global__ void __launch_bounds__(kGatherThreads)
             const int4* __restrict__ s = reinterpret_cast<const int4*>(g.src[t] + (int64_t)idx * rb);
             int4* __restrict__ d = reinterpret_cast<int4*>(g.dst[t] + r * rb);
             const int64_t n16 = rb >> 4;
-            int64_t c = lane;
-            for (; c + 96 < n16; c += 128) {
-                const int4 a0 = __ldcs(s + c);
-                const int4 a1 = __ldcs(s + c + 32);
-                const int4 a2 = __ldcs(s + c + 64);
-                const int4 a3 = __ldcs(s + c + 96);
-                __stcs(d + c, a0);
-                __stcs(d + c + 32, a1);
-                __stcs(d + c + 64, a2);
-                __stcs(d + c + 96, a3);
+            // up to 8 vectors per lane in flight (a 4 KB row in one round trip)
+            for (int64_t c = lane; c < n16; c += 256) {
+                int4 a[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                    if (c + 32 * u < n16) a[u] = __ldcs(s + c + 32 * u);
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                    if (c + 32 * u < n16) __stcs(d + c + 32 * u, a[u]);
             }
-            for (; c < n16; c += 32) __stcs(d + c, __ldcs(s + c));
         }
     }
 }

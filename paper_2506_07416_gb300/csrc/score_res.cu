@@ -120,26 +120,13 @@ __global__ void __launch_bounds__(kResThreads, 1)
 
     griddep_wait();
     griddep_launch_dependents();
+    // The request's offsets are loaded here and first used after the setup
+    // below (barriers, TMEM, cluster barrier), so their latency overlaps it.
     const int n0 = p.seq_off[b];
-    const int N = p.seq_off[b + 1] - n0;
+    const int n1 = p.seq_off[b + 1];
     const int t0 = p.text_off[b];
-    const int T = p.text_off[b + 1] - t0;
+    const int t1 = p.text_off[b + 1];
     const bool multi = p.groups > 1;
-    const int n2 = (T + 15) & ~15;
-    const int n_tiles = (N + kTileRows - 1) / kTileRows;
-    const int tpc = N > 0 ? (n_tiles + (int)csize - 1) / (int)csize : 0;
-    // Uniform for the whole cluster (same request). Shape errors are caught on
-    // the host; this only keeps the kernel within its buffers.
-    const int span = p.slot_cols / 2 + 32 * ((p.slot_cols / 2 + 31) / 32);  // columns the epilogue reads per slot
-    if (T > MROWS || n2 > p.slot_cols || (N > 0 && T <= 0) || (tpc > 0 && (tpc - 1) * p.slot_cols + span > kResTmemCols) ||
-        tpc > kResMaxSlots || (int)csize * p.slot_cols > L::RECV_COLS) {
-        if (threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
-        return;
-    }
-    if (N <= 0) return;
-    const int tile_begin = min(n_tiles, (int)rank * tpc);
-    const int tile_end = min(n_tiles, tile_begin + tpc);
-    const int mt = tile_end - tile_begin;
     const int G = p.hq / p.hkv;
     const int hpg = p.heads_per_group;
     const float cl = p.c_log2;
@@ -170,7 +157,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         }
         for (int i = 0; i < kResMaxSlots; ++i) {
             mbar_init(BAR(S_FULL + i), 1);
-            mbar_init(BAR(S_EMPTY + i), 256);
+            mbar_init(BAR(S_EMPTY + i), 8);  // one arrival per epilogue warp
         }
         mbar_init(BAR(DRAIN), 1);
         *abort_flag = 0;
@@ -190,6 +177,32 @@ __global__ void __launch_bounds__(kResThreads, 1)
     cluster_sync_all();
     const uint32_t tmem = *tmem_slot;
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
+
+    const int N = n1 - n0;
+    const int T = t1 - t0;
+    const int n2 = (T + 15) & ~15;
+    const int n_tiles = (N + kTileRows - 1) / kTileRows;
+    const int tpc = N > 0 ? (n_tiles + (int)csize - 1) / (int)csize : 0;
+    // Uniform for the whole cluster (same request). Shape errors are caught on
+    // the host; this only keeps the kernel within its buffers.
+    const int span = p.slot_cols / 2 + 32 * ((p.slot_cols / 2 + 31) / 32);  // columns the epilogue reads per slot
+    const bool bad_shape = T > MROWS || n2 > p.slot_cols || (N > 0 && T <= 0) ||
+                           (tpc > 0 && (tpc - 1) * p.slot_cols + span > kResTmemCols) || tpc > kResMaxSlots ||
+                           (int)csize * p.slot_cols > L::RECV_COLS;
+    if (bad_shape || N <= 0) {
+        if (bad_shape && threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
+        tc_fence_before();
+        __syncthreads();
+        if (warp == 1) {
+            tc_fence_after();
+            tmem_dealloc(tmem, kResTmemCols);
+        }
+        cluster_sync_all();
+        return;
+    }
+    const int tile_begin = min(n_tiles, (int)rank * tpc);
+    const int tile_end = min(n_tiles, tile_begin + tpc);
+    const int mt = tile_end - tile_begin;
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
@@ -472,8 +485,11 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 tmem_wait_ld();
             }
             // every slot of this head is consumed: hand them back to the MMA warp
+            // (one arrival per warp; arrivals on one barrier serialise)
             tc_fence_before();
-            for (int tl = 0; tl < mt; ++tl) mbar_arrive(BAR(S_EMPTY + tl));
+            __syncwarp();
+            if (lane == 0)
+                for (int tl = 0; tl < mt; ++tl) mbar_arrive(BAR(S_EMPTY + tl));
         }
         // ---- results: the two warpgroups' partial rows, added in a fixed order
         named_bar_sync(1, 256);

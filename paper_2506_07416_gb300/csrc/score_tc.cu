@@ -150,9 +150,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(BAR(T1_FULL + i), 1);
-            mbar_init(BAR(T1_EMPTY + i), 128);
+            mbar_init(BAR(T1_EMPTY + i), 4);   // one arrival per epilogue warp
             mbar_init(BAR(T2_FULL + i), 1);
-            mbar_init(BAR(T2_EMPTY + i), 128);
+            mbar_init(BAR(T2_EMPTY + i), 4);
         }
         for (int i = 0; i < kStatSlots; ++i) mbar_init(BAR(STATS + i), csize);
         mbar_init(BAR(DRAIN), 1);
@@ -323,7 +323,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         if (hh == NH - 1) {
                             tc_fence_before();
-                            mbar_arrive(BAR(T1_EMPTY + tb));
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(BAR(T1_EMPTY + tb));
                         }
                         if (p1_live) {
                             const int valid = N - t * kTileRows - (MROWS == 128 ? hh : phalf) * 64;
@@ -395,7 +396,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                     tc_fence_before();
-                    mbar_arrive(BAR(T2_EMPTY + tb));
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(BAR(T2_EMPTY + tb));
                     ++t2i;
                     acc_s[(t - tile_begin) * kTileRows + vrow] += (a0 + a1) + (a2 + a3);
                 }
