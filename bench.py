@@ -49,7 +49,8 @@ def parse_args():
     ap.add_argument("--workload", default="single", choices=["single", "highres", "fp8_ragged", "sweep"])
     ap.add_argument("--ratio", type=float, default=None, help="keep ratio override (sweep: 0.1/0.2/0.3/0.5)")
     ap.add_argument("--batch", type=int, default=None, help="use only the first B requests (profiling)")
-    ap.add_argument("--score-kernel", default="auto", choices=["auto", "reread", "resident"])
+    ap.add_argument("--score-kernel", default="auto", choices=["auto", "reread", "resident", "resident_1buf",
+                                                                     "resident_2buf"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="bounded CPU work for the oracle baseline")

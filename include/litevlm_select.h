@@ -71,6 +71,8 @@ typedef enum {
  * library picks the kernel and launch shape from the batch's sizes. */
 #define LITEVLM_FLAG_SCORE_REREAD 1   /* always use the kernel that streams K twice per head */
 #define LITEVLM_FLAG_SCORE_RESIDENT 2 /* use the TMEM-resident kernel whenever the shapes allow it */
+#define LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER 8 /* the same, with one TMEM head buffer only (no head overlap) */
+#define LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS 16 /* the same, two TMEM head buffers where the shapes allow it */
 
 typedef struct {
     int32_t max_batch;         /* largest batch any call will pass */
@@ -80,7 +82,7 @@ typedef struct {
     int32_t num_kv_heads;      /* Hkv, Hq % Hkv == 0 */
     int32_t head_dim;          /* d: 64 or 128 for bf16, 128 for e4m3 */
     litevlm_dtype_t qk_dtype;
-    int32_t flags;             /* 0, LITEVLM_FLAG_SCORE_REREAD or LITEVLM_FLAG_SCORE_RESIDENT */
+    int32_t flags;             /* 0 or one LITEVLM_FLAG_SCORE_* value */
 } litevlm_select_config_t;
 
 typedef struct litevlm_select* litevlm_select_t;
@@ -174,9 +176,11 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t handle, int64_t total_k
 /*
  * Launch shape litevlm_select_score would use for this batch (host only, no
  * device work; the occupancy of a kernel variant is queried once per handle).
- * plan[0] = kernel (1: K re-read per pass, 2: pass-2 products resident in
- * tensor memory), plan[1] = CTAs per thread-block cluster, plan[2] = 128-token
- * tiles per CTA, plan[3] = query-head groups (grid y). plan holds 4 int32.
+ * plan[0] = kernel (1: K re-read per pass; 2: logits resident in tensor
+ * memory, one head at a time; 3: the same with two heads in tensor memory, so
+ * one head's epilogue overlaps the next head's MMAs and statistics exchange),
+ * plan[1] = CTAs per thread-block cluster, plan[2] = 128-token tiles per CTA,
+ * plan[3] = query-head groups (grid y). plan holds 4 int32.
  * Errors as for litevlm_select_score's host-side checks.
  */
 litevlm_status_t litevlm_select_score_plan(litevlm_select_t handle, int32_t batch, const int32_t* text_offsets_h,

@@ -95,18 +95,24 @@ struct ScoreChoice {
 };
 
 // Picks the score kernel and its launch shape. Cost unit: one tile-head of
-// epilogue work; a CTA also pays a fixed ~6 units (launch, TMEM, pipeline
-// fill) and ~1 unit per head for the cluster exchange; waves of CTAs are
-// counted from the cluster occupancy of the kernel. The re-read kernel streams
-// every K tile twice, so its cost is weighted by 1.6.
+// the resident kernel with one TMEM head buffer (its MMAs, then its epilogue;
+// about 1.2 us at 64 text columns on GB300). A CTA also pays ~6 units (launch,
+// TMEM, pipeline fill) and, with one buffer, ~1 unit per head for the cluster
+// exchange. With two buffers the MMAs and the statistics exchange overlap the
+// epilogue, which then costs ~0.6 units per tile-head plus ~2.1 per head
+// (measured on GB300 at 3 tiles per CTA), and a head takes at least the time
+// its K tiles need at the CTA's share of HBM bandwidth. Waves of CTAs come from the measured
+// cluster occupancy of the kernel. The re-read kernel streams every K tile
+// twice (weight 1.6).
 ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, int max_tiles, int max_t, int row_bytes, bool fp8)
 {
     const litevlm_select_config_t& c = h->cfg;
-    const int hq = c.num_q_heads, G = c.num_q_heads / c.num_kv_heads;
+    const int hq = c.num_q_heads;
     const int mrows = max_t <= 64 ? 64 : 128;
     const int slot_cols = (max_t + 15) & ~15;
-    const int R = lvs::res_max_tiles(slot_cols);
     const int cmax = lvs::res_max_cluster(row_bytes, slot_cols);
+    const double unit_s = 1.17e-6, hbm_bytes_per_s = 6.8e12;
+    const double tile_bytes = (double)lvs::kTileRows * row_bytes;
     ScoreChoice best{false, lvs::plan_score(batch, max_tiles, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, h->num_sms)};
     double best_cost = 1e300;
     {
@@ -118,28 +124,45 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, int max_tiles, in
         best_cost = 1.6 * waves * ((double)pl.tiles_per_cta * hpg + 6.0 + hpg + (pl.groups > 1 ? 2.0 : 0.0));
     }
     if (c.flags == LITEVLM_FLAG_SCORE_REREAD) return best;
-    if (c.flags == LITEVLM_FLAG_SCORE_RESIDENT) best_cost = 1e300;
-    for (int cl = 1; cl <= cmax; ++cl) {
-        const int tpc = (max_tiles + cl - 1) / cl;
-        if (tpc > R) continue;
-        if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;  // an idle rank
-        int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
-        if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
-        if (cap <= 0) continue;
-        for (int g = 1; g <= hq; ++g) {
-            if (hq % g) continue;
-            const int hpg = hq / g;
-            const long long ctas = (long long)batch * cl * g;
-            const long long waves = (ctas + cap - 1) / cap;
-            const double per = (double)tpc * hpg + 6.0 + (cl > 1 ? 1.0 : 0.25) * hpg + (g > 1 ? 2.0 : 0.0);
-            const double cost = (double)waves * per;
-            if (cost < best_cost - 1e-9) {
-                best_cost = cost;
-                best = ScoreChoice{true, lvs::ScorePlan{cl, tpc, g}};
+    if (c.flags == LITEVLM_FLAG_SCORE_RESIDENT || c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
+        c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
+        best_cost = 1e300;
+    for (int nb = 1; nb <= 2; ++nb) {
+        if (nb == 2 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER) continue;
+        if (nb == 1 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) continue;
+        const int R = lvs::res_max_tiles(slot_cols, nb);
+        for (int cl = 1; cl <= cmax; ++cl) {
+            const int tpc = (max_tiles + cl - 1) / cl;
+            if (tpc > R) continue;
+            if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;  // an idle rank
+            int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
+            if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
+            if (cap <= 0) continue;
+            for (int g = 1; g <= hq; ++g) {
+                if (hq % g) continue;
+                const int hpg = hq / g;
+                if (nb == 2 && hpg < 2) continue;  // nothing to overlap
+                const long long ctas = (long long)batch * cl * g;
+                const long long waves = (ctas + cap - 1) / cap;
+                const double active = (double)(ctas < cap ? ctas : cap);
+                double per_head;
+                if (nb == 1) {
+                    per_head = (double)tpc + (cl > 1 ? 1.0 : 0.25);
+                } else {
+                    const double stream = tpc * tile_bytes * active / hbm_bytes_per_s / unit_s;
+                    per_head = 0.6 * tpc + 2.1;
+                    if (stream > per_head) per_head = stream;
+                }
+                const double cost = (double)waves * (6.0 + (g > 1 ? 2.0 : 0.0) + hpg * per_head);
+                if (cost < best_cost - 1e-9) {
+                    best_cost = cost;
+                    lvs::ScorePlan pl{cl, tpc, g};
+                    pl.res_nb = nb;
+                    best = ScoreChoice{true, pl};
+                }
             }
         }
     }
-    (void)G;
     return best;
 }
 
@@ -180,7 +203,8 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
     if (c->qk_dtype != LITEVLM_BF16 && c->qk_dtype != LITEVLM_FP8_E4M3)
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "qk_dtype must be LITEVLM_BF16 or LITEVLM_FP8_E4M3");
-    if (c->flags != 0 && c->flags != LITEVLM_FLAG_SCORE_REREAD && c->flags != LITEVLM_FLAG_SCORE_RESIDENT)
+    if (c->flags != 0 && c->flags != LITEVLM_FLAG_SCORE_REREAD && c->flags != LITEVLM_FLAG_SCORE_RESIDENT &&
+        c->flags != LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER && c->flags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "flags must be 0 or one LITEVLM_FLAG_SCORE_* value");
     if (c->head_dim <= 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "head_dim must be > 0");
     if (!lvs::score_shape_supported(c->head_dim, c->qk_dtype == LITEVLM_FP8_E4M3))
@@ -293,7 +317,7 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, co
     if (batch == 0 || sh.tot_n == 0) return LITEVLM_OK;
     const bool fp8 = h->cfg.qk_dtype == LITEVLM_FP8_E4M3;
     const ScoreChoice ch = choose_score_kernel(h, batch, sh.max_tiles, sh.max_t, h->cfg.head_dim * (fp8 ? 1 : 2), fp8);
-    plan[0] = ch.resident ? 2 : 1;
+    plan[0] = ch.resident ? 1 + ch.plan.res_nb : 1;
     plan[1] = ch.plan.cluster;
     plan[2] = ch.plan.tiles_per_cta;
     plan[3] = ch.plan.groups;

@@ -44,7 +44,8 @@ struct ScoreLaunch {
     int32_t heads_per_group;
     int32_t groups;
     int32_t ctas_per_request; // cluster size * groups
-    int32_t slot_cols;        // resident kernel: TMEM columns per pass-2 slot (T rounded up to 16, max over batch)
+    int32_t slot_cols;        // resident kernel: TMEM columns per slot (T rounded up to 16, max over batch)
+    int32_t res_nb;           // resident kernel: TMEM head buffers, 1 or 2 (2: heads overlap)
     float c_log2;             // q_scale * k_scale / sqrt(d) * log2(e)
     long long wait_budget;
 };
@@ -53,6 +54,7 @@ struct ScorePlan {
     int cluster;              // CTAs per (request, head group)
     int tiles_per_cta;
     int groups;               // head groups (grid.y); partial rows when > 1
+    int res_nb = 1;           // resident kernel: TMEM head buffers
 };
 
 // Host helpers (score_tc.cu)
@@ -62,7 +64,7 @@ cudaError_t launch_score(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const
 bool score_shape_supported(int head_dim, bool fp8);
 
 // score_res.cu (one contraction per K tile and head, logits resident in TMEM)
-int res_max_tiles(int slot_cols);                  // tiles per CTA that fit in tensor memory
+int res_max_tiles(int slot_cols, int nb);          // tiles per CTA that fit in tensor memory with nb head buffers
 int res_max_cluster(int row_bytes, int slot_cols); // cluster size limit of the statistics buffer
 int res_cluster_capacity(int row_bytes, bool fp8, int mrows, int cluster);
 cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,

@@ -46,19 +46,22 @@ namespace {
 constexpr int kResThreads = 320;
 constexpr int kResTmemCols = 512;
 constexpr int kResMaxSlots = 16;
+constexpr int kBufSlots = kResMaxSlots / 2;  // slots per buffer with two TMEM buffers
+constexpr int kBufCols = kResTmemCols / 2;   // columns per buffer with two TMEM buffers
+constexpr int kStatSlots = 4;                // heads whose statistics may be in flight
 
 template <int ROW_BYTES, int MROWS>
 struct ResLayout {
     static constexpr int KB = ROW_BYTES / 128;
     static constexpr int TILE_BYTES = kTileRows * ROW_BYTES;
     static constexpr int Q_BYTES = MROWS * ROW_BYTES;
-    // statistics receive buffer: [2 heads][cluster rank][column] (m, l); cluster size
-    // times slot columns must fit RECV_COLS
-    static constexpr int RECV_COLS = ROW_BYTES == 256 ? 512 : 1024;
+    // statistics receive buffer: [kStatSlots heads][cluster rank][column] (m, l);
+    // cluster size times slot columns must fit RECV_COLS
+    static constexpr int RECV_COLS = ROW_BYTES == 256 ? 640 : 1024;
     static constexpr int ACC_BYTES = 2 * kResMaxSlots * kTileRows * 4;  // per warpgroup partial rows
-    static constexpr int SCR_BYTES = 2 * 2 * 4 * 64 * 4;                // [max|sum][wg][warp][64 cols]
-    static constexpr int NBAR_FIXED = 2 * 2 + 2 * kResMaxSlots + 2 + 1;
-    static constexpr int FIXED = 2 * Q_BYTES + ACC_BYTES + SCR_BYTES + 2 * RECV_COLS * 8 + 2 * 64 * 4 +
+    static constexpr int SCR_BYTES = 3 * 2 * 4 * 64 * 4;  // [max of head s & 1 (2) | sum][wg][warp][64 cols]
+    static constexpr int NBAR_FIXED = 2 * 2 + 2 * kResMaxSlots + kStatSlots + 1;
+    static constexpr int FIXED = 2 * Q_BYTES + ACC_BYTES + SCR_BYTES + kStatSlots * RECV_COLS * 8 + 4 * 64 * 4 +
                                  kResMaxSlots * 4 + (NBAR_FIXED + 2 * 10) * 8 + 64 + 1024;
     static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
     static constexpr int kStages = STAGES_FIT > 10 ? 10 : STAGES_FIT;
@@ -67,8 +70,9 @@ struct ResLayout {
     static constexpr int OFF_ACC = OFF_Q + 2 * Q_BYTES;
     static constexpr int OFF_SCR = OFF_ACC + ACC_BYTES;
     static constexpr int OFF_RECV = OFF_SCR + SCR_BYTES;
-    static constexpr int OFF_B2 = OFF_RECV + 2 * RECV_COLS * 8;
-    static constexpr int OFF_FLAGS = OFF_B2 + 2 * 64 * 4;  // b per warpgroup column, +inf past its columns
+    static constexpr int OFF_B2 = OFF_RECV + kStatSlots * RECV_COLS * 8;
+    static constexpr int OFF_MC = OFF_B2 + 2 * 64 * 4;     // column weights per warpgroup column
+    static constexpr int OFF_FLAGS = OFF_MC + 2 * 64 * 4;  // CTA column max * c per warpgroup column
     static constexpr int OFF_BAR = OFF_FLAGS + kResMaxSlots * 4;
     static constexpr int NBAR = 2 * kStages + NBAR_FIXED;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
@@ -135,14 +139,15 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const uint32_t bar0 = base + L::OFF_BAR;
     auto BAR = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
     const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + 2, S_FULL = Q_EMPTY + 2,
-              S_EMPTY = S_FULL + kResMaxSlots, STATS = S_EMPTY + kResMaxSlots, DRAIN = STATS + 2;
+              S_EMPTY = S_FULL + kResMaxSlots, STATS = S_EMPTY + kResMaxSlots, DRAIN = STATS + kStatSlots;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
     float* acc_s = reinterpret_cast<float*>(smem + L::OFF_ACC);
-    float* scr_max = reinterpret_cast<float*>(smem + L::OFF_SCR);        // [wg][warp][64]
-    float* scr_sum = scr_max + 2 * 4 * 64;                                // [wg][warp][64]
+    float* scr_max = reinterpret_cast<float*>(smem + L::OFF_SCR);        // [head & 1][wg][warp][64]
+    float* scr_sum = scr_max + 2 * 2 * 4 * 64;                            // [wg][warp][64]
     const float2* recv = reinterpret_cast<const float2*>(smem + L::OFF_RECV);
     float* b2_s = reinterpret_cast<float*>(smem + L::OFF_B2);
+    float* mc_s = reinterpret_cast<float*>(smem + L::OFF_MC);
     volatile int* fold_flags = reinterpret_cast<volatile int*>(smem + L::OFF_FLAGS);
 
     if (threadIdx.x == 0) {
@@ -153,8 +158,8 @@ __global__ void __launch_bounds__(kResThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(BAR(Q_FULL + i), 1);
             mbar_init(BAR(Q_EMPTY + i), 1);
-            mbar_init(BAR(STATS + i), 1);  // the local arm; peers complete bytes
         }
+        for (int i = 0; i < kStatSlots; ++i) mbar_init(BAR(STATS + i), 1);  // the local arm; peers complete bytes
         for (int i = 0; i < kResMaxSlots; ++i) {
             mbar_init(BAR(S_FULL + i), 1);
             mbar_init(BAR(S_EMPTY + i), 8);  // one arrival per epilogue warp
@@ -186,9 +191,11 @@ __global__ void __launch_bounds__(kResThreads, 1)
     // Uniform for the whole cluster (same request). Shape errors are caught on
     // the host; this only keeps the kernel within its buffers.
     const int span = p.slot_cols / 2 + 32 * ((p.slot_cols / 2 + 31) / 32);  // columns the epilogue reads per slot
+    const int nb = p.res_nb == 2 ? 2 : 1;
+    const int buf_cols = nb == 2 ? kBufCols : kResTmemCols;
     const bool bad_shape = T > MROWS || n2 > p.slot_cols || (N > 0 && T <= 0) ||
-                           (tpc > 0 && (tpc - 1) * p.slot_cols + span > kResTmemCols) || tpc > kResMaxSlots ||
-                           (int)csize * p.slot_cols > L::RECV_COLS;
+                           (tpc > 0 && (tpc - 1) * p.slot_cols + span > buf_cols) ||
+                           tpc > (nb == 2 ? kBufSlots : kResMaxSlots) || (int)csize * p.slot_cols > L::RECV_COLS;
     if (bad_shape || N <= 0) {
         if (bad_shape && threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
         tc_fence_before();
@@ -252,15 +259,18 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 bool ok = true;
                 for (int s = 0; s < hpg && ok; ++s) {
                     const int qb = s & 1;
+                    const int buf = nb == 2 ? (s & 1) : 0;
+                    const uint32_t use = nb == 2 ? (uint32_t)(s >> 1) : (uint32_t)s;  // earlier heads in this buffer
                     if (!wait_phase(BAR(Q_FULL + qb), (s >> 1) & 1, ctl)) break;
                     tc_fence_after();
                     const uint32_t qaddr = base + L::OFF_Q + qb * L::Q_BYTES;
                     for (int tl = 0; tl < mt; ++tl) {
+                        const int sl = buf * kBufSlots + tl;
                         if (!wait_phase(BAR(K_FULL + ks), kph, ctl)) { ok = false; break; }
-                        if (!wait_phase(BAR(S_EMPTY + tl), ((uint32_t)s & 1u) ^ 1u, ctl)) { ok = false; break; }
+                        if (!wait_phase(BAR(S_EMPTY + sl), (use & 1u) ^ 1u, ctl)) { ok = false; break; }
                         tc_fence_after();
                         const uint32_t kaddr = base + L::OFF_K + ks * L::TILE_BYTES;
-                        const uint32_t d = tmem + (uint32_t)(tl * scols);
+                        const uint32_t d = tmem + (uint32_t)(buf * kBufCols + tl * scols);
 #pragma unroll
                         for (int st = 0; st < KSTEPS; ++st) {
                             const uint32_t qoff = (st >> 2) * (MROWS * 128) + (st & 3) * 32;
@@ -268,7 +278,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                             if (FP8) mma_f8(d, sdesc_k_sw128(kaddr + koff), sdesc_k_sw128(qaddr + qoff), idesc, st > 0);
                             else mma_f16(d, sdesc_k_sw128(kaddr + koff), sdesc_k_sw128(qaddr + qoff), idesc, st > 0);
                         }
-                        mma_commit(BAR(S_FULL + tl));
+                        mma_commit(BAR(S_FULL + sl));
                         mma_commit(BAR(K_EMPTY + ks));
                         if (++ks == kStages) { ks = 0; kph ^= 1; }
                     }
@@ -284,10 +294,14 @@ __global__ void __launch_bounds__(kResThreads, 1)
     } else {
         // ------------------------------------------------------------ epilogue (2 warpgroups)
         // Control flow is identical for every thread of a warpgroup (named
-        // barriers); after an abort every wait returns at once. Every
-        // warp-synchronous instruction (tcgen05.ld, redux.sync, shuffles) is
-        // executed unconditionally: always 32 columns per chunk, columns past
-        // the warpgroup's range masked arithmetically.
+        // barriers); after an abort every wait returns at once. Warp-synchronous
+        // instructions (tcgen05.ld, redux.sync, shuffles) run under branches
+        // that are uniform in the CTA only: always 32 columns per chunk, columns
+        // past the warpgroup's range masked arithmetically.
+        // Iteration i runs A and B of head i and sends its statistics, then C of
+        // head i - 1 with two TMEM buffers (the statistics of head i - 1 had a
+        // whole A + B to travel, and the MMAs of head i + 1 fill the other buffer
+        // while C reads it, slot by slot), or C of head i with one buffer.
         const int wg = (warp - 2) >> 2;
         const int quad = warp & 3;
         const int et = threadIdx.x - 64;               // 0..255
@@ -299,16 +313,28 @@ __global__ void __launch_bounds__(kResThreads, 1)
         const int c_begin = wg * h2;
         const int nch = (h2 + 31) >> 5;
         float* accw = acc_s + wg * kResMaxSlots * kTileRows;
-        float* smax = scr_max + wg * 4 * 64;
         float* ssum = scr_sum + wg * 4 * 64;
         float* b2w = b2_s + wg * 64;                   // weight of column c_begin + c, 0 for c >= h2 or >= T
+        float* mcw = mc_s + wg * 64;                   // CTA column max * c of column c_begin + c
         const uint32_t recv_base = base + L::OFF_RECV;
         const uint32_t tcol = tmem + lane_off;
         for (int tl = 0; tl < mt; ++tl) accw[tl * kTileRows + vrow] = 0.f;
         auto lane_valid = [&](int tl) { return tl < mt && (tile_begin + tl) * kTileRows + vrow < N; };
+        // slot tl of buffer b is read by this warp: hand it back to the MMA warp
+        // (one arrival per warp and slot)
+        auto release = [&](int b_, int tl_) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(BAR(S_EMPTY + b_ * kBufSlots + tl_));
+        };
 
-        for (int s = 0; s < hpg; ++s) {
-            const int slot = s & 1;
+        // A (and the column maxima) of head s
+        auto front_a = [&](const int s) {
+            const int buf = nb == 2 ? (s & 1) : 0;
+            const uint32_t use = nb == 2 ? (uint32_t)(s >> 1) : (uint32_t)s;
+            const int slot = s & (kStatSlots - 1);
+            const uint32_t tbuf = tcol + (uint32_t)(buf * kBufCols);
+            float* smax = scr_max + ((s & 1) * 2 + wg) * 4 * 64;
             if (et == 0) mbar_arrive_expect_tx(BAR(STATS + slot), (uint32_t)(csize * n2 * 8));
             for (int ch = 0; ch < nch; ++ch) {
                 const int cw = min(32, h2 - 32 * ch);
@@ -320,28 +346,28 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 {
                     float va[32], vb[32];
                     if (ch == 0 && mt > 0) {  // a rank without tiles gets no MMA
-                        wait_phase(BAR(S_FULL + 0), (uint32_t)s & 1u, ctl);
+                        wait_phase(BAR(S_FULL + buf * kBufSlots), use & 1u, ctl);
                         tc_fence_after();
                     }
-                    tmem_ld32(tcol + col0, va);
+                    tmem_ld32(tbuf + col0, va);
                     for (int tl = 0; tl < mt; tl += 2) {
                         const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
                         tmem_wait_ld();
                         if (ch == 0 && tl + 1 < mt) {
-                            wait_phase(BAR(S_FULL + t1), (uint32_t)s & 1u, ctl);
+                            wait_phase(BAR(S_FULL + buf * kBufSlots + t1), use & 1u, ctl);
                             tc_fence_after();
                         }
-                        tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
+                        tmem_ld32(tbuf + (uint32_t)(t1 * scols) + col0, vb);
                         if (lane_valid(tl)) {
 #pragma unroll
                             for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], va[c]);
                         }
                         tmem_wait_ld();
                         if (ch == 0 && tl + 2 < mt) {
-                            wait_phase(BAR(S_FULL + t2), (uint32_t)s & 1u, ctl);
+                            wait_phase(BAR(S_FULL + buf * kBufSlots + t2), use & 1u, ctl);
                             tc_fence_after();
                         }
-                        tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
+                        tmem_ld32(tbuf + (uint32_t)(t2 * scols) + col0, va);
                         if (lane_valid(tl + 1)) {
 #pragma unroll
                             for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], vb[c]);
@@ -358,23 +384,26 @@ __global__ void __launch_bounds__(kResThreads, 1)
                             make_float4(cm[c], cm[c + 1], cm[c + 2], cm[c + 3]);
                 }
                 named_bar_sync(wg_bar, 128);
-                float mc[32];  // CTA-local column max * c (columns past cw: garbage, never used)
+                // CTA-local column max * c, once per column, read back by B from shared
+                // memory (keeps 32 registers per thread free in B)
+                if (wt < 32) {
+                    float m = smax[32 * ch + wt];
 #pragma unroll
-                for (int c = 0; c < 32; c += 4) {
-                    float4 m4 = *reinterpret_cast<const float4*>(smax + 32 * ch + c);
-#pragma unroll
-                    for (int q = 1; q < 4; ++q) {
-                        const float4 o = *reinterpret_cast<const float4*>(smax + q * 64 + 32 * ch + c);
-                        m4.x = fmaxf(m4.x, o.x);
-                        m4.y = fmaxf(m4.y, o.y);
-                        m4.z = fmaxf(m4.z, o.z);
-                        m4.w = fmaxf(m4.w, o.w);
-                    }
-                    mc[c] = m4.x * cl;
-                    mc[c + 1] = m4.y * cl;
-                    mc[c + 2] = m4.z * cl;
-                    mc[c + 3] = m4.w * cl;
+                    for (int q = 1; q < 4; ++q) m = fmaxf(m, smax[q * 64 + 32 * ch + wt]);
+                    mcw[32 * ch + wt] = m * cl;  // columns past cw: garbage, never used
                 }
+                named_bar_sync(wg_bar, 128);
+            }
+        };
+        // B of head s: e written back, column sums, statistics sent to the cluster
+        auto front_b = [&](const int s) {
+            const int buf = nb == 2 ? (s & 1) : 0;
+            const int slot = s & (kStatSlots - 1);
+            const uint32_t tbuf = tcol + (uint32_t)(buf * kBufCols);
+            float* smax = scr_max + ((s & 1) * 2 + wg) * 4 * 64;
+            for (int ch = 0; ch < nch; ++ch) {
+                const int cw = min(32, h2 - 32 * ch);
+                const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
                 // ---- B: e = 2^(s*c - m*c) written back over the logits (this warpgroup's
                 // columns only); per-thread column sums of e, then over the warp's lanes
                 float sm[32];
@@ -382,15 +411,25 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 for (int c = 0; c < 32; ++c) sm[c] = 0.f;
                 for (int tl = 0; tl < mt; ++tl) {
                     float v[32];
-                    const uint32_t ta = tcol + (uint32_t)(tl * scols) + col0;
+                    const uint32_t ta = tbuf + (uint32_t)(tl * scols) + col0;
                     tmem_ld32(ta, v);
                     tmem_wait_ld();
                     const bool ok = lane_valid(tl);
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) {
-                        const float e = ok ? ex2(fmaf(v[c], cl, -mc[c])) : 0.f;
-                        v[c] = e;
-                        sm[c] += e;
+                    for (int c = 0; c < 32; c += 4) {
+                        const float4 m4 = *reinterpret_cast<const float4*>(mcw + 32 * ch + c);
+                        const float e0 = ok ? ex2(fmaf(v[c], cl, -m4.x)) : 0.f;
+                        const float e1 = ok ? ex2(fmaf(v[c + 1], cl, -m4.y)) : 0.f;
+                        const float e2 = ok ? ex2(fmaf(v[c + 2], cl, -m4.z)) : 0.f;
+                        const float e3 = ok ? ex2(fmaf(v[c + 3], cl, -m4.w)) : 0.f;
+                        v[c] = e0;
+                        v[c + 1] = e1;
+                        v[c + 2] = e2;
+                        v[c + 3] = e3;
+                        sm[c] += e0;
+                        sm[c + 1] += e1;
+                        sm[c + 2] += e2;
+                        sm[c + 3] += e3;
                     }
                     tmem_st_cols(ta, v, cw);
                 }
@@ -414,25 +453,28 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 }
             }
             tmem_wait_st();
-            // ---- merge the cluster's statistics of this head (rank order) into the
+        };
+        // statistics merge and C of head s; slots go back to the MMA warp as they are read
+        auto back = [&](const int s) {
+            const int buf = nb == 2 ? (s & 1) : 0;
+            const int slot = s & (kStatSlots - 1);
+            const uint32_t tbuf = tcol + (uint32_t)(buf * kBufCols);
+            const float* smax = scr_max + ((s & 1) * 2 + wg) * 4 * 64;
+            // merge the cluster's statistics of this head (rank order) into the
             // column weights w = 2^(m_local*c - b), b = M*c + log2(L); 0 for unused columns
-            wait_phase_cluster(BAR(STATS + slot), (uint32_t)(s >> 1) & 1u, ctl);
+            wait_phase_cluster(BAR(STATS + slot), (uint32_t)(s / kStatSlots) & 1u, ctl);
             if (wt < 64) {
                 const int col = c_begin + wt;
                 float wval = 0.f;
                 if (wt < h2 && col < T) {
-                    float2 st[kMaxCluster];
-#pragma unroll
-                    for (int r = 0; r < kMaxCluster; ++r)
-                        if (r < (int)csize) st[r] = recv[(slot * (int)csize + r) * scols + col];
+                    const float2* rs = recv + (slot * (int)csize) * scols + col;  // rank r at rs[r * scols]
                     float M = -INFINITY;
-#pragma unroll
-                    for (int r = 0; r < kMaxCluster; ++r)
-                        if (r < (int)csize) M = fmaxf(M, st[r].x);
+                    for (int r = 0; r < (int)csize; ++r) M = fmaxf(M, rs[r * scols].x);
                     float Ls = 0.f;
-#pragma unroll
-                    for (int r = 0; r < kMaxCluster; ++r)
-                        if (r < (int)csize && st[r].y > 0.f) Ls += st[r].y * ex2((st[r].x - M) * cl);
+                    for (int r = 0; r < (int)csize; ++r) {
+                        const float2 v2 = rs[r * scols];
+                        if (v2.y > 0.f) Ls += v2.y * ex2((v2.x - M) * cl);
+                    }
                     const float b = fmaf(M, cl, __log2f(Ls));
                     float mloc = smax[wt];  // this CTA's column max: the e values' reference
 #pragma unroll
@@ -442,10 +484,12 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 b2w[wt] = wval;
             }
             named_bar_sync(wg_bar, 128);
-            // ---- C: per-visual-token sums of e * w over this warpgroup's columns
+            // ---- C: per-visual-token sums of e * w over this warpgroup's columns;
+            // each slot goes back to the MMA warp after its last chunk is read
             for (int ch = 0; ch < nch; ++ch) {
                 const int cw = min(32, h2 - 32 * ch);
                 const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
+                const bool last = ch == nch - 1;
                 float wv[32];
 #pragma unroll
                 for (int c = 0; c < 32; c += 4) {
@@ -456,11 +500,11 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     wv[c + 3] = w4.w;
                 }
                 float va[32], vb[32];
-                tmem_ld32(tcol + col0, va);
+                if (mt > 0) tmem_ld32(tbuf + col0, va);
                 for (int tl = 0; tl < mt; tl += 2) {
-                    const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
-                    tmem_wait_ld();
-                    tmem_ld32(tcol + (uint32_t)(t1 * scols) + col0, vb);
+                    tmem_wait_ld();  // va: slot tl
+                    if (last) release(buf, tl);
+                    if (tl + 1 < mt) tmem_ld32(tbuf + (uint32_t)((tl + 1) * scols) + col0, vb);
                     float a0 = 0.f, a1 = 0.f;
 #pragma unroll
                     for (int c = 0; c < 32; c += 2) {
@@ -470,26 +514,40 @@ __global__ void __launch_bounds__(kResThreads, 1)
                         }
                     }
                     accw[tl * kTileRows + vrow] += a0 + a1;
-                    tmem_wait_ld();
-                    tmem_ld32(tcol + (uint32_t)(t2 * scols) + col0, va);
-                    a0 = a1 = 0.f;
+                    if (tl + 1 < mt) {
+                        tmem_wait_ld();  // vb: slot tl + 1
+                        if (last) release(buf, tl + 1);
+                        if (tl + 2 < mt) tmem_ld32(tbuf + (uint32_t)((tl + 2) * scols) + col0, va);
+                        a0 = a1 = 0.f;
 #pragma unroll
-                    for (int c = 0; c < 32; c += 2) {
-                        if (c < cw) {
-                            a0 = fmaf(vb[c], wv[c], a0);
-                            a1 = fmaf(vb[c + 1], wv[c + 1], a1);
+                        for (int c = 0; c < 32; c += 2) {
+                            if (c < cw) {
+                                a0 = fmaf(vb[c], wv[c], a0);
+                                a1 = fmaf(vb[c + 1], wv[c + 1], a1);
+                            }
                         }
+                        accw[(tl + 1) * kTileRows + vrow] += a0 + a1;
                     }
-                    if (tl + 1 < mt) accw[(tl + 1) * kTileRows + vrow] += a0 + a1;
                 }
-                tmem_wait_ld();
             }
-            // every slot of this head is consumed: hand them back to the MMA warp
-            // (one arrival per warp; arrivals on one barrier serialise)
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0)
-                for (int tl = 0; tl < mt; ++tl) mbar_arrive(BAR(S_EMPTY + tl));
+        };
+
+        // One buffer: A, B, C of each head in turn. Two buffers: iteration i runs
+        // A of head i, then C of head i - 1 (its statistics travelled during A),
+        // which frees the other buffer so the MMAs of head i + 1 run under B of
+        // head i.
+        if (nb == 2) {
+            for (int it = 0; it <= hpg; ++it) {
+                if (it < hpg) front_a(it);
+                if (it >= 1) back(it - 1);
+                if (it < hpg) front_b(it);
+            }
+        } else {
+            for (int s = 0; s < hpg; ++s) {
+                front_a(s);
+                front_b(s);
+                back(s);
+            }
         }
         // ---- results: the two warpgroups' partial rows, added in a fixed order
         named_bar_sync(1, 256);
@@ -574,13 +632,14 @@ int res_capacity(int cluster)
 
 // Tiles per CTA: the epilogue reads 32 columns per chunk, so the last slot's
 // padded read, (r - 1) * slot_cols + slot_cols / 2 + 32 * chunks, must stay
-// within the 512 TMEM columns.
-int res_max_tiles(int slot_cols)
+// within the 512 TMEM columns (256 per buffer with two head buffers).
+int res_max_tiles(int slot_cols, int nb)
 {
     if (slot_cols <= 0) return 0;
     const int h2 = slot_cols / 2, span = h2 + 32 * ((h2 + 31) / 32);
-    int r = kResMaxSlots;
-    while (r > 0 && (r - 1) * slot_cols + span > kResTmemCols) --r;
+    const int cols = nb == 2 ? kBufCols : kResTmemCols;
+    int r = nb == 2 ? kBufSlots : kResMaxSlots;
+    while (r > 0 && (r - 1) * slot_cols + span > cols) --r;
     return r;
 }
 
@@ -605,6 +664,7 @@ cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm
                                   cudaStream_t stream)
 {
     ScoreLaunch q = p;
+    q.res_nb = plan.res_nb;
     q.groups = plan.groups;
     q.heads_per_group = p.hq / plan.groups;
     q.ctas_per_request = plan.cluster * plan.groups;

@@ -66,8 +66,9 @@ LIB = _load()
 EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
            "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc"]
-FLAGS = {"auto": 0, "reread": 1, "resident": 2}
-KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (pass-2 products resident in TMEM)"}
+FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
+KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
+           3: "score_res (logits resident in TMEM, two heads overlapped)"}
 
 
 def _check(rc: int, handle) -> None:
