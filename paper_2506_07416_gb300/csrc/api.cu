@@ -6,6 +6,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <algorithm>
 #include <cstdio>
 #include <mutex>
 #include <new>
@@ -25,6 +26,15 @@ struct litevlm_select {
     int32_t* err_d = nullptr;   // device error word (bits lvs::kErr*)
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     int res_capacity[2][17];  // resident score kernel: CTAs at once per cluster size, by pass-1 rows (64/128); -1 unknown
+    // last score-kernel choices, keyed by a hash of the batch shape (planning walks every plan)
+    struct PlanMemo {
+        uint64_t key = 0;
+        bool used = false;
+        bool resident = false;
+        lvs::ScorePlan plan{1, 1, 1};
+    } plan_memo[4];
+    int plan_memo_next = 0;
+    std::vector<int> tiles_desc;  // scratch of the planner for batches above 4096 requests (host)
     std::string last_error;
 };
 
@@ -104,65 +114,93 @@ struct ScoreChoice {
 // its K tiles need at the CTA's share of HBM bandwidth. Waves of CTAs come from the measured
 // cluster occupancy of the kernel. The re-read kernel streams every K tile
 // twice (weight 1.6).
-ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, int max_tiles, int max_t, int row_bytes, bool fp8)
+ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* seq_offsets_h, int max_t, int row_bytes,
+                                bool fp8)
 {
     const litevlm_select_config_t& c = h->cfg;
     const int hq = c.num_q_heads;
     const int mrows = max_t <= 64 ? 64 : 128;
     const int slot_cols = (max_t + 15) & ~15;
+    // the batch's tiles per request, largest first; the memo key hashes them
+    int td_small[4096];
+    int* td = td_small;
+    if (batch > 4096) {
+        h->tiles_desc.resize((size_t)batch);
+        td = h->tiles_desc.data();
+    }
+    for (int b = 0; b < batch; ++b) td[b] = (seq_offsets_h[b + 1] - seq_offsets_h[b] + lvs::kTileRows - 1) / lvs::kTileRows;
+    std::sort(td, td + batch, [](int x, int y) { return x > y; });
+    uint64_t key = 1469598103934665603ull;
+    auto mix = [&](uint64_t v) { key = (key ^ v) * 1099511628211ull; };
+    mix((uint64_t)batch);
+    mix((uint64_t)max_t);
+    mix((uint64_t)hq);
+    mix((uint64_t)c.num_kv_heads);
+    mix((uint64_t)row_bytes);
+    mix((uint64_t)c.flags);
+    for (int b = 0; b < batch; ++b) mix((uint64_t)td[b]);
+    for (const auto& m : h->plan_memo)
+        if (m.used && m.key == key) return ScoreChoice{m.resident, m.plan};
+    const lvs::BatchTiles bt{td, batch};
+
     const int cmax = lvs::res_max_cluster(row_bytes, slot_cols);
     const double unit_s = 1.17e-6, hbm_bytes_per_s = 6.8e12;
     const double tile_bytes = (double)lvs::kTileRows * row_bytes;
-    ScoreChoice best{false, lvs::plan_score(batch, max_tiles, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, h->num_sms)};
-    double best_cost = 1e300;
-    {
-        const lvs::ScorePlan& pl = best.plan;
-        const int hpg = hq / pl.groups;
-        int cap = pl.cluster <= 2 ? h->num_sms : (pl.cluster <= 4 ? h->num_sms * 144 / 152 : h->num_sms * 112 / 152);
-        const long long ctas = (long long)batch * pl.cluster * pl.groups;
-        const long long waves = (ctas + cap - 1) / cap;
-        best_cost = 1.6 * waves * ((double)pl.tiles_per_cta * hpg + 6.0 + hpg + (pl.groups > 1 ? 2.0 : 0.0));
-    }
-    if (c.flags == LITEVLM_FLAG_SCORE_REREAD) return best;
-    if (c.flags == LITEVLM_FLAG_SCORE_RESIDENT || c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
-        c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
-        best_cost = 1e300;
-    for (int nb = 1; nb <= 2; ++nb) {
-        if (nb == 2 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER) continue;
-        if (nb == 1 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) continue;
-        const int R = lvs::res_max_tiles(slot_cols, nb);
-        for (int cl = 1; cl <= cmax; ++cl) {
-            const int tpc = (max_tiles + cl - 1) / cl;
-            if (tpc > R) continue;
-            if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;  // an idle rank
-            int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
-            if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
-            if (cap <= 0) continue;
-            for (int g = 1; g <= hq; ++g) {
-                if (hq % g) continue;
-                const int hpg = hq / g;
-                if (nb == 2 && hpg < 2) continue;  // nothing to overlap
-                const long long ctas = (long long)batch * cl * g;
-                const long long waves = (ctas + cap - 1) / cap;
-                const double active = (double)(ctas < cap ? ctas : cap);
-                double per_head;
-                if (nb == 1) {
-                    per_head = (double)tpc + (cl > 1 ? 1.0 : 0.25);
-                } else {
-                    const double stream = tpc * tile_bytes * active / hbm_bytes_per_s / unit_s;
-                    per_head = 0.6 * tpc + 2.1;
-                    if (stream > per_head) per_head = stream;
-                }
-                const double cost = (double)waves * (6.0 + (g > 1 ? 2.0 : 0.0) + hpg * per_head);
-                if (cost < best_cost - 1e-9) {
-                    best_cost = cost;
-                    lvs::ScorePlan pl{cl, tpc, g};
-                    pl.res_nb = nb;
-                    best = ScoreChoice{true, pl};
+    double tc_cost = 0.0;
+    ScoreChoice best{false, lvs::plan_score(bt, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, h->num_sms, &tc_cost)};
+    double best_cost = 1.6 * tc_cost;
+    const int max_tiles = batch > 0 ? td[0] : 0;
+    if (c.flags != LITEVLM_FLAG_SCORE_REREAD) {
+        if (c.flags == LITEVLM_FLAG_SCORE_RESIDENT || c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
+            c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
+            best_cost = 1e300;
+        for (int nb = 1; nb <= 2; ++nb) {
+            if (nb == 2 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER) continue;
+            if (nb == 1 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) continue;
+            const int R = lvs::res_max_tiles(slot_cols, nb);
+            for (int cl = 1; cl <= cmax; ++cl) {
+                const int tpc = (max_tiles + cl - 1) / cl;
+                if (tpc > R) continue;
+                if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;  // an idle rank on the largest request
+                int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
+                if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
+                if (cap <= 0) continue;
+                for (int g = 1; g <= hq; ++g) {
+                    if (hq % g) continue;
+                    const int hpg = hq / g;
+                    if (nb == 2 && hpg < 2) continue;  // nothing to overlap
+                    const long long ctas = (long long)batch * cl * g;
+                    const double active = (double)(ctas < cap ? ctas : cap);
+                    auto item_cost = [&](int tiles) {
+                        if (tiles <= 0) return 1.0;
+                        const int t = (tiles + cl - 1) / cl;
+                        double per_head;
+                        if (nb == 1) {
+                            per_head = (double)t + (cl > 1 ? 1.0 : 0.25);
+                        } else {
+                            const double stream = t * tile_bytes * active / hbm_bytes_per_s / unit_s;
+                            per_head = 0.6 * t + 2.1;
+                            if (stream > per_head) per_head = stream;
+                        }
+                        return 6.0 + (g > 1 ? 2.0 : 0.0) + hpg * per_head;
+                    };
+                    const double cost = lvs::makespan(bt, g, cap / cl, item_cost);
+                    if (cost < best_cost - 1e-9) {
+                        best_cost = cost;
+                        lvs::ScorePlan pl{cl, tpc, g};
+                        pl.res_nb = nb;
+                        best = ScoreChoice{true, pl};
+                    }
                 }
             }
         }
     }
+    auto& m = h->plan_memo[h->plan_memo_next];
+    h->plan_memo_next = (h->plan_memo_next + 1) & 3;
+    m.key = key;
+    m.used = true;
+    m.resident = best.resident;
+    m.plan = best.plan;
     return best;
 }
 
@@ -316,7 +354,7 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, co
     plan[0] = plan[1] = plan[2] = plan[3] = 0;
     if (batch == 0 || sh.tot_n == 0) return LITEVLM_OK;
     const bool fp8 = h->cfg.qk_dtype == LITEVLM_FP8_E4M3;
-    const ScoreChoice ch = choose_score_kernel(h, batch, sh.max_tiles, sh.max_t, h->cfg.head_dim * (fp8 ? 1 : 2), fp8);
+    const ScoreChoice ch = choose_score_kernel(h, batch, seq_offsets_h, sh.max_t, h->cfg.head_dim * (fp8 ? 1 : 2), fp8);
     plan[0] = ch.resident ? 1 + ch.plan.res_nb : 1;
     plan[1] = ch.plan.cluster;
     plan[2] = ch.plan.tiles_per_cta;
@@ -339,7 +377,7 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
     if (s != LITEVLM_OK) return s;
     if (batch == 0) return LITEVLM_OK;
     const int64_t tot_n = sh.tot_n, tot_t = sh.tot_t;
-    const int max_tiles = sh.max_tiles, max_t = sh.max_t;
+    const int max_t = sh.max_t;
     if (tot_n == 0) return LITEVLM_OK;
     if (!q_text || !k_vis || !scores || !text_offsets_d || !seq_offsets_d)
         return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
@@ -352,7 +390,7 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
         return fail(h, LITEVLM_ERR_INVALID_ARG, "q_scale and k_scale must be 1 for bf16 inputs");
     }
     const int row_bytes = c.head_dim * (fp8 ? 1 : 2);
-    const ScoreChoice choice = choose_score_kernel(h, batch, max_tiles, max_t, row_bytes, fp8);
+    const ScoreChoice choice = choose_score_kernel(h, batch, seq_offsets_h, max_t, row_bytes, fp8);
     const lvs::ScorePlan& plan = choice.plan;
     if (plan.tiles_per_cta > lvs::kMaxTilesPerCta)
         return fail(h, LITEVLM_ERR_UNSUPPORTED, "request too long for one cluster");
@@ -377,6 +415,23 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
     p.wait_budget = lvs::kWaitBudgetCycles;
     p.slot_cols = (max_t + 15) & ~15;
+    // clusters are launched largest request first (stable: ties keep index order)
+    p.order_n = 0;
+    if (batch > 1 && batch <= lvs::kOrderMax) {
+        int maxn = 0, minn = INT32_MAX;
+        for (int32_t b = 0; b < batch; ++b) {
+            const int n = seq_offsets_h[b + 1] - seq_offsets_h[b];
+            maxn = n > maxn ? n : maxn;
+            minn = n < minn ? n : minn;
+        }
+        if (maxn != minn) {
+            for (int32_t b = 0; b < batch; ++b) p.order[b] = (uint16_t)b;
+            std::stable_sort(p.order, p.order + batch, [&](uint16_t x, uint16_t y) {
+                return seq_offsets_h[x + 1] - seq_offsets_h[x] > seq_offsets_h[y + 1] - seq_offsets_h[y];
+            });
+            p.order_n = batch;
+        }
+    }
     const cudaError_t e =
         choice.resident
             ? lvs::launch_score_resident(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream)
@@ -513,6 +568,8 @@ struct NoAllocDevice {
     int32_t* tickets = nullptr;
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     int res_capacity[3][2][17];  // by kernel family (bf16 d=128, bf16 d=64, e4m3), as in the handle
+    litevlm_select::PlanMemo plan_memo[3][4];
+    int plan_memo_next[3] = {0, 0, 0};
 };
 
 NoAllocDevice g_noalloc[kNoAllocMaxDevices];
@@ -610,6 +667,8 @@ extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, in
         h.encode = d.encode;
         for (int r = 0; r < 2; ++r)
             for (int c = 0; c < 17; ++c) h.res_capacity[r][c] = d.res_capacity[fam][r][c];
+        for (int k = 0; k < 4; ++k) h.plan_memo[k] = d.plan_memo[fam][k];
+        h.plan_memo_next = d.plan_memo_next[fam];
     }
     h.err_d = err_d;
     h.cfg.max_batch = batch;
@@ -640,6 +699,8 @@ extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, in
         NoAllocDevice& d = g_noalloc[dev];
         for (int r = 0; r < 2; ++r)
             for (int c = 0; c < 17; ++c) d.res_capacity[fam][r][c] = h.res_capacity[r][c];
+        for (int k = 0; k < 4; ++k) d.plan_memo[fam][k] = h.plan_memo[k];
+        d.plan_memo_next[fam] = h.plan_memo_next;
     }
     if (s != LITEVLM_OK) g_create_error = h.last_error;
     return s;

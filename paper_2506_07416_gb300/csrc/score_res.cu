@@ -101,7 +101,7 @@ __device__ __forceinline__ float transpose_sum32(float (&x)[32], int lane)
 template <int ROW_BYTES, bool FP8, int MROWS>
 __global__ void __launch_bounds__(kResThreads, 1)
     score_res_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                     const ScoreLaunch p)
+                     const __grid_constant__ ScoreLaunch p)
 {
     using L = ResLayout<ROW_BYTES, MROWS>;
     constexpr int KSTEPS = ROW_BYTES / 32;
@@ -118,9 +118,12 @@ __global__ void __launch_bounds__(kResThreads, 1)
     uint8_t* smem = smem_raw + (base - raw);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = blockIdx.z, hg = blockIdx.y;
     const uint32_t rank = cluster_ctarank();
     const uint32_t csize = cluster_nctarank();
+    const int item = (int)(blockIdx.x / csize);  // this cluster's (request, head group)
+    const int req_i = item / p.groups;
+    const int b = p.order_n > 0 ? (int)p.order[req_i] : req_i;
+    const int hg = item - req_i * p.groups;
 
     griddep_wait();
     griddep_launch_dependents();
@@ -590,7 +593,7 @@ cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const S
     cudaError_t e = res_prepare<ROW_BYTES, FP8, MROWS>(plan.cluster);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(plan.cluster, plan.groups, batch);
+    cfg.gridDim = dim3((unsigned)(plan.cluster * plan.groups * batch), 1, 1);
     cfg.blockDim = dim3(kResThreads, 1, 1);
     cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS>::ALLOC;
     cfg.stream = stream;

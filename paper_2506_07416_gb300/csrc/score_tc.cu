@@ -81,7 +81,7 @@ struct SmemLayout {
 template <int ROW_BYTES, bool FP8, int MROWS>
 __global__ void __launch_bounds__(kThreads, 1)
     score_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                    const ScoreLaunch p)
+                    const __grid_constant__ ScoreLaunch p)
 {
     using L = SmemLayout<ROW_BYTES, MROWS>;
     constexpr int KSTEPS = ROW_BYTES / 32;                 // one MMA consumes 32 bytes of d
@@ -99,9 +99,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* smem = smem_raw + (base - raw);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = blockIdx.z, hg = blockIdx.y;
     const uint32_t rank = cluster_ctarank();
     const uint32_t csize = cluster_nctarank();
+    const int item = (int)(blockIdx.x / csize);  // this cluster's (request, head group)
+    const int req_i = item / p.groups;
+    const int b = p.order_n > 0 ? (int)p.order[req_i] : req_i;
+    const int hg = item - req_i * p.groups;
 
     griddep_wait();
     griddep_launch_dependents();
@@ -439,7 +442,7 @@ cudaError_t launch_variant(const CUtensorMap& tm_q, const CUtensorMap& tm_k, con
         if (e != cudaSuccess) return e;
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(plan.cluster, plan.groups, batch);
+    cfg.gridDim = dim3((unsigned)(plan.cluster * plan.groups * batch), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
@@ -475,11 +478,15 @@ static int cluster_capacity(int c, int num_sms)
     }
 }
 
-ScorePlan plan_score(int batch, int max_tiles, int hq, int hkv, int tile_bytes, int num_sms)
+ScorePlan plan_score(const BatchTiles& bt, int hq, int hkv, int tile_bytes, int num_sms, double* cost_out)
 {
     ScorePlan best{1, 1, 1};
-    if (max_tiles <= 0) return best;
     double best_cost = 1e300;
+    const int max_tiles = bt.n > 0 ? bt.desc[0] : 0;
+    if (max_tiles <= 0) {
+        if (cost_out) *cost_out = 0.0;
+        return best;
+    }
     const int G = hq / hkv;
     for (int pass = 0; pass < 2 && best_cost >= 1e299; ++pass) {
         for (int c = 1; c <= kMaxCluster; c *= 2) {
@@ -489,8 +496,7 @@ ScorePlan plan_score(int batch, int max_tiles, int hq, int hkv, int tile_bytes, 
             const int cap = cluster_capacity(c, num_sms);
             for (int g = 1; g <= hq; ++g) {
                 if (hq % g) continue;
-                const long long ctas = (long long)batch * c * g;
-                const long long waves = (ctas + cap - 1) / cap;
+                const long long ctas = (long long)bt.n * c * g;
                 const int hpg = hq / g;
                 // L2 window of the pass-2 re-read: while a CTA streams up to two
                 // slices (pass 1 of the next head, rest of the current one) the
@@ -500,11 +506,15 @@ ScorePlan plan_score(int batch, int max_tiles, int hq, int hkv, int tile_bytes, 
                 const int share = hpg >= G ? 1 : G / hpg;
                 const double window = 2.0 * tpc * tile_bytes * (double)active / share;
                 if (pass == 0 && window > 80.0 * 1024 * 1024) continue;
-                // per CTA: one tile-head of work per tile and head, plus a fixed
-                // launch / pipeline fill cost of about 6 tile-heads and a cluster
-                // exchange of about 1 tile-head per head; a fold when g > 1
-                const double per_cta = (double)tpc * hpg + 6.0 + (c > 1 ? 1.0 : 0.25) * hpg + (g > 1 ? 2.0 : 0.0);
-                const double cost = (double)waves * per_cta;
+                // one cluster (item): one tile-head of work per tile and head, plus
+                // a fixed launch / pipeline fill cost of about 6 tile-heads and a
+                // cluster exchange of about 1 tile-head per head; a fold when g > 1
+                auto item_cost = [&](int tiles) {
+                    const int t = (tiles + c - 1) / c;
+                    return tiles <= 0 ? 1.0
+                                      : (double)t * hpg + 6.0 + (c > 1 ? 1.0 : 0.25) * hpg + (g > 1 ? 2.0 : 0.0);
+                };
+                const double cost = makespan(bt, g, cap / c, item_cost);
                 if (cost < best_cost - 1e-9) {
                     best_cost = cost;
                     best = ScorePlan{c, tpc, g};
@@ -512,6 +522,7 @@ ScorePlan plan_score(int batch, int max_tiles, int hq, int hkv, int tile_bytes, 
             }
         }
     }
+    if (cost_out) *cost_out = best_cost;
     return best;
 }
 
