@@ -41,7 +41,7 @@ SCORE_CASES = [
     _case("e4m3_ragged", 8, 8, 128, "e4m3", [576, 1152, 100], [32, 128, 50]),
     _case("many_tiles_one_request", 2, 1, 128, "bf16", [9000], [40]),
     _case("sharp_logits", 4, 4, 128, "bf16", [513], [17], sigma=3.0),
-    _case("heads_overlap", 32, 32, 128, "bf16", [3456, 1000, 129], [64, 40, 7]),
+    _case("heads_overlap", 32, 32, 128, "bf16", [1536, 1000, 129], [64, 40, 7]),
 ]
 
 
