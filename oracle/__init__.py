@@ -65,6 +65,8 @@ def _bind(lib):
     lib.litevlm_oracle_topk.restype = ctypes.c_int
     lib.litevlm_oracle_compact.argtypes = [i64, P, P, P, i64]
     lib.litevlm_oracle_compact.restype = ctypes.c_int
+    lib.litevlm_oracle_splice.argtypes = [i32, P, P, P, P, P, P, P, P, i64, P, P, P]
+    lib.litevlm_oracle_splice.restype = ctypes.c_int
     return lib
 
 
@@ -147,6 +149,29 @@ def compact(kept_idx: np.ndarray, src: np.ndarray, lib=None) -> np.ndarray:
     if rc != 0:
         raise OracleError(f"litevlm_oracle_compact returned {rc}")
     return dst
+
+
+def splice(sys_offsets, seq_offsets, kept_offsets, kept_idx, text_offsets, sys_rows: np.ndarray,
+           vis_rows: np.ndarray, txt_rows: np.ndarray, lib=None):
+    """Prefill sequence [system; kept visual; text] per request with original
+    position ids. Rows are [n, row_bytes] uint8 (or any dtype, copied as bytes).
+    Returns (out_rows, out_offsets, position_ids)."""
+    lib = lib or load()
+    so, vo, ko, to = (np.ascontiguousarray(a, dtype=np.int32) for a in
+                      (sys_offsets, seq_offsets, kept_offsets, text_offsets))
+    batch = len(so) - 1
+    ki = np.ascontiguousarray(kept_idx, dtype=np.int32)
+    rows = [np.ascontiguousarray(r).view(np.uint8).reshape(r.shape[0], -1) for r in (sys_rows, vis_rows, txt_rows)]
+    rb = max(r.shape[1] for r in rows)
+    total = int(so[-1] + ko[-1] + to[-1])
+    out = np.zeros((max(total, 1), rb), np.uint8)
+    off = np.zeros(batch + 1, np.int32)
+    pos = np.zeros(max(total, 1), np.int32)
+    rc = lib.litevlm_oracle_splice(batch, _ptr(so), _ptr(vo), _ptr(ko), _ptr(ki), _ptr(to), _ptr(rows[0]),
+                                   _ptr(rows[1]), _ptr(rows[2]), rb, _ptr(out), _ptr(off), _ptr(pos))
+    if rc != 0:
+        raise OracleError(f"splice failed ({rc})")
+    return out[:total], off, pos[:total]
 
 
 def select(w_inputs: dict, hq: int, hkv: int, head_dim: int, dtype: str, keep_k=None, keep_ratio=0.0,

@@ -244,3 +244,48 @@ int litevlm_oracle_compact(int64_t total_kept, const int32_t* kept_idx,
         memcpy((char*)dst + r * row_bytes, (const char*)src + (int64_t)kept_idx[r] * row_bytes, (size_t)row_bytes);
     return OR_OK;
 }
+
+/*
+ * Prefill sequence splice (the LLM input after token selection; Design
+ * section: the module shortens the sequence the LLM prefills). Request b's
+ * output is its S_b system rows, then its k_b kept visual rows (kept_idx
+ * holds global visual-row indices, ascending within the request), then its
+ * T_b text rows, each row copied byte for byte.
+ *   out_offsets[b] = sys_offsets[b] + kept_offsets[b] + text_offsets[b]
+ * Position ids are the rows' positions in the unpruned sequence
+ * [system; all N_b visual; text]: system row i -> i, kept visual row with
+ * local index j -> S_b + j, text row t -> S_b + N_b + t (pruned tokens leave
+ * gaps; the kept tokens keep their original positions).
+ */
+int litevlm_oracle_splice(int32_t batch, const int32_t* sys_offsets, const int32_t* seq_offsets,
+                          const int32_t* kept_offsets, const int32_t* kept_idx, const int32_t* text_offsets,
+                          const void* sys_rows, const void* vis_rows, const void* txt_rows, int64_t row_bytes,
+                          void* out_rows, int32_t* out_offsets, int32_t* position_ids)
+{
+    if (batch < 0 || row_bytes <= 0) return OR_ERR_ARG;
+    for (int32_t b = 0; b <= batch; ++b) out_offsets[b] = sys_offsets[b] + kept_offsets[b] + text_offsets[b];
+    for (int32_t b = 0; b < batch; ++b) {
+        const int32_t S = sys_offsets[b + 1] - sys_offsets[b];
+        const int32_t N = seq_offsets[b + 1] - seq_offsets[b];
+        const int32_t k = kept_offsets[b + 1] - kept_offsets[b];
+        const int32_t T = text_offsets[b + 1] - text_offsets[b];
+        int64_t r = out_offsets[b];
+        for (int32_t i = 0; i < S; ++i, ++r) {
+            memcpy((char*)out_rows + r * row_bytes, (const char*)sys_rows + (int64_t)(sys_offsets[b] + i) * row_bytes,
+                   (size_t)row_bytes);
+            position_ids[r] = i;
+        }
+        for (int32_t i = 0; i < k; ++i, ++r) {
+            const int32_t g = kept_idx[kept_offsets[b] + i];
+            if (g < seq_offsets[b] || g >= seq_offsets[b] + N) return OR_ERR_ARG;
+            memcpy((char*)out_rows + r * row_bytes, (const char*)vis_rows + (int64_t)g * row_bytes, (size_t)row_bytes);
+            position_ids[r] = S + (g - seq_offsets[b]);
+        }
+        for (int32_t t = 0; t < T; ++t, ++r) {
+            memcpy((char*)out_rows + r * row_bytes, (const char*)txt_rows + (int64_t)(text_offsets[b] + t) * row_bytes,
+                   (size_t)row_bytes);
+            position_ids[r] = S + N + t;
+        }
+    }
+    return OR_OK;
+}

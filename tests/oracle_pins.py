@@ -288,7 +288,56 @@ def pin_compact(lib):
     np.testing.assert_array_equal(oracle.compact(idx, hid, lib=lib), hid[idx])
 
 
+# ---------------------------------------------------------------------------
+# prefill splice (system rows, kept visual rows, text rows; original positions)
+# ---------------------------------------------------------------------------
+
+def pin_splice_worked_example(lib):
+    """Two requests worked by hand. Request 0: 2 system rows, visual tokens 0..2
+    of which 0 and 2 are kept, 1 text row: rows s0 s1 v0 v2 t0 at positions
+    0 1 2 4 5 (the pruned token 1 leaves a gap). Request 1: 1 system row, visual
+    tokens 3..4 of which 4 (local 1) is kept, 2 text rows: s2 v4 t1 t2 at 0 2 3 4."""
+    sys_rows = np.array([[10], [11], [12]], np.uint8)
+    vis_rows = np.array([[20], [21], [22], [23], [24]], np.uint8)
+    txt_rows = np.array([[30], [31], [32]], np.uint8)
+    out, off, pos = oracle.splice([0, 2, 3], [0, 3, 5], [0, 2, 3], [0, 2, 4], [0, 1, 3], sys_rows, vis_rows, txt_rows,
+                                  lib=lib)
+    assert out.ravel().tolist() == [10, 11, 20, 22, 30, 12, 24, 31, 32]
+    assert off.tolist() == [0, 5, 9]
+    assert pos.tolist() == [0, 1, 2, 4, 5, 0, 2, 3, 4]
+
+
+def pin_splice_invariants(lib):
+    """Keeping every visual token gives the unpruned sequence with positions
+    0..L-1; keeping none gives [system; text] with text at S + N + t; rows are
+    byte copies of their sources and positions increase within a request."""
+    rng = np.random.Generator(np.random.PCG64(23))
+    S, N, T = [3, 0, 5], [7, 4, 0], [2, 6, 1]
+    so, vo, to = (np.concatenate([[0], np.cumsum(x)]).astype(np.int32) for x in (S, N, T))
+    sys_rows = rng.integers(0, 256, size=(so[-1], 40), dtype=np.uint8)
+    vis_rows = rng.integers(0, 256, size=(vo[-1], 40), dtype=np.uint8)
+    txt_rows = rng.integers(0, 256, size=(to[-1], 40), dtype=np.uint8)
+    out, off, pos = oracle.splice(so, vo, vo, np.arange(vo[-1], dtype=np.int32), to, sys_rows, vis_rows, txt_rows, lib=lib)
+    for b in range(3):
+        seq = np.concatenate([sys_rows[so[b]:so[b + 1]], vis_rows[vo[b]:vo[b + 1]], txt_rows[to[b]:to[b + 1]]])
+        np.testing.assert_array_equal(out[off[b]:off[b + 1]], seq)
+        assert pos[off[b]:off[b + 1]].tolist() == list(range(S[b] + N[b] + T[b]))
+    out, off, pos = oracle.splice(so, vo, np.zeros(4, np.int32), np.zeros(0, np.int32), to, sys_rows, vis_rows,
+                                  txt_rows, lib=lib)
+    for b in range(3):
+        assert pos[off[b]:off[b + 1]].tolist() == list(range(S[b])) + [S[b] + N[b] + t for t in range(T[b])]
+    keep = [np.sort(rng.choice(n, size=n // 2, replace=False)) for n in N]
+    ko = np.concatenate([[0], np.cumsum([len(k) for k in keep])]).astype(np.int32)
+    ki = np.concatenate([vo[b] + keep[b] for b in range(3)]).astype(np.int32)
+    out, off, pos = oracle.splice(so, vo, ko, ki, to, sys_rows, vis_rows, txt_rows, lib=lib)
+    for b in range(3):
+        p = pos[off[b]:off[b + 1]]
+        assert np.all(np.diff(p) > 0)
+        np.testing.assert_array_equal(out[off[b] + S[b]:off[b] + S[b] + len(keep[b])], vis_rows[vo[b] + keep[b]])
+        assert p[S[b]:S[b] + len(keep[b])].tolist() == [S[b] + j for j in keep[b]]
+
+
 ALL_PINS = [pin_bf16_decode, pin_e4m3_decode, pin_worked_example, pin_uniform_keys, pin_single_query_is_softmax,
             pin_row_and_total_sums, pin_batch_equals_single_requests, pin_permutation_equivariance, pin_gqa_replication, pin_scale_placement,
             pin_e4m3_scores, pin_salient_tokens_rank_first, pin_topk_bruteforce, pin_topk_batch_and_ratio,
-            pin_table1_token_counts, pin_compact]
+            pin_table1_token_counts, pin_compact, pin_splice_worked_example, pin_splice_invariants]

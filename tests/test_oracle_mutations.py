@@ -39,6 +39,9 @@ MUTANTS = [
     ("bf16_shift", "u = (uint32_t)h << 16;", "u = (uint32_t)h << 15;"),
     ("gather_wrong_row", "(const char*)src + (int64_t)kept_idx[r] * row_bytes",
      "(const char*)src + (int64_t)r * row_bytes"),
+    ("splice_visual_global_position", "position_ids[r] = S + (g - seq_offsets[b]);", "position_ids[r] = S + g;"),
+    ("splice_text_renumbered", "position_ids[r] = S + N + t;", "position_ids[r] = S + k + t;"),
+    ("splice_drops_visual", "for (int32_t i = 0; i < k; ++i, ++r) {", "for (int32_t i = 0; i < 0; ++i, ++r) {"),
 ]
 
 
