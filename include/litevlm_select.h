@@ -174,6 +174,41 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t handle, int64_t total_k
                                         litevlm_stream_t stream);
 
 /*
+ * Prefill sequence splice: the shortened LLM input after token selection
+ * (Design section: the LLM prefills only the kept visual tokens with the
+ * prompt). Request b's output rows are its S_b system rows, then its k_b kept
+ * visual rows, then its T_b text rows, each copied byte for byte; its position
+ * ids are the rows' positions in the unpruned sequence [system; all N_b
+ * visual; text]: system row i -> i, kept visual row of local index j ->
+ * S_b + j, text row t -> S_b + N_b + t (pruned tokens leave gaps, the kept ones
+ * keep their original rotary positions).
+ *   sys_rows         device [sum S_b, row_bytes]; sys_offsets_d/h int32 [batch+1]
+ *   vis_rows         device [sum N_b, row_bytes]; seq_offsets_d/h int32 [batch+1]
+ *   kept_idx         device int32 [sum k_b] global visual-row indices, ascending
+ *                    within each request (litevlm_select_topk's output);
+ *                    kept_offsets_d/h int32 [batch+1], k_b <= N_b
+ *   txt_rows         device [sum T_b, row_bytes]; text_offsets_d/h int32 [batch+1]
+ *   row_bytes        bytes per row (> 0), the same for the three sources
+ *   out_rows         device [sum (S_b + k_b + T_b), row_bytes]
+ *   out_offsets_d    device int32 [batch+1] = sys_offsets + kept_offsets + text_offsets
+ *   out_offsets_h    optional host int32 [batch+1], filled before the call returns
+ *   position_ids     device int32 [sum (S_b + k_b + T_b)]
+ * Rows move with 128-bit loads and stores when row_bytes and every row
+ * pointer are 16-byte aligned, byte by byte otherwise. A kept index outside
+ * its request's rows is skipped and reported by litevlm_select_check_device as
+ * LITEVLM_ERR_DEVICE_BOUNDS. Host-side checks as for the other calls.
+ */
+litevlm_status_t litevlm_select_splice(litevlm_select_t handle, int32_t batch, const void* sys_rows,
+                                       const int32_t* sys_offsets_d, const int32_t* sys_offsets_h,
+                                       const void* vis_rows, const int32_t* seq_offsets_d,
+                                       const int32_t* seq_offsets_h, const int32_t* kept_idx,
+                                       const int32_t* kept_offsets_d, const int32_t* kept_offsets_h,
+                                       const void* txt_rows, const int32_t* text_offsets_d,
+                                       const int32_t* text_offsets_h, int64_t row_bytes, void* out_rows,
+                                       int32_t* out_offsets_d, int32_t* out_offsets_h, int32_t* position_ids,
+                                       litevlm_stream_t stream);
+
+/*
  * Launch shape litevlm_select_score would use for this batch (host only, no
  * device work; the occupancy of a kernel variant is queried once per handle).
  * plan[0] = kernel (1: K re-read per pass; 2: logits resident in tensor

@@ -519,6 +519,69 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t h, int64_t total_kept, 
     return LITEVLM_OK;
 }
 
+litevlm_status_t litevlm_select_splice(litevlm_select_t h, int32_t batch, const void* sys_rows,
+                                       const int32_t* sys_offsets_d, const int32_t* sys_offsets_h,
+                                       const void* vis_rows, const int32_t* seq_offsets_d,
+                                       const int32_t* seq_offsets_h, const int32_t* kept_idx,
+                                       const int32_t* kept_offsets_d, const int32_t* kept_offsets_h,
+                                       const void* txt_rows, const int32_t* text_offsets_d,
+                                       const int32_t* text_offsets_h, int64_t row_bytes, void* out_rows,
+                                       int32_t* out_offsets_d, int32_t* out_offsets_h, int32_t* position_ids,
+                                       litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
+    if (batch > h->cfg.max_batch) return fail(h, LITEVLM_ERR_WORKSPACE, "batch exceeds max_batch");
+    if (row_bytes <= 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "row_bytes must be > 0");
+    int64_t tot_s = 0, tot_n = 0, tot_k = 0, tot_t = 0;
+    litevlm_status_t s = check_offsets(h, sys_offsets_h, batch, INT32_MAX, "sys_offsets", &tot_s);
+    if (s == LITEVLM_OK) s = check_offsets(h, seq_offsets_h, batch, h->cfg.max_total_visual, "seq_offsets", &tot_n);
+    if (s == LITEVLM_OK) s = check_offsets(h, kept_offsets_h, batch, h->cfg.max_total_visual, "kept_offsets", &tot_k);
+    if (s == LITEVLM_OK) s = check_offsets(h, text_offsets_h, batch, INT32_MAX, "text_offsets", &tot_t);
+    if (s != LITEVLM_OK) return s;
+    int max_rows = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int64_t kb = kept_offsets_h[b + 1] - kept_offsets_h[b];
+        const int64_t nb = seq_offsets_h[b + 1] - seq_offsets_h[b];
+        if (kb > nb)
+            return fail(h, LITEVLM_ERR_INVALID_ARG, "request " + std::to_string(b) + " keeps more rows than it has");
+        const int64_t L = (sys_offsets_h[b + 1] - sys_offsets_h[b]) + kb + (text_offsets_h[b + 1] - text_offsets_h[b]);
+        if (L > max_rows) max_rows = (int)L;
+    }
+    const int64_t tot_out = tot_s + tot_k + tot_t;
+    if (tot_out > INT32_MAX) return fail(h, LITEVLM_ERR_INVALID_ARG, "output rows exceed int32 indices");
+    if (out_offsets_h)
+        for (int32_t b = 0; b <= batch; ++b)
+            out_offsets_h[b] = sys_offsets_h[b] + kept_offsets_h[b] + text_offsets_h[b];
+    if (batch == 0) return LITEVLM_OK;
+    if (!sys_offsets_d || !seq_offsets_d || !kept_offsets_d || !text_offsets_d || !out_offsets_d)
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "a device offsets pointer is NULL");
+    if ((tot_s > 0 && !sys_rows) || (tot_k > 0 && (!vis_rows || !kept_idx)) || (tot_t > 0 && !txt_rows) ||
+        (tot_out > 0 && (!out_rows || !position_ids)))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "a device row pointer is NULL");
+    const bool vec16 = row_bytes % 16 == 0 && aligned16(sys_rows) && aligned16(vis_rows) && aligned16(txt_rows) &&
+                       aligned16(out_rows);
+    lvs::SpliceArgs a{};
+    a.sys_off = sys_offsets_d;
+    a.seq_off = seq_offsets_d;
+    a.kept_off = kept_offsets_d;
+    a.kept_idx = kept_idx;
+    a.text_off = text_offsets_d;
+    a.sys = static_cast<const uint8_t*>(sys_rows);
+    a.vis = static_cast<const uint8_t*>(vis_rows);
+    a.txt = static_cast<const uint8_t*>(txt_rows);
+    a.out = static_cast<uint8_t*>(out_rows);
+    a.out_off = out_offsets_d;
+    a.pos = position_ids;
+    a.row_bytes = row_bytes;
+    a.batch = batch;
+    a.err = h->err_d;
+    const cudaError_t e = lvs::launch_splice(a, max_rows, vec16, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "splice launch");
+    return LITEVLM_OK;
+}
+
 litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_t stream)
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;

@@ -140,4 +140,23 @@ struct GatherArgs {
 cudaError_t launch_compact(int64_t total_kept, const int32_t* kept_idx, int64_t src_rows, const GatherArgs& g,
                            bool vec16, int32_t* err, int num_sms, cudaStream_t stream);
 
+// splice.cu
+struct SpliceArgs {
+    const int32_t* sys_off;   // device [batch+1]
+    const int32_t* seq_off;   // device [batch+1] visual rows
+    const int32_t* kept_off;  // device [batch+1]
+    const int32_t* kept_idx;  // device [sum k]
+    const int32_t* text_off;  // device [batch+1]
+    const uint8_t* sys;
+    const uint8_t* vis;
+    const uint8_t* txt;
+    uint8_t* out;
+    int32_t* out_off;         // device [batch+1]
+    int32_t* pos;             // device [sum (S + k + T)]
+    int64_t row_bytes;
+    int32_t batch;
+    int32_t* err;
+};
+cudaError_t launch_splice(const SpliceArgs& a, int max_rows, bool vec16, cudaStream_t stream);
+
 }  // namespace lvs

@@ -54,8 +54,10 @@ def _load():
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
     lib.litevlm_select_score_plan.argtypes = [P, i32, P, P, P]
+    lib.litevlm_select_splice.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, P, P, i64, P, P, P, P, P]
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
-    for fn in ("create", "destroy", "score", "topk", "compact", "check_device", "score_plan", "score_noalloc"):
+    for fn in ("create", "destroy", "score", "topk", "compact", "check_device", "score_plan", "score_noalloc",
+               "splice"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -65,7 +67,7 @@ LIB = _load()
 # every symbol declared in include/litevlm_select.h
 EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
-           "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc"]
+           "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc", "litevlm_select_splice"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -151,6 +153,17 @@ def compact(handle: int, total_kept: int, kept_idx, src_rows: int, srcs: Sequenc
     rb_arr = (ctypes.c_int64 * n)(*[int(r) for r in row_bytes])
     _check(LIB.litevlm_select_compact(handle, total_kept, _ptr(kept_idx), src_rows, n, src_arr, dst_arr, rb_arr,
                                       _stream_ptr(stream)), handle)
+
+
+def splice(handle: int, batch: int, sys_rows, sys_offsets_d, sys_offsets_h, vis_rows, seq_offsets_d, seq_offsets_h,
+           kept_idx, kept_offsets_d, kept_offsets_h, txt_rows, text_offsets_d, text_offsets_h, row_bytes: int,
+           out_rows, out_offsets_d, position_ids, out_offsets_h: Optional[np.ndarray] = None, stream=None) -> None:
+    so, vo, ko, to = (_host_i32(a) for a in (sys_offsets_h, seq_offsets_h, kept_offsets_h, text_offsets_h))
+    _check(LIB.litevlm_select_splice(handle, batch, _ptr(sys_rows), _ptr(sys_offsets_d), _ptr(so), _ptr(vis_rows),
+                                     _ptr(seq_offsets_d), _ptr(vo), _ptr(kept_idx), _ptr(kept_offsets_d), _ptr(ko),
+                                     _ptr(txt_rows), _ptr(text_offsets_d), _ptr(to), int(row_bytes), _ptr(out_rows),
+                                     _ptr(out_offsets_d), _ptr(out_offsets_h), _ptr(position_ids),
+                                     _stream_ptr(stream)), handle)
 
 
 def check_device(handle: int, stream=None) -> None:
@@ -246,6 +259,26 @@ class Selector:
         rb = [s[0].numel() * s.element_size() if s.shape[0] else 1 for s in srcs]
         compact(self.handle, total_kept, kept_idx, min(rows) if rows else 0, srcs, dsts, rb, stream)
         return dsts
+
+    def splice(self, sys_rows, sys_offsets, vis_rows, seq_offsets, kept_idx, kept_offsets, txt_rows, text_offsets,
+               stream=None):
+        """[system; kept visual; text] rows per request and their original
+        position ids. Rows are 2-D torch CUDA tensors with equal row sizes;
+        offsets are int32 CUDA tensors. Returns (rows, out_offsets, out_offsets
+        host numpy, position_ids)."""
+        import torch
+        so, vo, ko, to = (_host_i32(a) for a in (sys_offsets, seq_offsets, kept_offsets, text_offsets))
+        batch = len(so) - 1
+        total = int(so[-1] + ko[-1] + to[-1])
+        ref = next(r for r in (sys_rows, vis_rows, txt_rows) if r is not None)
+        rb = ref[0].numel() * ref.element_size() if ref.shape[0] else ref.element_size() * int(np.prod(ref.shape[1:]))
+        out = torch.empty((max(total, 1),) + tuple(ref.shape[1:]), dtype=ref.dtype, device=ref.device)
+        pos = torch.empty(max(total, 1), dtype=torch.int32, device=ref.device)
+        off_d = torch.empty(batch + 1, dtype=torch.int32, device=ref.device)
+        off_h = np.zeros(batch + 1, np.int32)
+        splice(self.handle, batch, sys_rows, sys_offsets, so, vis_rows, seq_offsets, vo, kept_idx, kept_offsets, ko,
+               txt_rows, text_offsets, to, rb, out, off_d, pos, off_h, stream)
+        return out[:total], off_d, off_h, pos[:total]
 
     def check_device(self, stream=None) -> None:
         check_device(self.handle, stream)

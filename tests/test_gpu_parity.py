@@ -345,3 +345,80 @@ def test_full_size_workload(sel, name, sample):
                                else src.index_select(0, idx))
     del xd
     torch.cuda.empty_cache()
+
+
+# ----------------------------------------------------------------------------- prefill splice
+
+def _splice_case(rng, S, N, T, row_bytes, keep_frac=None):
+    so, vo, to = (np.concatenate([[0], np.cumsum(x)]).astype(np.int32) for x in (S, N, T))
+    keep = []
+    for b, n in enumerate(N):
+        k = int(rng.integers(0, n + 1)) if keep_frac is None else int(n * keep_frac)
+        keep.append(np.sort(rng.choice(n, size=k, replace=False)).astype(np.int32))
+    ko = np.concatenate([[0], np.cumsum([len(k) for k in keep])]).astype(np.int32)
+    ki = np.concatenate([vo[b] + keep[b] for b in range(len(N))] + [np.zeros(0, np.int32)]).astype(np.int32)
+    rows = [rng.integers(0, 256, size=(max(int(o[-1]), 1), row_bytes), dtype=np.uint8) for o in (so, vo, to)]
+    return so, vo, ko, ki, to, rows
+
+
+def _splice_gpu(s, so, vo, ko, ki, to, rows):
+    d = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    out, off_d, off_h, pos = s.splice(d(rows[0]), d(so), d(rows[1]), d(vo), d(ki if ki.size else np.zeros(1, np.int32)),
+                                      d(ko), d(rows[2]), d(to))
+    s.check_device()
+    return out.cpu().numpy(), off_d.cpu().numpy(), off_h, pos.cpu().numpy()
+
+
+@pytest.mark.parametrize("row_bytes", [4096, 112, 6])
+def test_splice_bit_exact(sel, row_bytes):
+    rng = np.random.Generator(np.random.PCG64(31 + row_bytes))
+    S, N, T = [0, 5, 32, 1, 0], [7, 0, 300, 129, 0], [3, 4, 0, 64, 0]
+    so, vo, ko, ki, to, rows = _splice_case(rng, S, N, T, row_bytes)
+    w = _case("splice", 1, 1, 128, "bf16", N, [1] * len(N))
+    s = _selector(sel, w)
+    out, off_d, off_h, pos = _splice_gpu(s, so, vo, ko, ki, to, rows)
+    o_out, o_off, o_pos = oracle.splice(so, vo, ko, ki, to, rows[0][:so[-1]], rows[1][:vo[-1]], rows[2][:to[-1]])
+    np.testing.assert_array_equal(out, o_out)
+    np.testing.assert_array_equal(off_d, o_off)
+    np.testing.assert_array_equal(off_h, o_off)
+    np.testing.assert_array_equal(pos, o_pos)
+
+
+def test_splice_out_of_range_kept_index_is_reported(sel):
+    rng = np.random.Generator(np.random.PCG64(37))
+    so, vo, ko, ki, to, rows = _splice_case(rng, [2, 2], [10, 10], [3, 3], 64, keep_frac=0.5)
+    ki = ki.copy()
+    ki[0] = 15  # a row of the second request listed under the first
+    w = _case("splice_bad", 1, 1, 128, "bf16", [10, 10], [1, 1])
+    s = _selector(sel, w)
+    d = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    s.splice(d(rows[0]), d(so), d(rows[1]), d(vo), d(ki), d(ko), d(rows[2]), d(to))
+    with pytest.raises(sel.LitevlmError) as ei:
+        s.check_device()
+    assert ei.value.name == "DEVICE_BOUNDS"
+
+
+def test_splice_after_selection_on_the_single_workload(sel):
+    """score -> top-k -> splice on the 1536-token request with 32 system and the
+    request's 64 text rows (hidden size rows), checked against the oracle's
+    splice of the same kept indices."""
+    w = inputs.workload("single")
+    xd = inputs.make_torch(w, "cuda")
+    s = _selector(sel, w)
+    so_v, to_t = w.seq_offsets(), w.text_offsets()
+    sc = s.score(xd["q"], xd["text_offsets"], xd["k"], xd["seq_offsets"], seq_offsets_h=so_v, text_offsets_h=to_t)
+    kept, ko_d, ko_h = s.topk(sc, xd["seq_offsets"], keep_ratio=w.keep_ratio, seq_offsets_h=so_v)
+    g = torch.Generator(device="cuda").manual_seed(41)
+    sys_rows = torch.randn((32, w.hidden), generator=g, device="cuda").to(torch.bfloat16)
+    txt_rows = torch.randn((int(to_t[-1]), w.hidden), generator=g, device="cuda").to(torch.bfloat16)
+    sys_off = torch.tensor([0, 32], dtype=torch.int32, device="cuda")
+    out, off_d, off_h, pos = s.splice(sys_rows, sys_off, xd["hidden"], xd["seq_offsets"], kept, ko_d, txt_rows,
+                                      xd["text_offsets"])
+    s.check_device()
+    as_bytes = lambda t: t.contiguous().view(torch.uint8).cpu().numpy().reshape(t.shape[0], -1)
+    o_out, o_off, o_pos = oracle.splice([0, 32], so_v, ko_h, kept.cpu().numpy(), to_t, as_bytes(sys_rows),
+                                        as_bytes(xd["hidden"]), as_bytes(txt_rows))
+    np.testing.assert_array_equal(as_bytes(out), o_out)
+    np.testing.assert_array_equal(off_h, o_off)
+    np.testing.assert_array_equal(pos.cpu().numpy(), o_pos)
+    assert int(off_h[-1]) == 32 + int(ko_h[-1]) + 64
