@@ -377,6 +377,10 @@ def run_ours(args):
                 "kernel": select.KERNELS.get(plan[0], "score"), "algorithmic_flops_per_launch": alg["score_flops"],
                 "peak_source": pk["source"] + " (burst cuBLAS bf16)"}
 
+    # prefill splice (a next-step row, timed on its own after the step): 32 system rows and
+    # the text rows of every request around its kept visual rows, hidden-size rows
+    nxt = {"splice": run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk)}
+
     # end to end through the public API with host buffers
     e2e = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept)
 
@@ -403,7 +407,7 @@ def run_ours(args):
                        "score_launch": {"kernel": select.KERNELS.get(plan[0]), "cluster": plan[1],
                                         "tiles_per_cta": plan[2], "head_groups": plan[3]}},
             "stages_p50_us": stage_us,
-            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "next": nxt,
             "gpu_launches": launches_per_step * steps, "clocks": clocks,
             "wall_s": wall}
     if rank == 0:
@@ -412,6 +416,49 @@ def run_ours(args):
         dist.destroy_process_group()
     sel.close()
     return 0
+
+
+def run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk):
+    """litevlm_select_splice on the step's kept indices: [32 system rows; kept
+    visual rows; text rows] per request, rows of `hidden` bf16, with position ids."""
+    import torch
+    from paper_2506_07416_gb300 import select
+    n_sys = 32
+    rb = w.hidden * 2
+    g = torch.Generator(device=dev).manual_seed(7)
+    sys_rows = torch.randn((n_sys * w.batch, w.hidden), generator=g, device=dev).to(torch.bfloat16)
+    txt_rows = torch.randn((max(1, w.total_txt), w.hidden), generator=g, device=dev).to(torch.bfloat16)
+    sys_h = np.arange(0, n_sys * (w.batch + 1), n_sys, dtype=np.int32)
+    sys_d = torch.from_numpy(sys_h).to(dev)
+    so_h, to_h = w.seq_offsets(), w.text_offsets()
+    total = int(sys_h[-1] + off_h[-1] + to_h[-1])
+    out = torch.empty((max(total, 1), w.hidden), dtype=torch.bfloat16, device=dev)
+    pos = torch.empty(max(total, 1), dtype=torch.int32, device=dev)
+    out_off = torch.empty(w.batch + 1, dtype=torch.int32, device=dev)
+    L = select.LIB
+    args = (sel.handle, w.batch, sys_rows.data_ptr(), sys_d.data_ptr(), sys_h.ctypes.data, xd["hidden"].data_ptr(),
+            xd["seq_offsets"].data_ptr(), so_h.ctypes.data, kept.data_ptr(), off_d.data_ptr(), off_h.ctypes.data,
+            txt_rows.data_ptr(), xd["text_offsets"].data_ptr(), to_h.ctypes.data, rb, out.data_ptr(),
+            out_off.data_ptr(), None, pos.data_ptr(), stream.cuda_stream)
+    n = max(3, min(steps, 200))
+    for _ in range(3):
+        assert L.litevlm_select_splice(*args) == 0
+    ts = []
+    for i in range(n):
+        if flush is not None:
+            flush.fill_(i)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        assert L.litevlm_select_splice(*args) == 0
+        e1.record(stream)
+        ts.append((e0, e1))
+    torch.cuda.synchronize()
+    sel.check_device()
+    us = float(np.median([a.elapsed_time(b) for a, b in ts]) * 1e3)
+    alg = 2 * total * rb + 4 * total
+    gbs = alg / (us * 1e-6) / 1e9
+    return {"us_p50": us, "rows": total, "row_bytes": rb, "algorithmic_bytes": alg, "achieved_gbs": gbs,
+            "frac_of_hbm": gbs / pk["hbm_gbs"], "system_rows_per_request": n_sys}
 
 
 def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept):
