@@ -73,6 +73,11 @@ typedef enum {
 #define LITEVLM_FLAG_SCORE_RESIDENT 2 /* use the TMEM-resident kernel whenever the shapes allow it */
 #define LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER 8 /* the same, with one TMEM head buffer only (no head overlap) */
 #define LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS 16 /* the same, two TMEM head buffers where the shapes allow it */
+/* OR-ed with at most one of the above: only the last text token of each request
+ * is a query, T_b counts as 1 in the mean (the last-token variant of attention-
+ * score pruning, Related Work / FastV). Requests may then have more than 128
+ * text tokens. */
+#define LITEVLM_FLAG_QUERY_LAST_TOKEN 32
 
 typedef struct {
     int32_t max_batch;         /* largest batch any call will pass */
@@ -82,7 +87,7 @@ typedef struct {
     int32_t num_kv_heads;      /* Hkv, Hq % Hkv == 0 */
     int32_t head_dim;          /* d: 64 or 128 for bf16, 128 for e4m3 */
     litevlm_dtype_t qk_dtype;
-    int32_t flags;             /* 0 or one LITEVLM_FLAG_SCORE_* value */
+    int32_t flags;             /* 0 or one LITEVLM_FLAG_SCORE_* value, optionally | LITEVLM_FLAG_QUERY_LAST_TOKEN */
 } litevlm_select_config_t;
 
 typedef struct litevlm_select* litevlm_select_t;

@@ -150,13 +150,14 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* se
     ScoreChoice best{false, lvs::plan_score(bt, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, h->num_sms, &tc_cost)};
     double best_cost = 1.6 * tc_cost;
     const int max_tiles = batch > 0 ? td[0] : 0;
-    if (c.flags != LITEVLM_FLAG_SCORE_REREAD) {
-        if (c.flags == LITEVLM_FLAG_SCORE_RESIDENT || c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
-            c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
+    const int kflags = c.flags & ~LITEVLM_FLAG_QUERY_LAST_TOKEN;
+    if (kflags != LITEVLM_FLAG_SCORE_REREAD) {
+        if (kflags == LITEVLM_FLAG_SCORE_RESIDENT || kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
+            kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
             best_cost = 1e300;
         for (int nb = 1; nb <= 2; ++nb) {
-            if (nb == 2 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER) continue;
-            if (nb == 1 && c.flags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) continue;
+            if (nb == 2 && kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER) continue;
+            if (nb == 1 && kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) continue;
             const int R = lvs::res_max_tiles(slot_cols, nb);
             for (int cl = 1; cl <= cmax; ++cl) {
                 const int tpc = (max_tiles + cl - 1) / cl;
@@ -241,8 +242,10 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
     if (c->qk_dtype != LITEVLM_BF16 && c->qk_dtype != LITEVLM_FP8_E4M3)
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "qk_dtype must be LITEVLM_BF16 or LITEVLM_FP8_E4M3");
-    if (c->flags != 0 && c->flags != LITEVLM_FLAG_SCORE_REREAD && c->flags != LITEVLM_FLAG_SCORE_RESIDENT &&
-        c->flags != LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER && c->flags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
+    const int kflags = c->flags & ~LITEVLM_FLAG_QUERY_LAST_TOKEN;
+    if (c->flags < 0 || (kflags != 0 && kflags != LITEVLM_FLAG_SCORE_REREAD && kflags != LITEVLM_FLAG_SCORE_RESIDENT &&
+                         kflags != LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER &&
+                         kflags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS))
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "flags must be 0 or one LITEVLM_FLAG_SCORE_* value");
     if (c->head_dim <= 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "head_dim must be > 0");
     if (!lvs::score_shape_supported(c->head_dim, c->qk_dtype == LITEVLM_FP8_E4M3))
@@ -328,7 +331,8 @@ litevlm_status_t check_score_shape(litevlm_select_t h, int32_t batch, const int3
         if (n > 0 && t == 0)
             return fail(h, LITEVLM_ERR_INVALID_ARG,
                         "request " + std::to_string(b) + " has visual tokens but no text query token");
-        if (t > lvs::kMaxText)
+        const bool last_only = (h->cfg.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
+        if (t > lvs::kMaxText && !last_only)
             return fail(h, LITEVLM_ERR_UNSUPPORTED, "request " + std::to_string(b) + " has " + std::to_string(t) +
                                                         " text tokens; the score kernel handles at most 128");
         if (n > 65536)
@@ -337,7 +341,8 @@ litevlm_status_t check_score_shape(litevlm_select_t h, int32_t batch, const int3
         const int tiles = (n + lvs::kTileRows - 1) / lvs::kTileRows;
         if (tiles > sh->max_tiles) sh->max_tiles = tiles;
         if (n > sh->max_n) sh->max_n = n;
-        if (n > 0 && t > sh->max_t) sh->max_t = t;
+        const int tq = last_only && t > 0 ? 1 : t;  // query rows the kernels use
+        if (n > 0 && tq > sh->max_t) sh->max_t = tq;
     }
     return LITEVLM_OK;
 }
@@ -415,6 +420,7 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
     p.wait_budget = lvs::kWaitBudgetCycles;
     p.slot_cols = (max_t + 15) & ~15;
+    p.query_last = (c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
     // clusters are launched largest request first (stable: ties keep index order)
     p.order_n = 0;
     if (batch > 1 && batch <= lvs::kOrderMax) {

@@ -47,6 +47,7 @@ struct ScoreLaunch {
     int32_t ctas_per_request; // cluster size * groups
     int32_t slot_cols;        // resident kernel: TMEM columns per slot (T rounded up to 16, max over batch)
     int32_t res_nb;           // resident kernel: TMEM head buffers, 1 or 2 (2: heads overlap)
+    int32_t query_last;       // 1: only the last text token of each request is a query
     float c_log2;             // q_scale * k_scale / sqrt(d) * log2(e)
     long long wait_budget;
     // Cluster k of the 1-D grid serves item k: request order[k / groups] (the

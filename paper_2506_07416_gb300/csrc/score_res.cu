@@ -131,7 +131,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
     // below (barriers, TMEM, cluster barrier), so their latency overlaps it.
     const int n0 = p.seq_off[b];
     const int n1 = p.seq_off[b + 1];
-    const int t0 = p.text_off[b];
+    const int tq = p.text_off[b];
     const int t1 = p.text_off[b + 1];
     const bool multi = p.groups > 1;
     const int G = p.hq / p.hkv;
@@ -187,6 +187,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
     const int N = n1 - n0;
+    const int t0 = p.query_last && t1 > tq ? t1 - 1 : tq;  // last-token queries: one row
     const int T = t1 - t0;
     const int n2 = (T + 15) & ~15;
     const int n_tiles = (N + kTileRows - 1) / kTileRows;

@@ -110,8 +110,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     griddep_launch_dependents();
     const int n0 = p.seq_off[b];
     const int N = p.seq_off[b + 1] - n0;
-    const int t0 = p.text_off[b];
-    const int T = p.text_off[b + 1] - t0;
+    const int t1 = p.text_off[b + 1];
+    const int t0 = p.query_last && t1 > p.text_off[b] ? t1 - 1 : p.text_off[b];  // last-token queries: one row
+    const int T = t1 - t0;
     const bool multi = p.groups > 1;
     // Uniform for the whole cluster (same request). With several head groups
     // every CTA must still take its fold ticket, so only shape errors return.

@@ -116,10 +116,14 @@ def _stream_ptr(stream) -> Optional[int]:
 # C functions, one to one
 # ----------------------------------------------------------------------------
 
+QUERY_LAST_TOKEN = 32
+
+
 def create(max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int, num_kv_heads: int,
-           head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto") -> int:
+           head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto", query: str = "all") -> int:
+    """query: "all" (every text token is a query) or "last" (only the last one)."""
     cfg = Config(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
-                 DTYPES[qk_dtype], FLAGS[score_kernel])
+                 DTYPES[qk_dtype], FLAGS[score_kernel] | (QUERY_LAST_TOKEN if query == "last" else 0))
     h = ctypes.c_void_p()
     _check(LIB.litevlm_select_create(ctypes.byref(cfg), ctypes.byref(h)), None)
     return h.value
@@ -197,9 +201,10 @@ class Selector:
     """Owns one handle. Tensors are torch CUDA tensors laid out as in the C header."""
 
     def __init__(self, max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int,
-                 num_kv_heads: int, head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto"):
+                 num_kv_heads: int, head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto",
+                 query: str = "all"):
         self.handle = create(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
-                             qk_dtype, score_kernel)
+                             qk_dtype, score_kernel, query)
         self.qk_dtype = qk_dtype
 
     def close(self) -> None:

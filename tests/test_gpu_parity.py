@@ -422,3 +422,27 @@ def test_splice_after_selection_on_the_single_workload(sel):
     np.testing.assert_array_equal(off_h, o_off)
     np.testing.assert_array_equal(pos.cpu().numpy(), o_pos)
     assert int(off_h[-1]) == 32 + int(ko_h[-1]) + 64
+
+
+# ----------------------------------------------------------------------------- last-token queries
+
+LAST_TOKEN_CASES = SCORE_CASES[:5] + [_case("long_text_last", 8, 8, 128, "bf16", [700, 129], [200, 3])]
+
+
+@pytest.mark.parametrize("kernel", ["reread", "resident"])
+@pytest.mark.parametrize("w", LAST_TOKEN_CASES, ids=lambda w: w.name)
+def test_last_token_queries_match_oracle(sel, w, kernel):
+    """Only the last text token of each request is a query: the same score as
+    the oracle's on each request's last text row alone."""
+    x = inputs.make_numpy(w)
+    xd = to_device(x, w)
+    s = sel.Selector(max(1, w.batch), max(1, w.total_vis), max(1, w.total_txt), w.hq, w.hkv, w.head_dim, w.dtype,
+                     score_kernel=kernel, query="last")
+    g = _gpu_scores(sel, s, w, x, xd)
+    to = np.asarray(x["text_offsets"])
+    last = np.array([to[b + 1] - 1 for b in range(w.batch) if to[b + 1] > to[b]], np.int64)
+    lens = [1 if to[b + 1] > to[b] else 0 for b in range(w.batch)]
+    to_last = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    o = oracle.score(x["q"][last], x["k"], x["seq_offsets"], to_last, w.hq, w.hkv, w.head_dim, w.dtype,
+                     x["q_scale"], x["k_scale"])
+    assert_scores_close(g, o, w.dtype)
