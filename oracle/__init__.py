@@ -65,6 +65,8 @@ def _bind(lib):
     lib.litevlm_oracle_topk.restype = ctypes.c_int
     lib.litevlm_oracle_compact.argtypes = [i64, P, P, P, i64]
     lib.litevlm_oracle_compact.restype = ctypes.c_int
+    lib.litevlm_oracle_score_full.argtypes = [i32, P, P, P, i32, i32, i32, i32, P, P, P, P, f64, f64, P, P, P]
+    lib.litevlm_oracle_score_full.restype = ctypes.c_int
     lib.litevlm_oracle_splice.argtypes = [i32, P, P, P, P, P, P, P, P, i64, P, P, P]
     lib.litevlm_oracle_splice.restype = ctypes.c_int
     return lib
@@ -110,6 +112,30 @@ def score(q: np.ndarray, k: np.ndarray, seq_offsets, text_offsets, hq: int, hkv:
         raise OracleError(f"litevlm_oracle_score returned {rc}")
     if details:
         return out, s64, rows, lse
+    return out
+
+
+def score_full(q: np.ndarray, k: np.ndarray, k_sys: np.ndarray, k_txt: np.ndarray, seq_offsets, text_offsets,
+               sys_offsets, hq: int, hkv: int, head_dim: int, dtype: str = "bf16", q_scale: float = 1.0,
+               k_scale: float = 1.0, lib=None, details: bool = False):
+    """Scores with the softmax over the full causal key set (system, visual,
+    text keys up to the query); details=True also returns the fp64 scores and
+    the visual attention share per (b, h, i)."""
+    lib = lib or load()
+    so, to, yo = (np.ascontiguousarray(a, dtype=np.int32) for a in (seq_offsets, text_offsets, sys_offsets))
+    batch = so.size - 1
+    n_tot, t_tot = int(so[-1]), int(to[-1])
+    arrs = [np.ascontiguousarray(a) for a in (q, k, k_sys, k_txt)]
+    out = np.zeros(n_tot, dtype=np.float32)
+    s64 = np.zeros(n_tot, dtype=np.float64)
+    share = np.zeros(max(1, hq * t_tot), dtype=np.float64)
+    rc = lib.litevlm_oracle_score_full(batch, _ptr(so), _ptr(to), _ptr(yo), hq, hkv, head_dim, DTYPE_CODES[dtype],
+                                       _ptr(arrs[0]), _ptr(arrs[1]), _ptr(arrs[2]), _ptr(arrs[3]), float(q_scale),
+                                       float(k_scale), _ptr(out), _ptr(s64), _ptr(share))
+    if rc != 0:
+        raise OracleError(f"litevlm_oracle_score_full returned {rc}")
+    if details:
+        return out, s64, share[:hq * t_tot]
     return out
 
 

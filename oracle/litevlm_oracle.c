@@ -43,6 +43,10 @@
  *   R12 NaN scores rank below everything, +inf above;
  *   R13 N_b = 0 or k_b = 0 give an empty output; N_b > 0 with T_b = 0 is an error.
  *
+ * litevlm_oracle_score_full is the variant without R2 and R3: the normaliser
+ * runs over the system, visual and causal text keys of the first decoder
+ * layer, so a request's scores sum to its visual attention share (< 1).
+ *
  * Element decoding: bf16 is the top half of an IEEE binary32; e4m3 follows the
  * OCP 8-bit floating point specification (E4M3, bias 7, no infinities, the
  * all-ones code is NaN, subnormals m * 2^-9).
@@ -286,6 +290,93 @@ int litevlm_oracle_splice(int32_t batch, const int32_t* sys_offsets, const int32
                    (size_t)row_bytes);
             position_ids[r] = S + N + t;
         }
+    }
+    return OR_OK;
+}
+
+/*
+ * Visual-token scores with the softmax normaliser over the full causal key
+ * set of the first decoder layer (a reading of the Design section's
+ * first-layer attention; the variant of litevlm_oracle_score that does not
+ * restrict the keys to the visual tokens). Text query i of request b, head h,
+ * attends to the S_b system keys, the N_b visual keys and the text keys
+ * t' <= i (causal); with s the scaled logits over all of them,
+ *     P[h][i][j] = exp(s[h][i][j] - m) / sum_{all keys} exp(s - m)
+ *     score[j]   = (sum_h sum_i P[h][i][j]) / (Hq * T_b),  j visual
+ * so a request's scores sum to the attention share of its visual tokens.
+ * k_sys [sum S_b, Hkv, d] and k_txt [sum T_b, Hkv, d] are the system and text
+ * tokens' keys, in the element type of q and k (same per-tensor k_scale).
+ * visual_share [sum_b Hq*T_b] (nullable): sum_j P[h][i][j] over visual j.
+ */
+int litevlm_oracle_score_full(int32_t batch, const int32_t* seq_offsets, const int32_t* text_offsets,
+                              const int32_t* sys_offsets, int32_t hq, int32_t hkv, int32_t head_dim, int32_t dtype,
+                              const void* q, const void* k, const void* k_sys, const void* k_txt, double q_scale,
+                              double k_scale, float* scores, double* scores64, double* visual_share)
+{
+    int64_t row_out = 0;
+    if (batch < 0 || hq <= 0 || hkv <= 0 || head_dim <= 0 || hq % hkv != 0) return OR_ERR_ARG;
+    if (dtype != OR_F32 && dtype != OR_BF16 && dtype != OR_E4M3) return OR_ERR_ARG;
+    for (int32_t b = 0; b < batch; ++b) {
+        if (seq_offsets[b + 1] < seq_offsets[b] || text_offsets[b + 1] < text_offsets[b] ||
+            sys_offsets[b + 1] < sys_offsets[b])
+            return OR_ERR_ARG;
+        if (seq_offsets[b + 1] > seq_offsets[b] && text_offsets[b + 1] == text_offsets[b]) return OR_ERR_ARG;
+    }
+    const int32_t group = hq / hkv;
+    const double scale = q_scale * k_scale / sqrt((double)head_dim);
+    for (int32_t b = 0; b < batch; ++b) {
+        const int64_t n0 = seq_offsets[b], nb = seq_offsets[b + 1] - seq_offsets[b];
+        const int64_t t0 = text_offsets[b], tb = text_offsets[b + 1] - text_offsets[b];
+        const int64_t s0 = sys_offsets[b], sb = sys_offsets[b + 1] - sys_offsets[b];
+        if (nb == 0) {
+            if (visual_share) for (int64_t r = 0; r < (int64_t)hq * tb; ++r) visual_share[row_out + r] = 0.0;
+            row_out += (int64_t)hq * tb;
+            continue;
+        }
+        const int64_t nkeys = sb + nb + tb;  /* system, visual, text keys of this request */
+        double* acc = (double*)calloc((size_t)nb, sizeof(double));
+        double* s = (double*)malloc((size_t)nkeys * sizeof(double));
+        double* qd = (double*)malloc((size_t)(tb * hq * head_dim) * sizeof(double));
+        double* kd = (double*)malloc((size_t)(nkeys * hkv * head_dim) * sizeof(double));
+        if (!acc || !s || !qd || !kd) { free(acc); free(s); free(qd); free(kd); return OR_ERR_NOMEM; }
+        const int64_t row = (int64_t)hkv * head_dim;
+        for (int64_t x = 0; x < tb * hq * head_dim; ++x) qd[x] = litevlm_oracle_decode(dtype, q, t0 * hq * head_dim + x);
+        for (int64_t x = 0; x < sb * row; ++x) kd[x] = litevlm_oracle_decode(dtype, k_sys, s0 * row + x);
+        for (int64_t x = 0; x < nb * row; ++x) kd[sb * row + x] = litevlm_oracle_decode(dtype, k, n0 * row + x);
+        for (int64_t x = 0; x < tb * row; ++x) kd[(sb + nb) * row + x] = litevlm_oracle_decode(dtype, k_txt, t0 * row + x);
+        for (int32_t h = 0; h < hq; ++h) {
+            const int32_t g = h / group;
+            for (int64_t i = 0; i < tb; ++i) {
+                const int64_t qrow = (i * hq + h) * head_dim;
+                const int64_t nk = sb + nb + i + 1;  /* keys visible to text query i */
+                double m = -INFINITY, z = 0.0, vis = 0.0;
+                for (int64_t j = 0; j < nk; ++j) {
+                    const int64_t krow = (j * hkv + g) * head_dim;
+                    double dot = 0.0;
+                    for (int32_t c = 0; c < head_dim; ++c) dot += qd[qrow + c] * kd[krow + c];
+                    s[j] = dot * scale;
+                    if (s[j] > m) m = s[j];
+                }
+                for (int64_t j = 0; j < nk; ++j) z += exp(s[j] - m);
+                for (int64_t j = 0; j < nb; ++j) {
+                    const double p = exp(s[sb + j] - m) / z;
+                    acc[j] += p;
+                    vis += p;
+                }
+                if (visual_share) visual_share[row_out] = vis;
+                ++row_out;
+            }
+        }
+        const double denom = (double)hq * (double)tb;
+        for (int64_t j = 0; j < nb; ++j) {
+            const double v = acc[j] / denom;
+            scores[n0 + j] = (float)v;
+            if (scores64) scores64[n0 + j] = v;
+        }
+        free(acc);
+        free(s);
+        free(qd);
+        free(kd);
     }
     return OR_OK;
 }

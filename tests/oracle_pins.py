@@ -289,6 +289,58 @@ def pin_compact(lib):
 
 
 # ---------------------------------------------------------------------------
+# full causal key set in the softmax normaliser
+# ---------------------------------------------------------------------------
+
+def pin_full_keys_worked_example(lib):
+    """The worked example with one system key and the two text tokens' keys in
+    the normaliser. Head 0's system and text keys are zero (logit 0); head 1's
+    queries are zero, so all its logits are 0 whatever the keys. Row i of a head
+    sees 1 system key, the 4 visual keys and i + 1 text keys:
+      head 0: row 0 [e,1,1,1] / (e+5), row 1 [1,e,1,1] / (e+6)
+      head 1: row 0 1/6 each, row 1 1/7 each."""
+    q, k, _ = worked_example()
+    rng = np.random.Generator(np.random.PCG64(29))
+    k_sys = np.zeros((1, 2, 4), np.float32)
+    k_txt = np.zeros((2, 2, 4), np.float32)
+    k_sys[:, 1, :] = rng.standard_normal((1, 4))
+    k_txt[:, 1, :] = rng.standard_normal((2, 4))
+    e = math.e
+    common = 1 / 6 + 1 / 7
+    expect = np.array([(e / (e + 5) + 1 / (e + 6) + common) / 4, (1 / (e + 5) + e / (e + 6) + common) / 4,
+                       (1 / (e + 5) + 1 / (e + 6) + common) / 4, (1 / (e + 5) + 1 / (e + 6) + common) / 4])
+    s, s64, share = oracle.score_full(q, k, k_sys, k_txt, [0, 4], [0, 2], [0, 1], 2, 2, 4, "f32", lib=lib,
+                                      details=True)
+    np.testing.assert_allclose(s64, expect, rtol=1e-14, atol=0)
+    np.testing.assert_allclose(share, [(e + 3) / (e + 5), (e + 3) / (e + 6), 4 / 6, 4 / 7], rtol=1e-14)
+
+
+def pin_full_keys_equal_duplicated_visual_keys(lib):
+    """With one text token per request, extra keys that copy visual keys act as
+    duplicated visual tokens: the full-key scores of the original visual tokens
+    equal the visual-only oracle's scores on the visual keys plus those copies."""
+    rng = np.random.Generator(np.random.PCG64(31))
+    hq, hkv, d = 4, 2, 16
+    N, S = [9, 5], [2, 1]
+    so, yo = (np.concatenate([[0], np.cumsum(x)]).astype(np.int32) for x in (N, S))
+    to = np.array([0, 1, 2], np.int32)
+    q = rng.standard_normal((2, hq, d)).astype(np.float32)
+    k = rng.standard_normal((int(so[-1]), hkv, d)).astype(np.float32)
+    # system keys: request 0 copies its tokens 3 and 4, request 1 its token 2;
+    # text keys: each request copies one of its tokens
+    k_sys = np.stack([k[so[0] + 3], k[so[0] + 4], k[so[1] + 2]]).astype(np.float32)
+    k_txt = np.stack([k[so[0] + 7], k[so[1] + 1]]).astype(np.float32)
+    s = oracle.score_full(q, k, k_sys, k_txt, so, to, yo, hq, hkv, d, "f32", lib=lib)
+    ext0 = np.concatenate([k[so[0]:so[1]], k_sys[:2], k_txt[:1]])
+    ext1 = np.concatenate([k[so[1]:so[2]], k_sys[2:], k_txt[1:]])
+    eo = np.array([0, len(ext0), len(ext0) + len(ext1)], np.int32)
+    ref = oracle.score(q, np.concatenate([ext0, ext1]), eo, to, hq, hkv, d, "f32", lib=lib)
+    np.testing.assert_allclose(s[so[0]:so[1]], ref[eo[0]:eo[0] + N[0]], rtol=2e-7)
+    np.testing.assert_allclose(s[so[1]:so[2]], ref[eo[1]:eo[1] + N[1]], rtol=2e-7)
+    assert s[so[0]:so[1]].sum() < 1.0 and s[so[1]:so[2]].sum() < 1.0
+
+
+# ---------------------------------------------------------------------------
 # prefill splice (system rows, kept visual rows, text rows; original positions)
 # ---------------------------------------------------------------------------
 
@@ -340,4 +392,5 @@ def pin_splice_invariants(lib):
 ALL_PINS = [pin_bf16_decode, pin_e4m3_decode, pin_worked_example, pin_uniform_keys, pin_single_query_is_softmax,
             pin_row_and_total_sums, pin_batch_equals_single_requests, pin_permutation_equivariance, pin_gqa_replication, pin_scale_placement,
             pin_e4m3_scores, pin_salient_tokens_rank_first, pin_topk_bruteforce, pin_topk_batch_and_ratio,
-            pin_table1_token_counts, pin_compact, pin_splice_worked_example, pin_splice_invariants]
+            pin_table1_token_counts, pin_compact, pin_splice_worked_example, pin_splice_invariants,
+            pin_full_keys_worked_example, pin_full_keys_equal_duplicated_visual_keys]
