@@ -138,6 +138,37 @@ litevlm_status_t litevlm_select_score(litevlm_select_t handle, int32_t batch,
                                       litevlm_stream_t stream);
 
 /*
+ * The same scores with the softmax normaliser over the full causal key set of
+ * the first decoder layer: the prompt is [system; image; text], so text query
+ * i of request b attends to the S_b system keys, the N_b visual keys and the
+ * text keys 0..i (causal mask). The probabilities of the visual keys are
+ * summed as in litevlm_select_score; a request's scores then add up to its
+ * visual attention share (< 1) instead of 1 (Design section, Token Selection
+ * Module: self-attention of the first decoder layer).
+ *     s[h][i][j] as above, for every key j of [system; visual; text 0..i]
+ *     score[j]   = (1 / (Hq * T_b)) * sum_h sum_i exp(s[h][i][j]) / sum_{j'} exp(s[h][i][j']),  j visual
+ * Arguments as for litevlm_select_score, plus
+ *   k_sys            device, [sum S_b, Hkv, d] system-prompt key rows (may be NULL when sum S_b = 0)
+ *   sys_offsets_d/h  int32 [batch+1] prefix of S_b (no limit on S_b)
+ *   k_text           device, [sum T_b, Hkv, d] key rows of the text tokens (rows follow text_offsets)
+ * k_sys and k_text have the element type and k_scale of k_vis and are 16-byte
+ * aligned. With LITEVLM_FLAG_QUERY_LAST_TOKEN the one query (the last text
+ * token) sees every system and text key. The extra statistics live in the
+ * handle's workspace ([max_total_text][Hq] floats, allocated by create).
+ * Errors: those of litevlm_select_score; INVALID_ARG for missing or unaligned
+ * k_sys / k_text or bad sys_offsets.
+ */
+litevlm_status_t litevlm_select_score_full_keys(litevlm_select_t handle, int32_t batch,
+                                                const void* q_text, const int32_t* text_offsets_d,
+                                                const int32_t* text_offsets_h,
+                                                const void* k_vis, const int32_t* seq_offsets_d,
+                                                const int32_t* seq_offsets_h,
+                                                const void* k_sys, const int32_t* sys_offsets_d,
+                                                const int32_t* sys_offsets_h, const void* k_text,
+                                                float q_scale, float k_scale, float* scores,
+                                                litevlm_stream_t stream);
+
+/*
  * Per-request top-k (Results section, ratio r of visual tokens kept; Table 1).
  *   scores           device, float [sum N_b]
  *   keep_k_d/h       int32 [batch] tokens to keep per request, 0 <= k_b <= N_b;

@@ -24,6 +24,7 @@ struct litevlm_select {
     int32_t* counters = nullptr;  // fold tickets of the score kernels, one per 128-token tile
     size_t n_counters = 0;
     int32_t* err_d = nullptr;   // device error word (bits lvs::kErr*)
+    float* ctx_stats = nullptr; // [max_total_text][Hq]: normaliser terms of system + causal text keys
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     int res_capacity[2][17];  // resident score kernel: CTAs at once per cluster size, by pass-1 rows (64/128); -1 unknown
     // last score-kernel choices, keyed by a hash of the batch shape (planning walks every plan)
@@ -284,12 +285,15 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
     h->n_counters = (size_t)(c->max_total_visual / lvs::kTileRows) + 2 * (size_t)c->max_batch + 2;
     if (e == cudaSuccess) e = cudaMalloc(&h->counters, sizeof(int32_t) * h->n_counters);
     if (e == cudaSuccess) e = cudaMemset(h->counters, 0, sizeof(int32_t) * h->n_counters);
+    if (e == cudaSuccess)
+        e = cudaMalloc(&h->ctx_stats, sizeof(float) * (size_t)c->num_q_heads * (size_t)c->max_total_text);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         const std::string msg = std::string("create: ") + cudaGetErrorString(e);
         if (h->counters) cudaFree(h->counters);
         if (h->err_d) cudaFree(h->err_d);
         if (h->partials) cudaFree(h->partials);
+        if (h->ctx_stats) cudaFree(h->ctx_stats);
         delete h;
         cudaGetLastError();
         return fail(nullptr, LITEVLM_ERR_CUDA, msg);
@@ -304,6 +308,7 @@ litevlm_status_t litevlm_select_destroy(litevlm_select_t h)
     if (h->partials) cudaFree(h->partials);
     if (h->counters) cudaFree(h->counters);
     if (h->err_d) cudaFree(h->err_d);
+    if (h->ctx_stats) cudaFree(h->ctx_stats);
     delete h;
     return LITEVLM_OK;
 }
@@ -367,14 +372,20 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, co
     return LITEVLM_OK;
 }
 
-litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const void* q_text,
-                                      const int32_t* text_offsets_d, const int32_t* text_offsets_h,
-                                      const void* k_vis, const int32_t* seq_offsets_d,
-                                      const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
-                                      litevlm_stream_t stream)
+namespace {
+// Keys beyond the visual tokens for the full-key-set normaliser (null: none).
+struct CtxKeys {
+    const void* k_sys;
+    const int32_t* sys_offsets_d;
+    const int32_t* sys_offsets_h;
+    const void* k_text;
+};
+
+litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_text, const int32_t* text_offsets_d,
+                            const int32_t* text_offsets_h, const void* k_vis, const int32_t* seq_offsets_d,
+                            const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
+                            const CtxKeys* ctx, litevlm_stream_t stream)
 {
-    if (!h) return LITEVLM_ERR_INVALID_ARG;
-    h->last_error.clear();
     const litevlm_select_config_t& c = h->cfg;
     const bool fp8 = c.qk_dtype == LITEVLM_FP8_E4M3;
     ScoreShape sh;
@@ -395,6 +406,17 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
         return fail(h, LITEVLM_ERR_INVALID_ARG, "q_scale and k_scale must be 1 for bf16 inputs");
     }
     const int row_bytes = c.head_dim * (fp8 ? 1 : 2);
+    if (ctx) {
+        if (!ctx->sys_offsets_d || !ctx->sys_offsets_h)
+            return fail(h, LITEVLM_ERR_INVALID_ARG, "sys_offsets_d and sys_offsets_h are required");
+        int64_t tot_s = 0;
+        s = check_offsets(h, ctx->sys_offsets_h, batch, INT32_MAX, "sys_offsets", &tot_s);
+        if (s != LITEVLM_OK) return s;
+        if (!ctx->k_text || (tot_s > 0 && !ctx->k_sys))
+            return fail(h, LITEVLM_ERR_INVALID_ARG, "k_text (and k_sys when sum S_b > 0) must not be NULL");
+        if (!aligned16(ctx->k_text) || (ctx->k_sys && !aligned16(ctx->k_sys)))
+            return fail(h, LITEVLM_ERR_INVALID_ARG, "k_sys and k_text must be 16-byte aligned");
+    }
     const ScoreChoice choice = choose_score_kernel(h, batch, seq_offsets_h, max_t, row_bytes, fp8);
     const lvs::ScorePlan& plan = choice.plan;
     if (plan.tiles_per_cta > lvs::kMaxTilesPerCta)
@@ -421,6 +443,27 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
     p.wait_budget = lvs::kWaitBudgetCycles;
     p.slot_cols = (max_t + 15) & ~15;
     p.query_last = (c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
+    p.extra = nullptr;
+    if (ctx) {
+        lvs::CtxArgs ca{};
+        ca.q = static_cast<const uint8_t*>(q_text);
+        ca.k_sys = static_cast<const uint8_t*>(ctx->k_sys);
+        ca.k_txt = static_cast<const uint8_t*>(ctx->k_text);
+        ca.seq_off = seq_offsets_d;
+        ca.text_off = text_offsets_d;
+        ca.sys_off = ctx->sys_offsets_d;
+        ca.out = h->ctx_stats;
+        ca.err = h->err_d;
+        ca.batch = batch;
+        ca.hq = c.num_q_heads;
+        ca.hkv = c.num_kv_heads;
+        ca.query_last = p.query_last;
+        ca.c_log2 = p.c_log2;
+        ca.wait_budget = lvs::kWaitBudgetCycles;
+        const cudaError_t ce = lvs::launch_ctx_stats(ca, row_bytes, fp8, (cudaStream_t)stream);
+        if (ce != cudaSuccess) return cuda_fail(h, ce, "context-key statistics launch");
+        p.extra = h->ctx_stats;
+    }
     // clusters are launched largest request first (stable: ties keep index order)
     p.order_n = 0;
     if (batch > 1 && batch <= lvs::kOrderMax) {
@@ -444,6 +487,34 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
             : lvs::launch_score(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "score launch");
     return LITEVLM_OK;
+}
+}  // namespace
+
+litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const void* q_text,
+                                      const int32_t* text_offsets_d, const int32_t* text_offsets_h,
+                                      const void* k_vis, const int32_t* seq_offsets_d,
+                                      const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
+                                      litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    return score_impl(h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h,
+                      q_scale, k_scale, scores, nullptr, stream);
+}
+
+litevlm_status_t litevlm_select_score_full_keys(litevlm_select_t h, int32_t batch, const void* q_text,
+                                                const int32_t* text_offsets_d, const int32_t* text_offsets_h,
+                                                const void* k_vis, const int32_t* seq_offsets_d,
+                                                const int32_t* seq_offsets_h, const void* k_sys,
+                                                const int32_t* sys_offsets_d, const int32_t* sys_offsets_h,
+                                                const void* k_text, float q_scale, float k_scale, float* scores,
+                                                litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    const CtxKeys ctx{k_sys, sys_offsets_d, sys_offsets_h, k_text};
+    return score_impl(h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h,
+                      q_scale, k_scale, scores, &ctx, stream);
 }
 
 litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const float* scores,

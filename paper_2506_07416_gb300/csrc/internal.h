@@ -50,6 +50,9 @@ struct ScoreLaunch {
     int32_t query_last;       // 1: only the last text token of each request is a query
     float c_log2;             // q_scale * k_scale / sqrt(d) * log2(e)
     long long wait_budget;
+    // [sum T][Hq] normaliser terms of the system and causal text keys (unit of
+    // the merged statistic b, from ctx_stats.cu), or null: visual keys only
+    const float* extra;
     // Cluster k of the 1-D grid serves item k: request order[k / groups] (the
     // requests from the largest to the smallest, so the hardware starts the
     // biggest clusters first and fills in with small ones), head group
@@ -140,6 +143,23 @@ struct GatherArgs {
 };
 cudaError_t launch_compact(int64_t total_kept, const int32_t* kept_idx, int64_t src_rows, const GatherArgs& g,
                            bool vec16, int32_t* err, int num_sms, cudaStream_t stream);
+
+// ctx_stats.cu: e[t][h] = log2 sum 2^(c q.k) over the system and causal text
+// keys of every text query row (the full-key-set normaliser's extra terms)
+struct CtxArgs {
+    const uint8_t* q;         // [sum T, Hq, d]
+    const uint8_t* k_sys;     // [sum S, Hkv, d]
+    const uint8_t* k_txt;     // [sum T, Hkv, d]
+    const int32_t* seq_off;   // device [batch+1] visual rows
+    const int32_t* text_off;  // device [batch+1]
+    const int32_t* sys_off;   // device [batch+1]
+    float* out;               // [sum T][Hq]
+    int32_t* err;
+    int32_t batch, hq, hkv, query_last;
+    float c_log2;
+    long long wait_budget;
+};
+cudaError_t launch_ctx_stats(const CtxArgs& a, int row_bytes, bool fp8, cudaStream_t stream);
 
 // splice.cu
 struct SpliceArgs {

@@ -93,6 +93,14 @@ __device__ __forceinline__ void row_stats_update(const float* v, int valid, floa
     m = m_new;
 }
 
+// log2(2^x + 2^y) for the merged statistic b and a normaliser term of other
+// keys in the same unit (x finite)
+__device__ __forceinline__ float log2_add(float x, float y)
+{
+    const float mx = fmaxf(x, y), mn = fminf(x, y);
+    return mx + __log2f(1.f + ex2(mn - mx));
+}
+
 // Merges the (max, sum) partials of one row from every CTA of the cluster in
 // rank order and returns b = M * c + log2(L). All remote loads are issued
 // before any is used, so their latencies overlap.

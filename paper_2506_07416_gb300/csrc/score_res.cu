@@ -479,7 +479,8 @@ __global__ void __launch_bounds__(kResThreads, 1)
                         const float2 v2 = rs[r * scols];
                         if (v2.y > 0.f) Ls += v2.y * ex2((v2.x - M) * cl);
                     }
-                    const float b = fmaf(M, cl, __log2f(Ls));
+                    float b = fmaf(M, cl, __log2f(Ls));
+                    if (p.extra) b = log2_add(b, p.extra[(int64_t)(t0 + col) * p.hq + hg * hpg + s]);
                     float mloc = smax[wt];  // this CTA's column max: the e values' reference
 #pragma unroll
                     for (int q = 1; q < 4; ++q) mloc = fmaxf(mloc, smax[q * 64 + wt]);

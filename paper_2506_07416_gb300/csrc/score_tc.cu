@@ -363,8 +363,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int slot = hs % kStatSlots;
                 float* b2 = b2_s + (hs & 1) * kMaxText;
                 wait_phase_cluster(BAR(STATS + slot), (uint32_t)(hs / kStatSlots) & 1u, ctl);
-                if (et < T) b2[et] = merge_cluster_row(base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u, csize, cl);
-                else b2[et] = INFINITY;
+                if (et < T) {
+                    float bm = merge_cluster_row(base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u, csize, cl);
+                    if (p.extra) bm = log2_add(bm, p.extra[(int64_t)(t0 + et) * p.hq + hg * hpg + hs]);
+                    b2[et] = bm;
+                } else {
+                    b2[et] = INFINITY;
+                }
                 named_bar_sync(1, 128);
                 // ---- pass 2 of head s-1: per-visual-token sums of probabilities
                 for (int t = tile_begin; t < tile_end; ++t) {

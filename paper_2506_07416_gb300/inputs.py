@@ -272,3 +272,64 @@ def make_torch(w: Workload, device, seed: Optional[int] = None, chunk_rows: int 
         out["v"] = normal(N, w.hkv * d, 1.0, torch.bfloat16).view(N, w.hkv, d)
     out["hidden"] = normal(N, w.hidden, 1.0, torch.bfloat16)
     return out
+
+
+# ----------------------------------------------------------------------------
+# keys of the system prompt and the text tokens (full-key-set scores)
+# ----------------------------------------------------------------------------
+
+def context_keys_numpy(w: Workload, sys_lens: Sequence[int], k_scale: float = 1.0, seed: Optional[int] = None,
+                       sink_gain: float = 0.0, q_f32: Optional[np.ndarray] = None) -> Dict[str, object]:
+    """Key rows of the system prompt ([sum S_b, Hkv, d]) and of the text tokens
+    ([sum T_b, Hkv, d]), drawn like the visual keys (normal, std sigma) and
+    encoded like them (bf16 bits, or e4m3 codes under the visual keys' scale
+    k_scale, clipped to +-448). sink_gain > 0 makes each request's first system
+    key an attention sink: each KV head's row points along the request's mean
+    query direction u of that head group (q_f32, the unrounded queries), scaled
+    so that the mean logit q.k / sqrt(d) of the group's queries is sink_gain."""
+    rng = np.random.Generator(np.random.PCG64((w.seed + 1000003) if seed is None else seed))
+    so = _offsets(sys_lens)
+    S, T, d = int(so[-1]), w.total_txt, w.head_dim
+    ks = (rng.standard_normal((S, w.hkv, d)) * w.sigma).astype(np.float32)
+    kt = (rng.standard_normal((T, w.hkv, d)) * w.sigma).astype(np.float32)
+    if sink_gain > 0 and S > 0:
+        to, g = w.text_offsets(), w.hq // w.hkv
+        for b in range(len(sys_lens)):
+            if sys_lens[b] == 0 or to[b + 1] == to[b]:
+                continue
+            for kv in range(w.hkv):
+                qg = q_f32[to[b]:to[b + 1], kv * g:(kv + 1) * g, :].astype(np.float64)
+                u = qg.sum(axis=(0, 1))
+                nrm = np.linalg.norm(u)
+                if nrm == 0:
+                    continue
+                u /= nrm
+                proj = float(np.mean(qg @ u))  # mean q.u > 0
+                ks[so[b], kv] = (sink_gain * math.sqrt(d) / proj * u).astype(np.float32)
+    out: Dict[str, object] = {"sys_offsets": so}
+    for name, x in (("k_sys", ks), ("k_txt", kt)):
+        if w.dtype == "bf16":
+            out[name] = f32_to_bf16_bits(x)
+        else:
+            import torch
+            y = np.clip(x / np.float32(k_scale), -E4M3_MAX, E4M3_MAX).astype(np.float32)
+            out[name] = torch.from_numpy(y).to(torch.float8_e4m3fn).view(torch.uint8).numpy().copy()
+    return out
+
+
+def context_keys_torch(w: Workload, sys_lens: Sequence[int], device, k_scale: float = 1.0,
+                       seed: Optional[int] = None):
+    """The same shapes drawn on a device (values differ from the numpy draw)."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed((w.seed + 1000003) if seed is None else seed)
+    so = _offsets(sys_lens)
+    S, T, d = int(so[-1]), w.total_txt, w.head_dim
+    out = {"sys_offsets": torch.from_numpy(so).to(device)}
+    for name, rows in (("k_sys", S), ("k_txt", T)):
+        x = torch.randn((max(rows, 0), w.hkv, d), generator=gen, device=device) * w.sigma
+        if w.dtype == "bf16":
+            out[name] = x.to(torch.bfloat16)
+        else:
+            out[name] = (x / k_scale).clamp(-E4M3_MAX, E4M3_MAX).to(torch.float8_e4m3fn).view(torch.uint8)
+    return out

@@ -50,14 +50,15 @@ def _load():
     lib.litevlm_status_string.argtypes = [ctypes.c_int]
     lib.litevlm_status_string.restype = ctypes.c_char_p
     lib.litevlm_select_score.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P]
+    lib.litevlm_select_score_full_keys.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, f32, f32, P, P]
     lib.litevlm_select_topk.argtypes = [P, i32, P, P, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
     lib.litevlm_select_score_plan.argtypes = [P, i32, P, P, P]
     lib.litevlm_select_splice.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, P, P, i64, P, P, P, P, P]
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
-    for fn in ("create", "destroy", "score", "topk", "compact", "check_device", "score_plan", "score_noalloc",
-               "splice"):
+    for fn in ("create", "destroy", "score", "score_full_keys", "topk", "compact", "check_device", "score_plan",
+               "score_noalloc", "splice"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -67,7 +68,8 @@ LIB = _load()
 # every symbol declared in include/litevlm_select.h
 EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
-           "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc", "litevlm_select_splice"]
+           "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc",
+           "litevlm_select_splice", "litevlm_select_score_full_keys"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -139,6 +141,16 @@ def score(handle: int, batch: int, q_text, text_offsets_d, text_offsets_h, k_vis
     _check(LIB.litevlm_select_score(handle, batch, _ptr(q_text), _ptr(text_offsets_d), _ptr(to_h), _ptr(k_vis),
                                     _ptr(seq_offsets_d), _ptr(so_h), q_scale, k_scale, _ptr(scores),
                                     _stream_ptr(stream)), handle)
+
+
+def score_full_keys(handle: int, batch: int, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d,
+                    seq_offsets_h, k_sys, sys_offsets_d, sys_offsets_h, k_text, q_scale: float, k_scale: float,
+                    scores, stream=None) -> None:
+    to_h, so_h, yo_h = _host_i32(text_offsets_h), _host_i32(seq_offsets_h), _host_i32(sys_offsets_h)
+    _check(LIB.litevlm_select_score_full_keys(handle, batch, _ptr(q_text), _ptr(text_offsets_d), _ptr(to_h),
+                                              _ptr(k_vis), _ptr(seq_offsets_d), _ptr(so_h), _ptr(k_sys),
+                                              _ptr(sys_offsets_d), _ptr(yo_h), _ptr(k_text), q_scale, k_scale,
+                                              _ptr(scores), _stream_ptr(stream)), handle)
 
 
 def topk(handle: int, batch: int, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h, keep_ratio: float,
@@ -227,6 +239,20 @@ class Selector:
             out = torch.empty(int(so_h[-1]), dtype=torch.float32, device=k.device)
         score(self.handle, len(so_h) - 1, q, text_offsets, to_h, k, seq_offsets, so_h, q_scale, k_scale, out,
               stream)
+        return out
+
+    def score_full_keys(self, q, text_offsets, k, seq_offsets, k_sys, sys_offsets, k_text, q_scale=1.0,
+                        k_scale=1.0, out=None, text_offsets_h=None, seq_offsets_h=None, sys_offsets_h=None,
+                        stream=None):
+        """Scores with the softmax over [system; visual; causal text] keys."""
+        import torch
+        so_h = _host_i32(seq_offsets if seq_offsets_h is None else seq_offsets_h)
+        to_h = _host_i32(text_offsets if text_offsets_h is None else text_offsets_h)
+        yo_h = _host_i32(sys_offsets if sys_offsets_h is None else sys_offsets_h)
+        if out is None:
+            out = torch.empty(int(so_h[-1]), dtype=torch.float32, device=k.device)
+        score_full_keys(self.handle, len(so_h) - 1, q, text_offsets, to_h, k, seq_offsets, so_h, k_sys, sys_offsets,
+                        yo_h, k_text, q_scale, k_scale, out, stream)
         return out
 
     def topk(self, scores, seq_offsets, keep_k=None, keep_ratio: float = 0.0, seq_offsets_h=None, kept_idx=None,
