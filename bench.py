@@ -379,7 +379,8 @@ def run_ours(args):
 
     # prefill splice (a next-step row, timed on its own after the step): 32 system rows and
     # the text rows of every request around its kept visual rows, hidden-size rows
-    nxt = {"splice": run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk)}
+    nxt = {"splice": run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk),
+           "full_keys": run_full_keys(w, xd, sel, dev, stream, steps, flush, pk)}
 
     # end to end through the public API with host buffers
     e2e = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept)
@@ -459,6 +460,51 @@ def run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk):
     gbs = alg / (us * 1e-6) / 1e9
     return {"us_p50": us, "rows": total, "row_bytes": rb, "algorithmic_bytes": alg, "achieved_gbs": gbs,
             "frac_of_hbm": gbs / pk["hbm_gbs"], "system_rows_per_request": n_sys}
+
+
+def run_full_keys(w, xd, sel, dev, stream, steps, flush, pk):
+    """litevlm_select_score_full_keys against litevlm_select_score on the same
+    batch: the softmax over [32 system keys; visual keys; causal text keys] per
+    request. Both calls timed alone (CUDA events, median); the difference is
+    the cost of the context-key statistics kernel and the merge."""
+    import torch
+    from paper_2506_07416_gb300 import inputs, select
+    n_sys = 32
+    c = inputs.context_keys_torch(w, [n_sys] * w.batch, dev, k_scale=xd["k_scale"])
+    sys_h = np.arange(0, n_sys * (w.batch + 1), n_sys, dtype=np.int32)
+    so_h, to_h = w.seq_offsets(), w.text_offsets()
+    scores = torch.empty(max(1, w.total_vis), dtype=torch.float32, device=dev)
+    L = select.LIB
+    base = (sel.handle, w.batch, xd["q"].data_ptr(), xd["text_offsets"].data_ptr(), to_h.ctypes.data,
+            xd["k"].data_ptr(), xd["seq_offsets"].data_ptr(), so_h.ctypes.data)
+    tail = (xd["q_scale"], xd["k_scale"], scores.data_ptr(), stream.cuda_stream)
+    full = base + (c["k_sys"].data_ptr(), c["sys_offsets"].data_ptr(), sys_h.ctypes.data, c["k_txt"].data_ptr()) + tail
+    calls = {"visual_keys": lambda: L.litevlm_select_score(*base, *tail),
+             "full_keys": lambda: L.litevlm_select_score_full_keys(*full)}
+    n = max(3, min(steps, 200))
+    us = {}
+    for name, fn in calls.items():
+        for _ in range(3):
+            assert fn() == 0
+        ts = []
+        for i in range(n):
+            if flush is not None:
+                flush.fill_(i)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            assert fn() == 0
+            e1.record(stream)
+            ts.append((e0, e1))
+        torch.cuda.synchronize()
+        us[name] = float(np.median([a.elapsed_time(b) for a, b in ts]) * 1e3)
+    sel.check_device()
+    rb = w.head_dim * (2 if w.dtype == "bf16" else 1)
+    # context-key statistics: q rows and the system / text key rows once, e[t][h] out
+    ctx_bytes = (w.total_txt * w.hq + (n_sys * w.batch + w.total_txt) * w.hkv) * rb + w.total_txt * w.hq * 4
+    return {"us_p50": us["full_keys"], "visual_keys_us_p50": us["visual_keys"],
+            "extra_us": us["full_keys"] - us["visual_keys"], "system_keys_per_request": n_sys,
+            "context_algorithmic_bytes": ctx_bytes,
+            "tokens_per_s_M": w.total_vis / (us["full_keys"] * 1e-6) / 1e6}
 
 
 def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept):
