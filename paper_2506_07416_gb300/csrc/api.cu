@@ -36,6 +36,7 @@ struct litevlm_select {
     } plan_memo[4];
     int plan_memo_next = 0;
     std::vector<int> tiles_desc;  // scratch of the planner for batches above 4096 requests (host)
+    lvs::TopkShape topk_shape;    // per-request sizes passed to the top-k kernel by value
     std::string last_error;
 };
 
@@ -560,8 +561,16 @@ litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const fl
     if (total_k > 0 && (!kept_idx || !scores)) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
     if (out_offsets_h)
         for (int32_t b = 0; b <= batch; ++b) out_offsets_h[b] = off[(size_t)b];
+    lvs::TopkShape& sh = h->topk_shape;
+    sh.n = batch <= lvs::kTopkShapeMax ? batch : 0;
+    for (int32_t b = 0; b < sh.n; ++b) {
+        sh.n0[b] = seq_offsets_h[b];
+        sh.len[b] = seq_offsets_h[b + 1] - seq_offsets_h[b];
+        sh.k[b] = off[(size_t)b + 1] - off[(size_t)b];
+        sh.out0[b] = off[(size_t)b];
+    }
     const cudaError_t e = lvs::launch_topk(batch, scores, seq_offsets_d, keep_k_d, keep_ratio, kept_idx,
-                                           out_offsets_d, max_n, (cudaStream_t)stream);
+                                           out_offsets_d, max_n, sh, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "topk launch");
     return LITEVLM_OK;
 }

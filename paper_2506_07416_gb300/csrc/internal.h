@@ -130,8 +130,20 @@ cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm
                                   cudaStream_t stream);
 
 // topk.cu
+// Per-request sizes from the host mirrors, passed by value for small batches
+// so the kernel needs no dependent global loads before it reads the scores
+// (the mirrors equal the device arrays by contract).
+constexpr int kTopkShapeMax = 256;
+struct TopkShape {
+    int32_t n;                      // requests described; 0: the kernel reads the device arrays
+    int32_t n0[kTopkShapeMax];      // first visual row of the request
+    int32_t len[kTopkShapeMax];     // N_b
+    int32_t k[kTopkShapeMax];       // k_b
+    int32_t out0[kTopkShapeMax];    // sum of k over earlier requests
+};
 cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,
-                        float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, cudaStream_t stream);
+                        float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, const TopkShape& shape,
+                        cudaStream_t stream);
 
 // compact.cu
 constexpr int kMaxGatherTensors = 8;

@@ -145,24 +145,24 @@ __device__ __forceinline__ void fold_tiles(const ScoreLaunch& p, int b, int n0, 
     named_bar_sync(bar_id, nthreads);
     __threadfence();
     const float denom = (float)p.hq * (float)T;
-    for (int tl = 0; tl < mt; ++tl) {
+    // (tile, row) pairs spread over all threads; up to 16 group partials in
+    // flight per row, added in group order
+    for (int x = tid; x < mt * kTileRows; x += nthreads) {
+        const int tl = x / kTileRows;
         if (!flags[tl]) continue;
-        for (int r = tid; r < kTileRows; r += nthreads) {
-            const int j = (tile_begin + tl) * kTileRows + r;
-            if (j >= N) break;
-            const float* src = p.partials + n0 + j;
-            float sum = 0.f;
-            int g = 0;
-            for (; g + 8 <= p.groups; g += 8) {
-                float x[8];
+        const int j = (tile_begin + tl) * kTileRows + (x - tl * kTileRows);
+        if (j >= N) continue;
+        const float* src = p.partials + n0 + j;
+        float sum = 0.f;
+        for (int g = 0; g < p.groups; g += 16) {
+            float v[16];
 #pragma unroll
-                for (int q = 0; q < 8; ++q) x[q] = __ldcg(src + (int64_t)(g + q) * p.total_vis);
+            for (int q = 0; q < 16; ++q) v[q] = g + q < p.groups ? __ldcg(src + (int64_t)(g + q) * p.total_vis) : 0.f;
 #pragma unroll
-                for (int q = 0; q < 8; ++q) sum += x[q];
-            }
-            for (; g < p.groups; ++g) sum += __ldcg(src + (int64_t)g * p.total_vis);
-            p.out[n0 + j] = sum / denom;
+            for (int q = 0; q < 16; ++q)
+                if (g + q < p.groups) sum += v[q];
         }
+        p.out[n0 + j] = sum / denom;
     }
 }
 

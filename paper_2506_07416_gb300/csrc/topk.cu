@@ -208,7 +208,7 @@ template <int KPT>
 __global__ void __launch_bounds__(kTopkThreads)
     topk_reg_kernel(const float* __restrict__ scores, const int32_t* __restrict__ seq_off,
                     const int32_t* __restrict__ keep_k, float ratio, int32_t* __restrict__ kept_idx,
-                    int32_t* __restrict__ out_off)
+                    int32_t* __restrict__ out_off, const __grid_constant__ TopkShape sh)
 {
     __shared__ uint32_t hist[3][256];
     __shared__ uint32_t wmin[kTopkWarps], wmax[kTopkWarps];
@@ -217,10 +217,22 @@ __global__ void __launch_bounds__(kTopkThreads)
 
     const int b = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // sizes in the parameters (read before the wait: they are not produced on
+    // the device), so the scores are the kernel's first global loads
+    const bool by_value = sh.n > 0;
+    int n0 = 0, N = 0, k_v = 0, out0_v = 0;
+    if (by_value) {
+        n0 = sh.n0[b];
+        N = sh.len[b];
+        k_v = sh.k[b];
+        out0_v = sh.out0[b];
+    }
     griddep_wait();
     griddep_launch_dependents();
-    const int n0 = seq_off[b];
-    const int N = seq_off[b + 1] - n0;
+    if (!by_value) {
+        n0 = seq_off[b];
+        N = seq_off[b + 1] - n0;
+    }
 
     uint32_t key[KPT];
 #pragma unroll
@@ -231,13 +243,14 @@ __global__ void __launch_bounds__(kTopkThreads)
 
     // output base = sum of k over earlier requests
     long long part = 0;
-    for (int bb = tid; bb < b; bb += kTopkThreads) part += keep_count(seq_off, keep_k, ratio, bb);
+    if (!by_value)
+        for (int bb = tid; bb < b; bb += kTopkThreads) part += keep_count(seq_off, keep_k, ratio, bb);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
-    if (tid == 0) s_base = 0;
+    if (tid == 0) s_base = by_value ? (long long)out0_v : 0;
     __syncthreads();
     if (lane == 0 && part) atomicAdd(reinterpret_cast<unsigned long long*>(&s_base), (unsigned long long)part);
-    const int k = keep_count(seq_off, keep_k, ratio, b);
+    const int k = by_value ? k_v : keep_count(seq_off, keep_k, ratio, b);
 
     // key range of the request (padding slots take part only through valid keys)
     uint32_t lo_k = 0xFFFFFFFFu, hi_k = 0u;
@@ -412,7 +425,8 @@ cudaError_t launch_pdl(void (*kern)(Args...), unsigned grid, unsigned block, siz
 }
 
 cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,
-                        float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, cudaStream_t stream)
+                        float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, const TopkShape& shape,
+                        cudaStream_t stream)
 {
     if (batch <= 0) return cudaSuccess;
     // requests up to 16 keys per thread: registers only
@@ -422,7 +436,7 @@ cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, 
                     : max_n <= 8 * kTopkThreads ? topk_reg_kernel<8>
                                                 : topk_reg_kernel<16>;
         return launch_pdl(kern, (unsigned)batch, kTopkThreads, 0, stream, scores, seq_off, keep_k, keep_ratio,
-                          kept_idx, out_off);
+                          kept_idx, out_off, shape);
     }
     const int keys = max_n < kTopkSmemKeys ? max_n : kTopkSmemKeys;
     const size_t smem = (size_t)keys * 4;
