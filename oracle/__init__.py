@@ -69,6 +69,9 @@ def _bind(lib):
     lib.litevlm_oracle_score_full.restype = ctypes.c_int
     lib.litevlm_oracle_splice.argtypes = [i32, P, P, P, P, P, P, P, P, i64, P, P, P]
     lib.litevlm_oracle_splice.restype = ctypes.c_int
+    lib.litevlm_oracle_select_views.argtypes = [i32, i32, P, P, P, ctypes.c_float, ctypes.c_float, ctypes.c_float,
+                                                 i32, P, P, P, P]
+    lib.litevlm_oracle_select_views.restype = ctypes.c_int
     return lib
 
 
@@ -198,6 +201,26 @@ def splice(sys_offsets, seq_offsets, kept_offsets, kept_idx, text_offsets, sys_r
     if rc != 0:
         raise OracleError(f"splice failed ({rc})")
     return out[:total], off, pos[:total]
+
+
+def select_views(lexical: np.ndarray, logits: np.ndarray, tokens_per_view, w_lex: float, w_logit: float,
+                 threshold: float, min_views: int = 0, lib=None):
+    """Patch-selection gating. lexical, logits: float32 [B, V]. Returns
+    (view_mask uint8 [B, V], view_offsets [B+1], selected_views, seq_offsets [B+1])."""
+    lib = lib or load()
+    lx = np.ascontiguousarray(lexical, dtype=np.float32)
+    lg = np.ascontiguousarray(logits, dtype=np.float32)
+    batch, nv = lx.shape
+    tpv = np.ascontiguousarray(tokens_per_view, dtype=np.int32)
+    mask = np.zeros((batch, nv), np.uint8)
+    vo = np.zeros(batch + 1, np.int32)
+    sv = np.zeros(max(1, batch * nv), np.int32)
+    so = np.zeros(batch + 1, np.int32)
+    rc = lib.litevlm_oracle_select_views(batch, nv, _ptr(lx), _ptr(lg), _ptr(tpv), float(w_lex), float(w_logit),
+                                         float(threshold), int(min_views), _ptr(mask), _ptr(vo), _ptr(sv), _ptr(so))
+    if rc != 0:
+        raise OracleError(f"litevlm_oracle_select_views returned {rc}")
+    return mask, vo, sv[:int(vo[-1])], so
 
 
 def select(w_inputs: dict, hq: int, hkv: int, head_dim: int, dtype: str, keep_k=None, keep_ratio=0.0,

@@ -43,6 +43,9 @@
  *   R12 NaN scores rank below everything, +inf above;
  *   R13 N_b = 0 or k_b = 0 give an empty output; N_b > 0 with T_b = 0 is an error.
  *
+ * litevlm_oracle_select_views is the patch-selection gating upstream of the
+ * path (its readings are stated at the function).
+ *
  * litevlm_oracle_score_full is the variant without R2 and R3: the normaliser
  * runs over the system, visual and causal text keys of the first decoder
  * layer, so a request's scores sum to its visual attention share (< 1).
@@ -377,6 +380,73 @@ int litevlm_oracle_score_full(int32_t batch, const int32_t* seq_offsets, const i
         free(s);
         free(qd);
         free(kd);
+    }
+    return OR_OK;
+}
+
+/*
+ * Patch-selection gating (Design section, Patch Selection Module: the final
+ * score of a camera view is a weighted sum of the lexical-mapping score and
+ * the module's logit; the views scoring above a predefined threshold go on to
+ * the vision encoder). For request b and view v, in fp32 arithmetic:
+ *     s[b][v] = w_lex * lexical[b][v] + w_logit * logit[b][v]
+ *     view v is selected when s[b][v] > threshold
+ * Readings: the logit enters as is (no sigmoid); "above" is strict; when fewer
+ * than min_views views pass, the min_views highest-scoring views are taken
+ * instead (ties to the lower view index; NaN scores rank lowest and never pass
+ * the threshold); min_views = 0 allows an empty selection.
+ * Outputs: view_mask[b][v] in {0, 1}; view_offsets (prefix of the selected
+ * view counts) and selected_views (view indices, ascending per request);
+ * seq_offsets (prefix of the visual tokens: sum over selected v of
+ * tokens_per_view[v]), the N_b of the token-selection path.
+ */
+static int oracle_view_before(float a, int ia, float b, int ib)
+{
+    /* strict order of (score desc, index asc), NaN lowest */
+    const int an = a != a, bn = b != b;
+    if (an != bn) return bn;
+    if (!an && a != b) return a > b;
+    return ia < ib;
+}
+
+int litevlm_oracle_select_views(int32_t batch, int32_t num_views, const float* lexical, const float* logits,
+                                const int32_t* tokens_per_view, float w_lex, float w_logit, float threshold,
+                                int32_t min_views, uint8_t* view_mask, int32_t* view_offsets,
+                                int32_t* selected_views, int32_t* seq_offsets)
+{
+    if (batch < 0 || num_views <= 0 || num_views > 64 || min_views < 0 || min_views > num_views) return OR_ERR_ARG;
+    view_offsets[0] = 0;
+    seq_offsets[0] = 0;
+    int64_t nsel = 0, ntok = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        float s[64];
+        int pass = 0;
+        for (int32_t v = 0; v < num_views; ++v) {
+            const float a = w_lex * lexical[(int64_t)b * num_views + v];
+            const float c = w_logit * logits[(int64_t)b * num_views + v];
+            s[v] = a + c;
+            const int sel = s[v] > threshold;
+            view_mask[(int64_t)b * num_views + v] = (uint8_t)sel;
+            pass += sel;
+        }
+        if (pass < min_views) {
+            /* the min_views best views: rank each view by how many views come before it */
+            for (int32_t v = 0; v < num_views; ++v) {
+                int rank = 0;
+                for (int32_t u = 0; u < num_views; ++u)
+                    if (u != v && oracle_view_before(s[u], u, s[v], v)) ++rank;
+                view_mask[(int64_t)b * num_views + v] = (uint8_t)(rank < min_views);
+            }
+        }
+        for (int32_t v = 0; v < num_views; ++v) {
+            if (view_mask[(int64_t)b * num_views + v]) {
+                selected_views[nsel++] = v;
+                ntok += tokens_per_view[v];
+            }
+        }
+        if (ntok > INT32_MAX) return OR_ERR_ARG;
+        view_offsets[b + 1] = (int32_t)nsel;
+        seq_offsets[b + 1] = (int32_t)ntok;
     }
     return OR_OK;
 }

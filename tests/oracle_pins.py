@@ -389,8 +389,62 @@ def pin_splice_invariants(lib):
         assert p[S[b]:S[b] + len(keep[b])].tolist() == [S[b] + j for j in keep[b]]
 
 
+# ---------------------------------------------------------------------------
+# patch-selection gating
+# ---------------------------------------------------------------------------
+
+def pin_views_worked_example(lib):
+    """Hand-worked gating of three requests over four views (w_lex 2, w_logit 1,
+    threshold 0.5, min_views 1; tokens per view 512, 512, 256, 128):
+      request 0: s = [2.2, -1, 3, 0.5]  -> views 0, 2 (0.5 is not above 0.5)   768 tokens
+      request 1: s = [-5, -2, -3, -2]   -> none pass; the best is -2 at views 1
+                                           and 3, the lower index wins: view 1   512 tokens
+      request 2: s = [NaN, 0, -1, -7]   -> none pass; NaN ranks lowest: view 1  512 tokens"""
+    lex = np.array([[1, 0, 0, 1], [0, 0, 0, 0], [0, 0, 0, 0]], np.float32)
+    lg = np.array([[0.2, -1, 3, -1.5], [-5, -2, -3, -2], [np.nan, 0, -1, -7]], np.float32)
+    mask, vo, sv, so = oracle.select_views(lex, lg, [512, 512, 256, 128], 2.0, 1.0, 0.5, 1, lib=lib)
+    assert mask.tolist() == [[1, 0, 1, 0], [0, 1, 0, 0], [0, 1, 0, 0]], mask
+    assert vo.tolist() == [0, 2, 3, 4] and sv.tolist() == [0, 2, 1, 1]
+    assert so.tolist() == [0, 768, 1280, 1792]
+    # min_views 0: an empty selection is allowed
+    mask0, vo0, sv0, so0 = oracle.select_views(lex, lg, [512, 512, 256, 128], 2.0, 1.0, 0.5, 0, lib=lib)
+    assert mask0.tolist() == [[1, 0, 1, 0], [0, 0, 0, 0], [0, 0, 0, 0]] and so0.tolist() == [0, 768, 768, 768]
+
+
+def pin_views_properties(lib):
+    """On random inputs: a threshold below every score keeps every view and
+    N_b = sum of tokens_per_view; one above every score keeps none (min_views
+    0) or exactly the min_views best (every kept score >= every dropped one);
+    raising the threshold never adds a view; offsets are prefix sums."""
+    rng = np.random.Generator(np.random.PCG64(37))
+    B, V = 50, 6
+    lex = (rng.random((B, V)) < 0.3).astype(np.float32)
+    lg = rng.standard_normal((B, V)).astype(np.float32) * 2
+    tpv = np.array([256, 512, 256, 576, 256, 128], np.int32)
+    m, vo, sv, so = oracle.select_views(lex, lg, tpv, 1.5, 0.7, -1e30, 0, lib=lib)
+    assert m.all() and np.array_equal(np.diff(so), np.full(B, tpv.sum())) and np.array_equal(np.diff(vo), np.full(B, V))
+    m, vo, sv, so = oracle.select_views(lex, lg, tpv, 1.5, 0.7, 1e30, 0, lib=lib)
+    assert not m.any() and so[-1] == 0 and vo[-1] == 0
+    for k in (1, 2, 3):
+        m, vo, sv, so = oracle.select_views(lex, lg, tpv, 1.5, 0.7, 1e30, k, lib=lib)
+        assert np.array_equal(m.sum(axis=1), np.full(B, k))
+        s = np.float32(1.5) * lex + np.float32(0.7) * lg
+        for b in range(B):
+            assert s[b][m[b] == 1].min() >= s[b][m[b] == 0].max()
+    prev = None
+    for t in (-2.0, -0.5, 0.0, 0.7, 1.5, 3.0):
+        m, vo, sv, so = oracle.select_views(lex, lg, tpv, 1.5, 0.7, t, 0, lib=lib)
+        if prev is not None:
+            assert np.all(m <= prev)
+        prev = m
+        assert np.array_equal(np.diff(so), (m * tpv[None, :]).sum(axis=1))
+        assert np.array_equal(np.diff(vo), m.sum(axis=1))
+        assert sv.tolist() == [v for b in range(B) for v in range(V) if m[b, v]]
+
+
 ALL_PINS = [pin_bf16_decode, pin_e4m3_decode, pin_worked_example, pin_uniform_keys, pin_single_query_is_softmax,
             pin_row_and_total_sums, pin_batch_equals_single_requests, pin_permutation_equivariance, pin_gqa_replication, pin_scale_placement,
             pin_e4m3_scores, pin_salient_tokens_rank_first, pin_topk_bruteforce, pin_topk_batch_and_ratio,
             pin_table1_token_counts, pin_compact, pin_splice_worked_example, pin_splice_invariants,
-            pin_full_keys_worked_example, pin_full_keys_equal_duplicated_visual_keys]
+            pin_full_keys_worked_example, pin_full_keys_equal_duplicated_visual_keys, pin_views_worked_example,
+            pin_views_properties]

@@ -63,6 +63,13 @@ MUTANTS = [
     ("full_keys_visual_normaliser", "for (int64_t j = 0; j < nk; ++j) z += exp(s[j] - m);",
      "for (int64_t j = sb; j < sb + nb; ++j) z += exp(s[j] - m);"),
     ("full_keys_no_system", "const int64_t nk = sb + nb + i + 1;", "const int64_t nk = nb + i + 1;"),
+    ("views_threshold_not_strict", "const int sel = s[v] > threshold;", "const int sel = s[v] >= threshold;"),
+    ("views_weights_swapped", "const float a = w_lex * lexical[(int64_t)b * num_views + v];",
+     "const float a = w_logit * lexical[(int64_t)b * num_views + v];"),
+    ("views_tie_to_higher_index", "    return ia < ib;\n", "    return ia > ib;\n"),
+    ("views_nan_ranks_first", "    if (an != bn) return bn;\n", "    if (an != bn) return an;\n"),
+    ("views_tokens_of_first_view", "ntok += tokens_per_view[v];", "ntok += tokens_per_view[0];"),
+    ("views_no_fallback", "if (pass < min_views) {", "if (pass < 0) {"),
     ("splice_visual_global_position", "position_ids[r] = S + (g - seq_offsets[b]);", "position_ids[r] = S + g;"),
     ("splice_text_renumbered", "position_ids[r] = S + N + t;", "position_ids[r] = S + k + t;"),
     ("splice_drops_visual", "for (int32_t i = 0; i < k; ++i, ++r) {", "for (int32_t i = 0; i < 0; ++i, ++r) {"),
