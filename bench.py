@@ -384,7 +384,8 @@ def run_ours(args):
     # prefill splice (a next-step row, timed on its own after the step): 32 system rows and
     # the text rows of every request around its kept visual rows, hidden-size rows
     nxt = {"splice": run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk),
-           "full_keys": run_full_keys(w, xd, sel, dev, stream, steps, flush, pk)}
+           "full_keys": run_full_keys(w, xd, sel, dev, stream, steps, flush, pk),
+           "views": run_views(w, sel, dev, stream, steps)}
 
     # end to end through the public API with host buffers
     e2e = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept)
@@ -508,6 +509,39 @@ def run_full_keys(w, xd, sel, dev, stream, steps, flush, pk):
             "extra_us": us["full_keys"] - us["visual_keys"], "system_keys_per_request": n_sys,
             "context_algorithmic_bytes": ctx_bytes,
             "tokens_per_s_M": w.total_vis / (us["full_keys"] * 1e-6) / 1e6}
+
+
+def run_views(w, sel, dev, stream, steps):
+    """litevlm_select_views (patch-selection gating) on the workload's batch x 6
+    camera views (2 tiles x 256 tokens each), timed alone (CUDA events, median)."""
+    import torch
+    from paper_2506_07416_gb300 import inputs, select
+    nv = 6
+    lex, lg = inputs.view_gating_numpy(w.batch, nv, seed=w.seed)
+    lex_d, lg_d = torch.from_numpy(lex).to(dev), torch.from_numpy(lg).to(dev)
+    tpv = np.full(nv, 512, np.int32)
+    mask = torch.empty((w.batch, nv), dtype=torch.uint8, device=dev)
+    vo = torch.empty(w.batch + 1, dtype=torch.int32, device=dev)
+    sv = torch.empty(w.batch * nv, dtype=torch.int32, device=dev)
+    so = torch.empty(w.batch + 1, dtype=torch.int32, device=dev)
+    L = select.LIB
+    args = (sel.handle, w.batch, nv, lex_d.data_ptr(), lg_d.data_ptr(), tpv.ctypes.data, 2.0, 1.0, 1.0, 1,
+            mask.data_ptr(), vo.data_ptr(), sv.data_ptr(), so.data_ptr(), None, stream.cuda_stream)
+    for _ in range(3):
+        assert L.litevlm_select_views(*args) == 0
+    ts = []
+    for _ in range(max(3, min(steps, 200))):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        assert L.litevlm_select_views(*args) == 0
+        e1.record(stream)
+        ts.append((e0, e1))
+    torch.cuda.synchronize()
+    sel.check_device()
+    sel_views = int(vo[-1].item())
+    return {"us_p50": float(np.median([a.elapsed_time(b) for a, b in ts]) * 1e3), "requests": w.batch,
+            "views_per_request": nv, "selected_views": sel_views,
+            "mean_views_selected": sel_views / max(1, w.batch)}
 
 
 def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept):

@@ -169,6 +169,39 @@ litevlm_status_t litevlm_select_score_full_keys(litevlm_select_t handle, int32_t
                                                 litevlm_stream_t stream);
 
 /*
+ * Patch-selection gating, upstream of the scores (Design section, Patch
+ * Selection Module: the final score of a camera view is a weighted sum of the
+ * lexical-mapping score and the module's logit; the views scoring above a
+ * predefined threshold are encoded; Results: 3.5 of 12 patches on average).
+ * For request b and view v, in fp32 with no fused multiply-add:
+ *     s[b][v] = w_lex * lexical[b][v] + w_logit * logits[b][v];  selected <=> s > threshold
+ * When fewer than min_views views pass, the min_views best views are selected
+ * instead (score descending, lower view index first, NaN lowest); min_views = 0
+ * allows an empty selection. The selection fixes N_b for the score path.
+ *   batch             requests, >= 0 (not limited by the handle's maxima)
+ *   num_views         V, 1..64 (camera views per request)
+ *   lexical, logits   device, float [batch, V]
+ *   tokens_per_view_h host, int32 [V] visual tokens each view contributes (>= 0)
+ *   w_lex, w_logit, threshold  the gating weights and threshold (threshold not NaN)
+ *   view_mask         device, uint8 [batch, V]: 1 = selected
+ *   view_offsets      device, int32 [batch+1]: prefix of the selected-view counts
+ *   selected_views    device, int32 [sum of selected views] (at most batch*V): view
+ *                     indices, ascending within each request
+ *   seq_offsets       device, int32 [batch+1]: prefix of N_b = sum of tokens_per_view
+ *                     over the selected views (the score path's seq_offsets)
+ *   seq_offsets_h     optional host int32 [batch+1]: when given, the call copies
+ *                     seq_offsets to it and synchronises the stream before returning
+ * Errors: INVALID_ARG for sizes out of range, a NULL pointer, negative token
+ * counts, a NaN threshold, or batch * sum(tokens_per_view) beyond int32.
+ */
+litevlm_status_t litevlm_select_views(litevlm_select_t handle, int32_t batch, int32_t num_views,
+                                      const float* lexical, const float* logits,
+                                      const int32_t* tokens_per_view_h, float w_lex, float w_logit,
+                                      float threshold, int32_t min_views, uint8_t* view_mask,
+                                      int32_t* view_offsets, int32_t* selected_views, int32_t* seq_offsets,
+                                      int32_t* seq_offsets_h, litevlm_stream_t stream);
+
+/*
  * Per-request top-k (Results section, ratio r of visual tokens kept; Table 1).
  *   scores           device, float [sum N_b]
  *   keep_k_d/h       int32 [batch] tokens to keep per request, 0 <= k_b <= N_b;

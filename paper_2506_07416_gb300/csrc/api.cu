@@ -668,6 +668,56 @@ litevlm_status_t litevlm_select_splice(litevlm_select_t h, int32_t batch, const 
     return LITEVLM_OK;
 }
 
+litevlm_status_t litevlm_select_views(litevlm_select_t h, int32_t batch, int32_t num_views, const float* lexical,
+                                      const float* logits, const int32_t* tokens_per_view_h, float w_lex,
+                                      float w_logit, float threshold, int32_t min_views, uint8_t* view_mask,
+                                      int32_t* view_offsets, int32_t* selected_views, int32_t* seq_offsets,
+                                      int32_t* seq_offsets_h, litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
+    if (num_views < 1 || num_views > lvs::kMaxViews)
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "num_views must be in [1, 64]");
+    if (min_views < 0 || min_views > num_views)
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "min_views must be in [0, num_views]");
+    if (!tokens_per_view_h) return fail(h, LITEVLM_ERR_INVALID_ARG, "tokens_per_view_h is NULL");
+    if (isnan(threshold)) return fail(h, LITEVLM_ERR_INVALID_ARG, "threshold is NaN");
+    int64_t per_request = 0;
+    lvs::ViewsArgs a{};
+    for (int32_t v = 0; v < num_views; ++v) {
+        if (tokens_per_view_h[v] < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "tokens_per_view must be >= 0");
+        per_request += tokens_per_view_h[v];
+        a.tokens_per_view[v] = tokens_per_view_h[v];
+    }
+    if ((int64_t)batch * per_request > INT32_MAX)
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "batch x tokens per request could exceed int32 offsets");
+    if (!view_offsets || !seq_offsets) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
+    if (batch > 0 && (!lexical || !logits || !view_mask || !selected_views))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
+    a.lexical = lexical;
+    a.logits = logits;
+    a.w_lex = w_lex;
+    a.w_logit = w_logit;
+    a.threshold = threshold;
+    a.batch = batch;
+    a.num_views = num_views;
+    a.min_views = min_views;
+    a.view_mask = view_mask;
+    a.view_offsets = view_offsets;
+    a.selected_views = selected_views;
+    a.seq_offsets = seq_offsets;
+    cudaError_t e = lvs::launch_views(a, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "views launch");
+    if (seq_offsets_h) {
+        e = cudaMemcpyAsync(seq_offsets_h, seq_offsets, sizeof(int32_t) * ((size_t)batch + 1), cudaMemcpyDeviceToHost,
+                            (cudaStream_t)stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(h, e, "views: seq_offsets to host");
+    }
+    return LITEVLM_OK;
+}
+
 litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_t stream)
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;

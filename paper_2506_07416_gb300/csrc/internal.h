@@ -173,6 +173,21 @@ struct CtxArgs {
 };
 cudaError_t launch_ctx_stats(const CtxArgs& a, int row_bytes, bool fp8, cudaStream_t stream);
 
+// views.cu: patch-selection gating (views -> N_b)
+constexpr int kMaxViews = 64;
+struct ViewsArgs {
+    const float* lexical;     // [B, V]
+    const float* logits;      // [B, V]
+    float w_lex, w_logit, threshold;
+    int32_t batch, num_views, min_views;
+    int32_t tokens_per_view[kMaxViews];
+    uint8_t* view_mask;       // [B, V]
+    int32_t* view_offsets;    // [B+1]
+    int32_t* selected_views;  // [sum of selected views]
+    int32_t* seq_offsets;     // [B+1]
+};
+cudaError_t launch_views(const ViewsArgs& a, cudaStream_t stream);
+
 // splice.cu
 struct SpliceArgs {
     const int32_t* sys_off;   // device [batch+1]

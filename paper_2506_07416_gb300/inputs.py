@@ -333,3 +333,21 @@ def context_keys_torch(w: Workload, sys_lens: Sequence[int], device, k_scale: fl
         else:
             out[name] = (x / k_scale).clamp(-E4M3_MAX, E4M3_MAX).to(torch.float8_e4m3fn).view(torch.uint8)
     return out
+
+
+# ----------------------------------------------------------------------------
+# patch-selection gating inputs
+# ----------------------------------------------------------------------------
+
+def view_gating_numpy(batch: int, num_views: int = 6, seed: int = 5, lexical_p: float = 0.25,
+                      logit_sigma: float = 2.0, quantum: float = 0.0):
+    """Per-view lexical-mapping scores (1 with probability lexical_p, else 0)
+    and module logits (normal, std logit_sigma; rounded to multiples of quantum
+    when quantum > 0, which produces ties), float32 [batch, num_views]. The
+    paper's setting has 6 cameras of 2 tiles x 256 tokens (12 tiles)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    lex = (rng.random((batch, num_views)) < lexical_p).astype(np.float32)
+    lg = rng.standard_normal((batch, num_views)) * logit_sigma
+    if quantum > 0:
+        lg = np.round(lg / quantum) * quantum
+    return lex, lg.astype(np.float32)

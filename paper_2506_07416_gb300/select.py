@@ -51,6 +51,7 @@ def _load():
     lib.litevlm_status_string.restype = ctypes.c_char_p
     lib.litevlm_select_score.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P]
     lib.litevlm_select_score_full_keys.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, f32, f32, P, P]
+    lib.litevlm_select_views.argtypes = [P, i32, i32, P, P, P, f32, f32, f32, i32, P, P, P, P, P, P]
     lib.litevlm_select_topk.argtypes = [P, i32, P, P, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
@@ -58,7 +59,7 @@ def _load():
     lib.litevlm_select_splice.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, P, P, i64, P, P, P, P, P]
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
     for fn in ("create", "destroy", "score", "score_full_keys", "topk", "compact", "check_device", "score_plan",
-               "score_noalloc", "splice"):
+               "score_noalloc", "splice", "views"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -69,7 +70,7 @@ LIB = _load()
 EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
            "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc",
-           "litevlm_select_splice", "litevlm_select_score_full_keys"]
+           "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -151,6 +152,15 @@ def score_full_keys(handle: int, batch: int, q_text, text_offsets_d, text_offset
                                               _ptr(k_vis), _ptr(seq_offsets_d), _ptr(so_h), _ptr(k_sys),
                                               _ptr(sys_offsets_d), _ptr(yo_h), _ptr(k_text), q_scale, k_scale,
                                               _ptr(scores), _stream_ptr(stream)), handle)
+
+
+def views(handle: int, batch: int, num_views: int, lexical, logits, tokens_per_view_h, w_lex: float, w_logit: float,
+          threshold: float, min_views: int, view_mask, view_offsets, selected_views, seq_offsets,
+          seq_offsets_h: Optional[np.ndarray] = None, stream=None) -> None:
+    tpv = _host_i32(tokens_per_view_h)
+    _check(LIB.litevlm_select_views(handle, batch, num_views, _ptr(lexical), _ptr(logits), _ptr(tpv), w_lex, w_logit,
+                                    threshold, min_views, _ptr(view_mask), _ptr(view_offsets), _ptr(selected_views),
+                                    _ptr(seq_offsets), _ptr(seq_offsets_h), _stream_ptr(stream)), handle)
 
 
 def topk(handle: int, batch: int, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h, keep_ratio: float,
@@ -254,6 +264,23 @@ class Selector:
         score_full_keys(self.handle, len(so_h) - 1, q, text_offsets, to_h, k, seq_offsets, so_h, k_sys, sys_offsets,
                         yo_h, k_text, q_scale, k_scale, out, stream)
         return out
+
+    def select_views(self, lexical, logits, tokens_per_view, w_lex: float, w_logit: float, threshold: float,
+                     min_views: int = 0, stream=None):
+        """Patch-selection gating on float32 CUDA tensors [B, V]. Returns
+        (view_mask, view_offsets, selected_views, seq_offsets device tensors,
+        seq_offsets host numpy; the call synchronises to fill the latter)."""
+        import torch
+        batch, nv = lexical.shape
+        dev = lexical.device
+        mask = torch.empty((max(batch, 1), nv), dtype=torch.uint8, device=dev)
+        vo = torch.empty(batch + 1, dtype=torch.int32, device=dev)
+        sv = torch.empty(max(batch * nv, 1), dtype=torch.int32, device=dev)
+        so = torch.empty(batch + 1, dtype=torch.int32, device=dev)
+        so_h = np.zeros(batch + 1, np.int32)
+        views(self.handle, batch, nv, lexical, logits, tokens_per_view, w_lex, w_logit, threshold, min_views, mask,
+              vo, sv, so, so_h, stream)
+        return mask[:batch], vo, sv, so, so_h
 
     def topk(self, scores, seq_offsets, keep_k=None, keep_ratio: float = 0.0, seq_offsets_h=None, kept_idx=None,
              out_offsets=None, stream=None):
