@@ -72,6 +72,8 @@ def _bind(lib):
     lib.litevlm_oracle_select_views.argtypes = [i32, i32, P, P, P, ctypes.c_float, ctypes.c_float, ctypes.c_float,
                                                  i32, P, P, P, P]
     lib.litevlm_oracle_select_views.restype = ctypes.c_int
+    lib.litevlm_oracle_project.argtypes = [i64, i32, i32, P, P, f64, P, P, i32, P, f64, P]
+    lib.litevlm_oracle_project.restype = ctypes.c_int
     return lib
 
 
@@ -221,6 +223,27 @@ def select_views(lexical: np.ndarray, logits: np.ndarray, tokens_per_view, w_lex
     if rc != 0:
         raise OracleError(f"litevlm_oracle_select_views returned {rc}")
     return mask, vo, sv[:int(vo[-1])], so
+
+
+def project(x_bf16: np.ndarray, gamma, eps: float, w_bf16: np.ndarray, bias=None, head_dim: int = 0,
+            positions=None, rope_base: float = 10000.0, lib=None) -> np.ndarray:
+    """RoPE(W . RMSNorm(x) + bias) in fp64. x_bf16 [rows, H] and w_bf16 [O, H]
+    as uint16 bf16 bits; gamma [H], bias [O] float32; positions int32 [rows].
+    Returns float64 [rows, O]."""
+    lib = lib or load()
+    x = np.ascontiguousarray(x_bf16, dtype=np.uint16)
+    w = np.ascontiguousarray(w_bf16, dtype=np.uint16)
+    rows, hidden = x.shape
+    out_f = w.shape[0]
+    g = np.ascontiguousarray(gamma, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    pos = np.ascontiguousarray(np.zeros(rows, np.int32) if positions is None else positions, dtype=np.int32)
+    y = np.zeros((rows, out_f), np.float64)
+    rc = lib.litevlm_oracle_project(rows, hidden, out_f, _ptr(x), _ptr(g), float(eps), _ptr(w), _ptr(b), head_dim,
+                                    _ptr(pos), float(rope_base), _ptr(y))
+    if rc != 0:
+        raise OracleError(f"litevlm_oracle_project returned {rc}")
+    return y
 
 
 def select(w_inputs: dict, hq: int, hkv: int, head_dim: int, dtype: str, keep_k=None, keep_ratio=0.0,

@@ -44,7 +44,8 @@
  *   R13 N_b = 0 or k_b = 0 give an empty output; N_b > 0 with T_b = 0 is an error.
  *
  * litevlm_oracle_select_views is the patch-selection gating upstream of the
- * path (its readings are stated at the function).
+ * path, litevlm_oracle_project the layer-0 projection that makes q and k
+ * (each states its definition and readings at the function).
  *
  * litevlm_oracle_score_full is the variant without R2 and R3: the normaliser
  * runs over the system, visual and causal text keys of the first decoder
@@ -448,5 +449,60 @@ int litevlm_oracle_select_views(int32_t batch, int32_t num_views, const float* l
         view_offsets[b + 1] = (int32_t)nsel;
         seq_offsets[b + 1] = (int32_t)ntok;
     }
+    return OR_OK;
+}
+
+/*
+ * Layer-0 projection feeding the scores (Design section: the module is the
+ * first decoder layer; its queries and keys are RoPE(W . RMSNorm(x))). For
+ * token row r with hidden x_r (bf16, H values), position p_r:
+ *     s_r   = 1 / sqrt(mean_h x_r[h]^2 + eps)
+ *     y_r[o] = sum_h (x_r[h] * s_r * gamma[h]) * W[o][h] + bias[o]
+ * then, when head_dim > 0, rotary position embedding on each head of head_dim
+ * values, pairing element j with element j + head_dim/2 (rotate-half form):
+ *     theta_j = rope_base^(-2j / head_dim),  a = p_r * theta_j
+ *     y[j]           <- y[j] cos a - y[j + d/2] sin a
+ *     y[j + d/2]     <- y[j + d/2] cos a + y[j] sin a
+ * W is [O, H] bf16 (out x in); gamma [H] and bias [O] (nullable) are fp32;
+ * y is [rows, O] in fp64.
+ */
+int litevlm_oracle_project(int64_t rows, int32_t hidden, int32_t out_features, const uint16_t* x, const float* gamma,
+                           double eps, const uint16_t* w, const float* bias, int32_t head_dim,
+                           const int32_t* positions, double rope_base, double* y)
+{
+    if (rows < 0 || hidden <= 0 || out_features <= 0 || head_dim < 0) return OR_ERR_ARG;
+    if (head_dim > 0 && (head_dim % 2 != 0 || out_features % head_dim != 0)) return OR_ERR_ARG;
+    double* xn = (double*)malloc((size_t)hidden * sizeof(double));
+    if (!xn) return OR_ERR_NOMEM;
+    for (int64_t r = 0; r < rows; ++r) {
+        double ss = 0.0;
+        for (int32_t h = 0; h < hidden; ++h) {
+            const double v = litevlm_oracle_decode(OR_BF16, x, r * hidden + h);
+            xn[h] = v;
+            ss += v * v;
+        }
+        const double s = 1.0 / sqrt(ss / (double)hidden + eps);
+        for (int32_t h = 0; h < hidden; ++h) xn[h] = xn[h] * s * (double)gamma[h];
+        double* yr = y + r * out_features;
+        for (int32_t o = 0; o < out_features; ++o) {
+            double acc = 0.0;
+            for (int32_t h = 0; h < hidden; ++h)
+                acc += xn[h] * litevlm_oracle_decode(OR_BF16, w, (int64_t)o * hidden + h);
+            yr[o] = acc + (bias ? (double)bias[o] : 0.0);
+        }
+        if (head_dim > 0) {
+            const int32_t half = head_dim / 2;
+            for (int32_t h0 = 0; h0 < out_features; h0 += head_dim) {
+                for (int32_t j = 0; j < half; ++j) {
+                    const double theta = pow(rope_base, -2.0 * (double)j / (double)head_dim);
+                    const double a = (double)positions[r] * theta;
+                    const double y1 = yr[h0 + j], y2 = yr[h0 + j + half];
+                    yr[h0 + j] = y1 * cos(a) - y2 * sin(a);
+                    yr[h0 + j + half] = y2 * cos(a) + y1 * sin(a);
+                }
+            }
+        }
+    }
+    free(xn);
     return OR_OK;
 }

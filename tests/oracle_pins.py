@@ -442,9 +442,71 @@ def pin_views_properties(lib):
         assert sv.tolist() == [v for b in range(B) for v in range(V) if m[b, v]]
 
 
+# ---------------------------------------------------------------------------
+# layer-0 projection (RMSNorm -> W -> RoPE)
+# ---------------------------------------------------------------------------
+
+def _bf(a):
+    return inputs.f32_to_bf16_bits(np.asarray(a, np.float32))
+
+
+def pin_project_worked_example(lib):
+    """Hand-worked rows, H = O = head_dim = 4, eps = 0 unless stated:
+      x = [3,4,0,0], W = I, p = 1, base 1e4: rms 2.5 -> [1.2,1.6,0,0]; pairs (0,2),
+        (1,3) with theta = 1, 0.01 -> [1.2 cos 1, 1.6 cos .01, 1.2 sin 1, 1.6 sin .01]
+      x = [0,0,0,5], p = 2: -> [0, -2 sin .02, 0, 2 cos .02]
+      no RoPE, gamma = [2,1,1,1], bias = [1,0,0,0], x = [3,4,0,0]: [3.4, 1.6, 0, 0]
+      eps = 3, x = [1,1,1,1], W = I: every output 1/sqrt(1 + 3) = 0.5
+      W with one 1 at [0][1], x = [1,3,1,1]: rms sqrt(3) -> y = [sqrt 3, 0, 0, 0]"""
+    eye = _bf(np.eye(4))
+    one = np.ones(4, np.float32)
+    y = oracle.project(_bf([[3, 4, 0, 0], [0, 0, 0, 5]]), one, 0.0, eye, None, 4, [1, 2], 1e4, lib=lib)
+    np.testing.assert_allclose(y[0], [1.2 * math.cos(1), 1.6 * math.cos(0.01), 1.2 * math.sin(1),
+                                      1.6 * math.sin(0.01)], rtol=1e-14, atol=1e-15)
+    np.testing.assert_allclose(y[1], [0, -2 * math.sin(0.02), 0, 2 * math.cos(0.02)], rtol=1e-14, atol=1e-15)
+    y = oracle.project(_bf([[3, 4, 0, 0]]), [2, 1, 1, 1], 0.0, eye, [1, 0, 0, 0], 0, None, lib=lib)
+    np.testing.assert_allclose(y[0], [3.4, 1.6, 0, 0], rtol=1e-14, atol=1e-15)
+    y = oracle.project(_bf([[1, 1, 1, 1]]), one, 3.0, eye, None, 0, None, lib=lib)
+    np.testing.assert_allclose(y[0], [0.5] * 4, rtol=1e-14)
+    w = np.zeros((4, 4), np.float32)
+    w[0, 1] = 1.0
+    y = oracle.project(_bf([[1, 3, 1, 1]]), one, 0.0, _bf(w), None, 0, None, lib=lib)
+    np.testing.assert_allclose(y[0], [math.sqrt(3), 0, 0, 0], rtol=1e-14, atol=1e-15)
+
+
+def pin_project_properties(lib):
+    """Random rows and weights (H 48, two heads of 16): RoPE keeps each head's
+    norm, and rotated query . key depends only on the position difference;
+    scaling x by a power of two leaves y unchanged (eps 0); doubling gamma
+    doubles y; with W = I, gamma 1 and no bias or RoPE every row has mean
+    square 1 (a mean over H, not a sum)."""
+    rng = np.random.Generator(np.random.PCG64(41))
+    H, O, d = 48, 32, 16
+    x = _bf(rng.standard_normal((6, H)))
+    w = _bf(rng.standard_normal((O, H)) / math.sqrt(H))
+    g = rng.uniform(0.5, 1.5, H).astype(np.float32)
+    base = oracle.project(x, g, 0.0, w, None, 0, None, lib=lib)
+    pos = np.array([0, 3, 17, 100, 2048, 5], np.int32)
+    rot = oracle.project(x, g, 0.0, w, None, d, pos, 1e4, lib=lib)
+    for h in range(O // d):
+        np.testing.assert_allclose(np.linalg.norm(rot[:, h * d:(h + 1) * d], axis=1),
+                                   np.linalg.norm(base[:, h * d:(h + 1) * d], axis=1), rtol=1e-12)
+    shift = oracle.project(x, g, 0.0, w, None, d, pos + 37, 1e4, lib=lib)
+    for i, j in ((0, 1), (2, 5), (3, 4)):
+        for h in range(O // d):
+            sl = slice(h * d, (h + 1) * d)
+            assert abs(rot[i, sl] @ rot[j, sl] - shift[i, sl] @ shift[j, sl]) < 1e-10
+    xs = inputs.f32_to_bf16_bits(inputs.bf16_bits_to_f32(x) * 8.0)
+    np.testing.assert_allclose(oracle.project(xs, g, 0.0, w, None, 0, None, lib=lib), base, rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(oracle.project(x, 2 * g, 0.0, w, None, 0, None, lib=lib), 2 * base, rtol=1e-12,
+                               atol=1e-14)
+    y = oracle.project(x, np.ones(H, np.float32), 0.0, _bf(np.eye(H)), None, 0, None, lib=lib)
+    np.testing.assert_allclose(np.mean(y * y, axis=1), 1.0, rtol=1e-12)
+
+
 ALL_PINS = [pin_bf16_decode, pin_e4m3_decode, pin_worked_example, pin_uniform_keys, pin_single_query_is_softmax,
             pin_row_and_total_sums, pin_batch_equals_single_requests, pin_permutation_equivariance, pin_gqa_replication, pin_scale_placement,
             pin_e4m3_scores, pin_salient_tokens_rank_first, pin_topk_bruteforce, pin_topk_batch_and_ratio,
             pin_table1_token_counts, pin_compact, pin_splice_worked_example, pin_splice_invariants,
             pin_full_keys_worked_example, pin_full_keys_equal_duplicated_visual_keys, pin_views_worked_example,
-            pin_views_properties]
+            pin_views_properties, pin_project_worked_example, pin_project_properties]

@@ -70,6 +70,18 @@ MUTANTS = [
     ("views_nan_ranks_first", "    if (an != bn) return bn;\n", "    if (an != bn) return an;\n"),
     ("views_tokens_of_first_view", "ntok += tokens_per_view[v];", "ntok += tokens_per_view[0];"),
     ("views_no_fallback", "if (pass < min_views) {", "if (pass < 0) {"),
+    ("project_rms_sum", "const double s = 1.0 / sqrt(ss / (double)hidden + eps);",
+     "const double s = 1.0 / sqrt(ss + eps);"),
+    ("project_eps_outside", "const double s = 1.0 / sqrt(ss / (double)hidden + eps);",
+     "const double s = 1.0 / (sqrt(ss / (double)hidden) + eps);"),
+    ("project_no_gamma", "xn[h] = xn[h] * s * (double)gamma[h];", "xn[h] = xn[h] * s;"),
+    ("project_weight_transposed", "acc += xn[h] * litevlm_oracle_decode(OR_BF16, w, (int64_t)o * hidden + h);",
+     "acc += xn[h] * litevlm_oracle_decode(OR_BF16, w, (int64_t)h * out_features + o);"),
+    ("project_no_bias", "yr[o] = acc + (bias ? (double)bias[o] : 0.0);", "yr[o] = acc;"),
+    ("project_rope_sign", "yr[h0 + j] = y1 * cos(a) - y2 * sin(a);", "yr[h0 + j] = y1 * cos(a) + y2 * sin(a);"),
+    ("project_rope_frequency", "pow(rope_base, -2.0 * (double)j / (double)head_dim)",
+     "pow(rope_base, -1.0 * (double)j / (double)head_dim)"),
+    ("project_rope_adjacent_pairs", "const int32_t half = head_dim / 2;", "const int32_t half = 1;"),
     ("splice_visual_global_position", "position_ids[r] = S + (g - seq_offsets[b]);", "position_ids[r] = S + g;"),
     ("splice_text_renumbered", "position_ids[r] = S + N + t;", "position_ids[r] = S + k + t;"),
     ("splice_drops_visual", "for (int32_t i = 0; i < k; ++i, ++r) {", "for (int32_t i = 0; i < 0; ++i, ++r) {"),
