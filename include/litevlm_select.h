@@ -202,6 +202,52 @@ litevlm_status_t litevlm_select_views(litevlm_select_t handle, int32_t batch, in
                                       int32_t* seq_offsets_h, litevlm_stream_t stream);
 
 /*
+ * Layer-0 projection that makes q and k for the scores (Design section: the
+ * module is the first decoder layer of the LLM, whose queries and keys are
+ * RoPE(W . RMSNorm(x))). Three calls:
+ *
+ * litevlm_select_fold_norm: w_folded[o][h] = bf16(w[o][h] * gamma[h]) -- the
+ * RMSNorm weight folded into the projection weight, once per weight matrix.
+ *   w, w_folded  device bf16 [out_features, hidden] (nn.Linear layout: out x in)
+ *   gamma        device float [hidden]
+ *
+ * litevlm_select_rope_table: table[p][j] = (cos a, sin a), a = p * theta_j in
+ * fp32 with theta_j = rope_base^(-2j / head_dim) rounded to fp32, for
+ * p < max_positions, j < head_dim / 2.
+ *   table        device float [max_positions][head_dim / 2][2]; head_dim 64 or 128
+ *
+ * litevlm_select_project: for each row r of x,
+ *     s_r = 1 / sqrt(mean_h x[r][h]^2 + eps)
+ *     y[r][o] = s_r * sum_h x[r][h] * w_folded[o][h] + bias[o]
+ * then, when head_dim > 0, each head of head_dim outputs is rotated: element
+ * j pairs with j + head_dim/2, (y1, y2) -> (y1 cos - y2 sin, y2 cos + y1 sin)
+ * with (cos, sin) = table[positions[r]][j]. One tcgen05 contraction per
+ * 128 x 256 (or 128) output tile; the row scale, bias and rotation are applied
+ * to the fp32 accumulator, which is rounded once to bf16.
+ *   rows             >= 0 token rows; hidden a multiple of 8; out_features a multiple of 128
+ *   x                device bf16 [rows, hidden];  y device bf16 [rows, out_features]
+ *                    (= [rows, heads, head_dim], the layout litevlm_select_score reads)
+ *   bias             device float [out_features] or NULL
+ *   eps              >= 0
+ *   head_dim         0 (no rotation), 64 or 128
+ *   positions        device int32 [rows] (with head_dim > 0); a position outside
+ *                    [0, max_positions) uses row 0 of the table and sets DEVICE_BOUNDS
+ *   rope_table       device, from litevlm_select_rope_table with the same head_dim
+ * x, w_folded and y must be 16-byte aligned. Errors: INVALID_ARG / UNSUPPORTED
+ * for sizes, pointers or head_dim outside the above.
+ */
+litevlm_status_t litevlm_select_fold_norm(litevlm_select_t handle, int32_t out_features, int32_t hidden,
+                                          const void* w, const float* gamma, void* w_folded,
+                                          litevlm_stream_t stream);
+litevlm_status_t litevlm_select_rope_table(litevlm_select_t handle, int32_t max_positions, int32_t head_dim,
+                                           float rope_base, float* table, litevlm_stream_t stream);
+litevlm_status_t litevlm_select_project(litevlm_select_t handle, int64_t rows, int32_t hidden,
+                                        int32_t out_features, const void* x, const void* w_folded,
+                                        const float* bias, float eps, int32_t head_dim,
+                                        const int32_t* positions, const float* rope_table,
+                                        int32_t max_positions, void* y, litevlm_stream_t stream);
+
+/*
  * Per-request top-k (Results section, ratio r of visual tokens kept; Table 1).
  *   scores           device, float [sum N_b]
  *   keep_k_d/h       int32 [batch] tokens to keep per request, 0 <= k_b <= N_b;

@@ -17,7 +17,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 OBJ = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "liblitevlm_select.so")
-SOURCES = ["api.cu", "score_tc.cu", "score_res.cu", "ctx_stats.cu", "topk.cu", "compact.cu", "splice.cu", "views.cu"]
+SOURCES = ["api.cu", "score_tc.cu", "score_res.cu", "ctx_stats.cu", "topk.cu", "compact.cu", "splice.cu", "views.cu", "proj.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -718,6 +718,85 @@ litevlm_status_t litevlm_select_views(litevlm_select_t h, int32_t batch, int32_t
     return LITEVLM_OK;
 }
 
+litevlm_status_t litevlm_select_fold_norm(litevlm_select_t h, int32_t out_features, int32_t hidden, const void* w,
+                                          const float* gamma, void* w_folded, litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (out_features <= 0 || hidden <= 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "sizes must be > 0");
+    if (!w || !gamma || !w_folded) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
+    const cudaError_t e = lvs::launch_fold_norm(static_cast<const __nv_bfloat16*>(w), gamma,
+                                                static_cast<__nv_bfloat16*>(w_folded),
+                                                (int64_t)out_features * hidden, hidden, h->num_sms,
+                                                (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "fold_norm launch");
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_rope_table(litevlm_select_t h, int32_t max_positions, int32_t head_dim,
+                                           float rope_base, float* table, litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (max_positions <= 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "max_positions must be > 0");
+    if (head_dim != 64 && head_dim != 128) return fail(h, LITEVLM_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
+    if (!(rope_base > 1.f) || isinf(rope_base)) return fail(h, LITEVLM_ERR_INVALID_ARG, "rope_base must be > 1");
+    if (!table) return fail(h, LITEVLM_ERR_INVALID_ARG, "table is NULL");
+    lvs::RopeArgs a{};
+    a.table = reinterpret_cast<float2*>(table);
+    a.max_positions = max_positions;
+    a.half = head_dim / 2;
+    for (int j = 0; j < a.half; ++j) a.inv_freq[j] = (float)pow((double)rope_base, -2.0 * j / (double)head_dim);
+    const cudaError_t e = lvs::launch_rope_table(a, h->num_sms, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "rope_table launch");
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_t hidden, int32_t out_features,
+                                        const void* x, const void* w_folded, const float* bias, float eps,
+                                        int32_t head_dim, const int32_t* positions, const float* rope_table,
+                                        int32_t max_positions, void* y, litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (rows < 0 || rows > INT32_MAX) return fail(h, LITEVLM_ERR_INVALID_ARG, "rows must be in [0, 2^31)");
+    if (hidden <= 0 || hidden % 8 != 0)
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "hidden must be a positive multiple of 8 (16-byte rows)");
+    if (out_features <= 0 || out_features % 128 != 0)
+        return fail(h, LITEVLM_ERR_UNSUPPORTED, "out_features must be a positive multiple of 128");
+    if (head_dim != 0 && head_dim != 64 && head_dim != 128)
+        return fail(h, LITEVLM_ERR_UNSUPPORTED, "head_dim must be 0 (no rotation), 64 or 128");
+    if (!(eps >= 0.f) || isinf(eps)) return fail(h, LITEVLM_ERR_INVALID_ARG, "eps must be finite and >= 0");
+    if (rows == 0) return LITEVLM_OK;
+    if (!x || !w_folded || !y) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
+    if (!aligned16(x) || !aligned16(w_folded) || !aligned16(y))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "x, w_folded and y must be 16-byte aligned");
+    if (head_dim > 0 && (!positions || !rope_table || max_positions <= 0))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "positions, rope_table and max_positions are required with RoPE");
+    const int bn = lvs::proj_tile_cols(out_features);
+    CUtensorMap tm_x, tm_w;
+    litevlm_status_t s = encode_rows_map(h, &tm_x, x, hidden, 1, rows, 128, false, "x");
+    if (s != LITEVLM_OK) return s;
+    s = encode_rows_map(h, &tm_w, w_folded, hidden, 1, out_features, bn, false, "w_folded");
+    if (s != LITEVLM_OK) return s;
+    lvs::ProjArgs p{};
+    p.rows = rows;
+    p.hidden = hidden;
+    p.out_features = out_features;
+    p.head_dim = head_dim;
+    p.max_positions = max_positions;
+    p.eps = eps;
+    p.bias = bias;
+    p.positions = positions;
+    p.rope = reinterpret_cast<const float2*>(rope_table);
+    p.y = static_cast<__nv_bfloat16*>(y);
+    p.err = h->err_d;
+    p.wait_budget = lvs::kWaitBudgetCycles;
+    const cudaError_t e = lvs::launch_proj(tm_x, tm_w, p, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "project launch");
+    return LITEVLM_OK;
+}
+
 litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_t stream)
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;

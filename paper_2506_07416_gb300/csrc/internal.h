@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -187,6 +188,29 @@ struct ViewsArgs {
     int32_t* seq_offsets;     // [B+1]
 };
 cudaError_t launch_views(const ViewsArgs& a, cudaStream_t stream);
+
+// proj.cu: layer-0 projection RoPE(s_r * x W'^T + bias), W' = W * gamma
+struct ProjArgs {
+    int64_t rows;
+    int32_t hidden, out_features, head_dim, max_positions;
+    float eps;
+    const float* bias;        // [O] or null
+    const int32_t* positions; // [rows] (head_dim > 0)
+    const float2* rope;       // [max_positions][head_dim / 2] (cos, sin)
+    __nv_bfloat16* y;         // [rows, O]
+    int32_t* err;
+    long long wait_budget;
+};
+struct RopeArgs {
+    float2* table;            // [max_positions][half]
+    int32_t max_positions, half;
+    float inv_freq[128];      // rope_base^(-2j / head_dim), rounded to fp32
+};
+int proj_tile_cols(int out_features);
+cudaError_t launch_proj(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const ProjArgs& p, cudaStream_t stream);
+cudaError_t launch_fold_norm(const __nv_bfloat16* w, const float* gamma, __nv_bfloat16* out, int64_t total,
+                             int hidden, int num_sms, cudaStream_t stream);
+cudaError_t launch_rope_table(const RopeArgs& a, int num_sms, cudaStream_t stream);
 
 // splice.cu
 struct SpliceArgs {

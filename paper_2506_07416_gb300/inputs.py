@@ -351,3 +351,21 @@ def view_gating_numpy(batch: int, num_views: int = 6, seed: int = 5, lexical_p: 
     if quantum > 0:
         lg = np.round(lg / quantum) * quantum
     return lex, lg.astype(np.float32)
+
+
+# ----------------------------------------------------------------------------
+# layer-0 projection inputs (random weights of the decoder layer's shapes)
+# ----------------------------------------------------------------------------
+
+def projection_numpy(rows: int, hidden: int, out_features: int, seed: int = 6, bias: bool = False,
+                     max_position: int = 4096):
+    """Hidden rows x ~ N(0, 1) (bf16 bits), RMSNorm weight gamma ~ U(0.5, 1.5),
+    projection weight W ~ N(0, 1/hidden) (bf16 bits, [out, in]), optional bias
+    ~ N(0, 0.1), and positions drawn uniformly below max_position."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    x = f32_to_bf16_bits(rng.standard_normal((rows, hidden)).astype(np.float32))
+    gamma = rng.uniform(0.5, 1.5, hidden).astype(np.float32)
+    w = f32_to_bf16_bits((rng.standard_normal((out_features, hidden)) / math.sqrt(hidden)).astype(np.float32))
+    b = (rng.standard_normal(out_features) * 0.1).astype(np.float32) if bias else None
+    pos = rng.integers(0, max_position, rows).astype(np.int32)
+    return x, gamma, w, b, pos

@@ -52,6 +52,9 @@ def _load():
     lib.litevlm_select_score.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P]
     lib.litevlm_select_score_full_keys.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, f32, f32, P, P]
     lib.litevlm_select_views.argtypes = [P, i32, i32, P, P, P, f32, f32, f32, i32, P, P, P, P, P, P]
+    lib.litevlm_select_fold_norm.argtypes = [P, i32, i32, P, P, P, P]
+    lib.litevlm_select_rope_table.argtypes = [P, i32, i32, f32, P, P]
+    lib.litevlm_select_project.argtypes = [P, i64, i32, i32, P, P, P, f32, i32, P, P, i32, P, P]
     lib.litevlm_select_topk.argtypes = [P, i32, P, P, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
@@ -59,7 +62,7 @@ def _load():
     lib.litevlm_select_splice.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, P, P, i64, P, P, P, P, P]
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
     for fn in ("create", "destroy", "score", "score_full_keys", "topk", "compact", "check_device", "score_plan",
-               "score_noalloc", "splice", "views"):
+               "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -70,7 +73,8 @@ LIB = _load()
 EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_last_error",
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
            "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc",
-           "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views"]
+           "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views",
+           "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -161,6 +165,23 @@ def views(handle: int, batch: int, num_views: int, lexical, logits, tokens_per_v
     _check(LIB.litevlm_select_views(handle, batch, num_views, _ptr(lexical), _ptr(logits), _ptr(tpv), w_lex, w_logit,
                                     threshold, min_views, _ptr(view_mask), _ptr(view_offsets), _ptr(selected_views),
                                     _ptr(seq_offsets), _ptr(seq_offsets_h), _stream_ptr(stream)), handle)
+
+
+def fold_norm(handle: int, out_features: int, hidden: int, w, gamma, w_folded, stream=None) -> None:
+    _check(LIB.litevlm_select_fold_norm(handle, out_features, hidden, _ptr(w), _ptr(gamma), _ptr(w_folded),
+                                        _stream_ptr(stream)), handle)
+
+
+def rope_table(handle: int, max_positions: int, head_dim: int, rope_base: float, table, stream=None) -> None:
+    _check(LIB.litevlm_select_rope_table(handle, max_positions, head_dim, rope_base, _ptr(table),
+                                         _stream_ptr(stream)), handle)
+
+
+def project(handle: int, rows: int, hidden: int, out_features: int, x, w_folded, bias, eps: float, head_dim: int,
+            positions, table, max_positions: int, y, stream=None) -> None:
+    _check(LIB.litevlm_select_project(handle, rows, hidden, out_features, _ptr(x), _ptr(w_folded), _ptr(bias), eps,
+                                      head_dim, _ptr(positions), _ptr(table), max_positions, _ptr(y),
+                                      _stream_ptr(stream)), handle)
 
 
 def topk(handle: int, batch: int, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h, keep_ratio: float,
@@ -281,6 +302,31 @@ class Selector:
         views(self.handle, batch, nv, lexical, logits, tokens_per_view, w_lex, w_logit, threshold, min_views, mask,
               vo, sv, so, so_h, stream)
         return mask[:batch], vo, sv, so, so_h
+
+    def fold_norm(self, w, gamma, stream=None):
+        """bf16 W * gamma (per input column) for project()."""
+        import torch
+        out = torch.empty_like(w)
+        fold_norm(self.handle, w.shape[0], w.shape[1], w, gamma, out, stream)
+        return out
+
+    def rope_table(self, max_positions: int, head_dim: int, rope_base: float, device="cuda", stream=None):
+        import torch
+        t = torch.empty((max_positions, head_dim // 2, 2), dtype=torch.float32, device=device)
+        rope_table(self.handle, max_positions, head_dim, rope_base, t, stream)
+        return t
+
+    def project(self, x, w_folded, bias=None, eps: float = 1e-6, head_dim: int = 0, positions=None, table=None,
+                out=None, stream=None):
+        """y = RoPE(RMS-scale(x) . w_folded^T + bias), bf16 [rows, out_features]."""
+        import torch
+        rows, hidden = x.shape
+        out_f = w_folded.shape[0]
+        if out is None:
+            out = torch.empty((rows, out_f), dtype=torch.bfloat16, device=x.device)
+        project(self.handle, rows, hidden, out_f, x, w_folded, bias, eps, head_dim, positions, table,
+                0 if table is None else table.shape[0], out, stream)
+        return out
 
     def topk(self, scores, seq_offsets, keep_k=None, keep_ratio: float = 0.0, seq_offsets_h=None, kept_idx=None,
              out_offsets=None, stream=None):
