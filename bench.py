@@ -385,7 +385,8 @@ def run_ours(args):
     # the text rows of every request around its kept visual rows, hidden-size rows
     nxt = {"splice": run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk),
            "full_keys": run_full_keys(w, xd, sel, dev, stream, steps, flush, pk),
-           "views": run_views(w, sel, dev, stream, steps)}
+           "views": run_views(w, sel, dev, stream, steps),
+           "project": run_project(w, xd, sel, dev, stream, steps, pk)}
 
     # end to end through the public API with host buffers
     e2e = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept)
@@ -509,6 +510,58 @@ def run_full_keys(w, xd, sel, dev, stream, steps, flush, pk):
             "extra_us": us["full_keys"] - us["visual_keys"], "system_keys_per_request": n_sys,
             "context_algorithmic_bytes": ctx_bytes,
             "tokens_per_s_M": w.total_vis / (us["full_keys"] * 1e-6) / 1e6}
+
+
+def run_project(w, xd, sel, dev, stream, steps, pk):
+    """litevlm_select_project: the keys of the workload's visual rows from their
+    hidden states (RMSNorm folded into a random W_k [Hkv*d, hidden], RoPE at
+    positions 32 + j), at most 65536 rows, timed alone (CUDA events, median),
+    with a plain cuBLAS bf16 GEMM of the same shape (no norm, no rotation) timed
+    beside it for reference."""
+    import torch
+    from paper_2506_07416_gb300 import select
+    rows = min(w.total_vis, 65536)
+    H, O, d = w.hidden, w.hkv * w.head_dim, w.head_dim
+    if O % 128 != 0 or H % 8 != 0:
+        return None
+    g = torch.Generator(device=dev).manual_seed(17)
+    x = xd["hidden"][:rows]
+    wk = (torch.randn((O, H), generator=g, device=dev) / H ** 0.5).to(torch.bfloat16)
+    gamma = torch.rand(H, generator=g, device=dev) + 0.5
+    wf = sel.fold_norm(wk, gamma)
+    table = sel.rope_table(rows + 64, d, 1e6)
+    pos = (torch.arange(rows, device=dev, dtype=torch.int32) + 32).contiguous()
+    y = torch.empty((rows, O), dtype=torch.bfloat16, device=dev)
+    L = select.LIB
+    args = (sel.handle, rows, H, O, x.data_ptr(), wf.data_ptr(), None, 1e-6, d, pos.data_ptr(), table.data_ptr(),
+            rows + 64, y.data_ptr(), stream.cuda_stream)
+    n = max(3, min(steps, 50))
+    res = {}
+    def ours():
+        assert L.litevlm_select_project(*args) == 0
+
+    def plain():
+        torch.matmul(x, wk.t(), out=y)
+
+    for name, fn in (("ours", ours), ("cublas_plain_gemm", plain)):
+        for _ in range(3):
+            fn()
+        ts = []
+        for _ in range(n):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            ts.append((e0, e1))
+        torch.cuda.synchronize()
+        res[name] = float(np.median([a.elapsed_time(b) for a, b in ts]) * 1e3)
+    sel.check_device()
+    flops = 2.0 * rows * H * O
+    tf = flops / (res["ours"] * 1e-6) / 1e12
+    return {"rows": rows, "hidden": H, "out_features": O, "head_dim": d, "us_p50": res["ours"],
+            "tflops": tf, "frac_of_bf16_peak": tf / pk["bf16_tflops"],
+            "cublas_plain_gemm_us_p50": res["cublas_plain_gemm"],
+            "cublas_plain_gemm_tflops": flops / (res["cublas_plain_gemm"] * 1e-6) / 1e12}
 
 
 def run_views(w, sel, dev, stream, steps):

@@ -224,7 +224,7 @@ litevlm_status_t litevlm_select_views(litevlm_select_t handle, int32_t batch, in
  * with (cos, sin) = table[positions[r]][j]. One tcgen05 contraction per
  * 128 x 256 (or 128) output tile; the row scale, bias and rotation are applied
  * to the fp32 accumulator, which is rounded once to bf16.
- *   rows             >= 0 token rows; hidden a multiple of 8; out_features a multiple of 128
+ *   rows             0 .. 65535 * 128 token rows; hidden a multiple of 8; out_features a multiple of 128
  *   x                device bf16 [rows, hidden];  y device bf16 [rows, out_features]
  *                    (= [rows, heads, head_dim], the layout litevlm_select_score reads)
  *   bias             device float [out_features] or NULL

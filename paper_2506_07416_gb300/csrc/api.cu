@@ -759,7 +759,7 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
-    if (rows < 0 || rows > INT32_MAX) return fail(h, LITEVLM_ERR_INVALID_ARG, "rows must be in [0, 2^31)");
+    if (rows < 0 || rows > 65535LL * 128) return fail(h, LITEVLM_ERR_INVALID_ARG, "rows must be in [0, 65535 * 128]");
     if (hidden <= 0 || hidden % 8 != 0)
         return fail(h, LITEVLM_ERR_INVALID_ARG, "hidden must be a positive multiple of 8 (16-byte rows)");
     if (out_features <= 0 || out_features % 128 != 0)

@@ -61,8 +61,10 @@ __global__ void __launch_bounds__(kProjThreads, 1)
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t* smem = smem_raw + (base - raw);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t m0 = (int64_t)blockIdx.x * 128;
-    const int n0 = (int)blockIdx.y * BN;
+    // N tiles run fastest: the CTAs in flight share their A rows (read from DRAM
+    // once, then from L2), and W' (all N tiles) stays in L2
+    const int64_t m0 = (int64_t)blockIdx.y * 128;
+    const int n0 = (int)blockIdx.x * BN;
     const int nk = (p.hidden + kProjK - 1) / kProjK;
 
     const uint32_t bar0 = base + L::OFF_BAR;
@@ -285,7 +287,7 @@ cudaError_t launch_proj_variant(const CUtensorMap& tm_x, const CUtensorMap& tm_w
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)((p.rows + 127) / 128), (unsigned)(p.out_features / BN), 1);
+    cfg.gridDim = dim3((unsigned)(p.out_features / BN), (unsigned)((p.rows + 127) / 128), 1);
     cfg.blockDim = dim3(kProjThreads, 1, 1);
     cfg.dynamicSmemBytes = L::ALLOC;
     cfg.stream = stream;

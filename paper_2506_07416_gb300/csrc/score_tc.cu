@@ -29,8 +29,9 @@
 // several the CTAs write partial rows and the last CTA of the request to finish
 // (atomic ticket) adds them in a fixed order.
 //
-// Warp roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
-// MMA issuer, warps 2..5 = epilogue (TMEM lane quadrant = warp % 4).
+// Warp roles (320 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
+// MMA issuer, warps 2..9 = epilogue in two warpgroups (TMEM lane quadrant =
+// warp % 4); warpgroup g takes the tiles that land in TMEM buffer g of a pass.
 // Every wait is bounded (clock budget); on expiry the kernel sets the error
 // word, drains its own copies and MMAs, frees TMEM and returns.
 
@@ -44,7 +45,7 @@ namespace lvs {
 
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
 constexpr int kStatSlots = 4;  // stats of heads s-3..s may be live across the cluster
 
 // Shared-memory plan. The ring gets whatever is left of the 227 KB after the
@@ -60,7 +61,7 @@ struct SmemLayout {
     // Q(s+2) load while pass 2 of head s is still reading Q(s).
     static constexpr int QBUF = MROWS == 64 ? 3 : 2;
     static constexpr int FIXED = QBUF * Q_BYTES + kMaxTilesPerCta * kTileRows * 4 + kStatSlots * kMaxText * 8 +
-                                 2 * kMaxText * 4 + kMaxTilesPerCta * 4 + 512 + 64 + 1024;
+                                 2 * kMaxText * 4 + kMaxText * 8 + kMaxTilesPerCta * 4 + 512 + 64 + 1024;
     static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
     static constexpr int kStages = STAGES_FIT > 10 ? 10 : STAGES_FIT;
     static constexpr int OFF_K = 0;
@@ -68,7 +69,8 @@ struct SmemLayout {
     static constexpr int OFF_ACC = OFF_Q + QBUF * Q_BYTES;
     static constexpr int OFF_STATS = OFF_ACC + kMaxTilesPerCta * kTileRows * 4;
     static constexpr int OFF_B2 = OFF_STATS + kStatSlots * kMaxText * 8;
-    static constexpr int OFF_FLAGS = OFF_B2 + 2 * kMaxText * 4;   // [32] int, fold flags
+    static constexpr int OFF_XS = OFF_B2 + 2 * kMaxText * 4;      // [128] float2: warpgroup 1's row statistics
+    static constexpr int OFF_FLAGS = OFF_XS + kMaxText * 8;       // [32] int, fold flags
     static constexpr int OFF_BAR = OFF_FLAGS + kMaxTilesPerCta * 4;
     // k_full[S], k_empty[S], q_full[QBUF], q_empty[QBUF], t1_full[2], t1_empty[2],
     // t2_full[2], t2_empty[2], stats[4], drain
@@ -142,6 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* acc_s = reinterpret_cast<float*>(smem + L::OFF_ACC);
     float2* stats_s = reinterpret_cast<float2*>(smem + L::OFF_STATS);
     float* b2_s = reinterpret_cast<float*>(smem + L::OFF_B2);
+    float2* xs_s = reinterpret_cast<float2*>(smem + L::OFF_XS);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -154,7 +157,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(BAR(T1_FULL + i), 1);
-            mbar_init(BAR(T1_EMPTY + i), 4);   // one arrival per epilogue warp
+            mbar_init(BAR(T1_EMPTY + i), 4);   // one arrival per warp of the consuming warpgroup
             mbar_init(BAR(T2_FULL + i), 1);
             mbar_init(BAR(T2_EMPTY + i), 4);
         }
@@ -288,41 +291,41 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        // Control flow here is identical for all 128 threads (named barriers);
-        // after an abort every wait returns at once and the steps run out.
+        // Two warpgroups (warps 2-5 and 6-9). The two TMEM buffers of each pass
+        // alternate from tile to tile; warpgroup g takes the tiles that land in
+        // buffer g, so both work at once. Control flow is identical within a
+        // warpgroup (named barriers); after an abort every wait returns at once
+        // and the steps run out.
         const int quad = warp & 3;
-        const int et = threadIdx.x - 64;                      // 0..127
+        const int wg = (warp - 2) >> 2;                       // 0 or 1
+        const int et = threadIdx.x - 64;                      // 0..255
         const int vrow = quad * 32 + lane;                    // pass 2: TMEM lane = visual token in tile
         const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
         // pass 1 row of this thread: M=128 -> lane; M=64 -> lanes 16q..16q+15, two column halves
         const int prow = MROWS == 128 ? quad * 32 + lane : quad * 16 + (lane & 15);
         const int phalf = MROWS == 128 ? 0 : (lane >> 4);
         const bool p1_live = MROWS == 128 ? (quad * 32 < T) : (quad * 16 < T);
-        for (int tl = 0; tl < mt; ++tl) acc_s[tl * kTileRows + vrow] = 0.f;
+        for (int tl = wg; tl < mt; tl += 2) acc_s[tl * kTileRows + vrow] = 0.f;
         uint32_t t1i = 0, t2i = 0;
         for (int s = 0; s <= hpg; ++s) {
             if (s < hpg) {
-                // ---- pass 1 of head s: online row statistics over this CTA's tiles
+                // ---- pass 1 of head s: online row statistics over this warpgroup's tiles
                 float m = -INFINITY, l = 0.f;
-                for (int t = tile_begin; t < tile_end; ++t) {
+                for (int t = tile_begin; t < tile_end; ++t, ++t1i) {
                     const uint32_t tb = t1i & 1;
+                    if ((int)tb != wg) continue;
                     wait_phase(BAR(T1_FULL + tb), (t1i >> 1) & 1, ctl);
                     tc_fence_after();
                     const uint32_t ta = tmem + lane_off + tb * 128u;
-                    // 64 columns at a time: M = 64 -> this thread's half of the row;
-                    // M = 128 -> the row's two halves one after the other
-                    constexpr int NH = MROWS == 128 ? 2 : 1;
+                    // 32 columns at a time: M = 64 -> this thread's half of the row
+                    // (columns 64 * phalf + [0, 64)); M = 128 -> the whole row
+                    constexpr int NH = MROWS == 128 ? 4 : 2;
 #pragma unroll
                     for (int hh = 0; hh < NH; ++hh) {
-                        float v[64];
+                        float v[32];
                         if (p1_live) {
-                            if constexpr (MROWS == 128) {
-                                tmem_ld32(ta + hh * 64, v);
-                                tmem_ld32(ta + hh * 64 + 32, v + 32);
-                            } else {
-                                tmem_ld16x2_32<64>(ta + 0, v);
-                                tmem_ld16x2_32<64>(ta + 32, v + 32);
-                            }
+                            if constexpr (MROWS == 128) tmem_ld32(ta + hh * 32, v);
+                            else tmem_ld16x2_32<64>(ta + hh * 32, v);
                             tmem_wait_ld();
                         }
                         if (hh == NH - 1) {
@@ -331,11 +334,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (lane == 0) mbar_arrive(BAR(T1_EMPTY + tb));
                         }
                         if (p1_live) {
-                            const int valid = N - t * kTileRows - (MROWS == 128 ? hh : phalf) * 64;
-                            row_stats_update<64>(v, valid, cl, m, l);
+                            const int valid = N - t * kTileRows - (MROWS == 128 ? 0 : phalf * 64) - hh * 32;
+                            row_stats_update<32>(v, valid, cl, m, l);
                         }
                     }
-                    ++t1i;
                 }
                 if (MROWS == 64) {
                     // merge the two column halves of each row (threads t and t ^ 16)
@@ -347,14 +349,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                         m = mm;
                     }
                 }
-                // ---- publish (m, l) of head s to the cluster
-                const int slot = s % kStatSlots;
-                if (MROWS == 128 || lane < 16) stats_s[slot * kMaxText + prow] = make_float2(m, l);
-                named_bar_sync(1, 128);
-                if (et == 0) {
-                    fence_acq_rel_cluster();
-                    const uint32_t sb = BAR(STATS + slot);
-                    for (uint32_t r = 0; r < csize; ++r) mbar_arrive_remote(mapa_shared(sb, r));
+                // ---- merge the warpgroups, publish (m, l) of head s to the cluster
+                const bool writer = MROWS == 128 || lane < 16;
+                if (wg == 1 && writer) xs_s[prow] = make_float2(m, l);
+                named_bar_sync(1, 256);
+                if (wg == 0) {
+                    if (writer) {
+                        const float2 o = xs_s[prow];
+                        const float mm = fmaxf(m, o.x);
+                        if (mm != -INFINITY) {
+                            l = (l > 0.f ? l * ex2((m - mm) * cl) : 0.f) + (o.y > 0.f ? o.y * ex2((o.x - mm) * cl) : 0.f);
+                            m = mm;
+                        }
+                        stats_s[(s % kStatSlots) * kMaxText + prow] = make_float2(m, l);
+                    }
+                    named_bar_sync(2, 128);
+                    if (et == 0) {
+                        fence_acq_rel_cluster();
+                        const uint32_t sb = BAR(STATS + s % kStatSlots);
+                        for (uint32_t r = 0; r < csize; ++r) mbar_arrive_remote(mapa_shared(sb, r));
+                    }
                 }
             }
             if (s >= 1) {
@@ -362,39 +376,39 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int hs = s - 1;
                 const int slot = hs % kStatSlots;
                 float* b2 = b2_s + (hs & 1) * kMaxText;
-                wait_phase_cluster(BAR(STATS + slot), (uint32_t)(hs / kStatSlots) & 1u, ctl);
-                if (et < T) {
-                    float bm = merge_cluster_row(base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u, csize, cl);
-                    if (p.extra) bm = log2_add(bm, p.extra[(int64_t)(t0 + et) * p.hq + hg * hpg + hs]);
-                    b2[et] = bm;
-                } else {
-                    b2[et] = INFINITY;
+                if (wg == 0) {
+                    wait_phase_cluster(BAR(STATS + slot), (uint32_t)(hs / kStatSlots) & 1u, ctl);
+                    if (et < T) {
+                        float bm = merge_cluster_row(base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u, csize, cl);
+                        if (p.extra) bm = log2_add(bm, p.extra[(int64_t)(t0 + et) * p.hq + hg * hpg + hs]);
+                        b2[et] = bm;
+                    } else {
+                        b2[et] = INFINITY;
+                    }
                 }
-                named_bar_sync(1, 128);
+                named_bar_sync(1, 256);
                 // ---- pass 2 of head s-1: per-visual-token sums of probabilities
-                for (int t = tile_begin; t < tile_end; ++t) {
+                for (int t = tile_begin; t < tile_end; ++t, ++t2i) {
                     const uint32_t tb = t2i & 1;
+                    if ((int)tb != wg) continue;
                     wait_phase(BAR(T2_FULL + tb), (t2i >> 1) & 1, ctl);
                     tc_fence_after();
                     const uint32_t ta = tmem + lane_off + 256u + tb * 128u;
                     float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
-                    for (int hh = 0; hh < MROWS / 64; ++hh) {
-                        if (hh * 64 < n2) {
-                            float v[64];
-#pragma unroll
-                            for (int k = 0; k < 2; ++k) {
-                                const int c0 = hh * 64 + k * 32;
-                                if (c0 + 32 <= n2) tmem_ld32(ta + c0, v + k * 32);
-                                else if (c0 + 16 <= n2) tmem_ld16(ta + c0, v + k * 32);
-                            }
+                    for (int hh = 0; hh < MROWS / 32; ++hh) {
+                        const int c0 = hh * 32;
+                        if (c0 < n2) {
+                            float v[32];
+                            if (c0 + 32 <= n2) tmem_ld32(ta + c0, v);
+                            else tmem_ld16(ta + c0, v);
                             tmem_wait_ld();
 #pragma unroll
-                            for (int k = 0; k < 4; ++k) {
-                                if (hh * 64 + k * 16 < n2) {
+                            for (int k = 0; k < 2; ++k) {
+                                if (c0 + k * 16 < n2) {
 #pragma unroll
                                     for (int e = 0; e < 16; e += 4) {
-                                        const float4 bb = *reinterpret_cast<const float4*>(b2 + hh * 64 + k * 16 + e);
+                                        const float4 bb = *reinterpret_cast<const float4*>(b2 + c0 + k * 16 + e);
                                         a0 += ex2(fmaf(v[k * 16 + e], cl, -bb.x));
                                         a1 += ex2(fmaf(v[k * 16 + e + 1], cl, -bb.y));
                                         a2 += ex2(fmaf(v[k * 16 + e + 2], cl, -bb.z));
@@ -407,14 +421,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(BAR(T2_EMPTY + tb));
-                    ++t2i;
                     acc_s[(t - tile_begin) * kTileRows + vrow] += (a0 + a1) + (a2 + a3);
                 }
             }
         }
+        named_bar_sync(1, 256);  // every tile's sums are in acc_s
         // ---- results
         const float denom = (float)p.hq * (float)T;
-        for (int tl = 0; tl < mt; ++tl) {
+        for (int tl = wg; tl < mt; tl += 2) {
             const int j = (tile_begin + tl) * kTileRows + vrow;
             if (j < N) {
                 const float a = acc_s[tl * kTileRows + vrow];
@@ -422,7 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
             }
         }
-        if (multi) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 128, 1, fold_flags);
+        if (multi) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 256, 1, fold_flags);
         tc_fence_before();
     }
 
