@@ -774,8 +774,9 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
     if (head_dim > 0 && (!positions || !rope_table || max_positions <= 0))
         return fail(h, LITEVLM_ERR_INVALID_ARG, "positions, rope_table and max_positions are required with RoPE");
     const int bn = lvs::proj_tile_cols(out_features);
+    const int bm = lvs::proj_tile_rows(rows, out_features, h->num_sms);
     CUtensorMap tm_x, tm_w;
-    litevlm_status_t s = encode_rows_map(h, &tm_x, x, hidden, 1, rows, 128, false, "x");
+    litevlm_status_t s = encode_rows_map(h, &tm_x, x, hidden, 1, rows, bm, false, "x");
     if (s != LITEVLM_OK) return s;
     s = encode_rows_map(h, &tm_w, w_folded, hidden, 1, out_features, bn, false, "w_folded");
     if (s != LITEVLM_OK) return s;
@@ -792,7 +793,7 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
     p.y = static_cast<__nv_bfloat16*>(y);
     p.err = h->err_d;
     p.wait_budget = lvs::kWaitBudgetCycles;
-    const cudaError_t e = lvs::launch_proj(tm_x, tm_w, p, (cudaStream_t)stream);
+    const cudaError_t e = lvs::launch_proj(tm_x, tm_w, p, bm, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "project launch");
     return LITEVLM_OK;
 }

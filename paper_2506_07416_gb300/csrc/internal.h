@@ -207,7 +207,9 @@ struct RopeArgs {
     float inv_freq[128];      // rope_base^(-2j / head_dim), rounded to fp32
 };
 int proj_tile_cols(int out_features);
-cudaError_t launch_proj(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const ProjArgs& p, cudaStream_t stream);
+int proj_tile_rows(int64_t rows, int out_features, int num_sms);
+cudaError_t launch_proj(const CUtensorMap& tm_x, const CUtensorMap& tm_w, const ProjArgs& p, int tile_rows,
+                        cudaStream_t stream);
 cudaError_t launch_fold_norm(const __nv_bfloat16* w, const float* gamma, __nv_bfloat16* out, int64_t total,
                              int hidden, int num_sms, cudaStream_t stream);
 cudaError_t launch_rope_table(const RopeArgs& a, int num_sms, cudaStream_t stream);

@@ -61,6 +61,7 @@ def _run(sel, rows, hidden, out_f, head_dim, bias, eps=1e-6, base=1e6, max_pos=4
     (129, 136, 384, 0, False),       # no rotation, 128-column tiles
     (200, 3584, 512, 128, True),     # 4 KV heads x 128 from hidden 3584
     (1, 512, 256, 128, False),       # one row
+    (4900, 128, 4096, 128, True),    # enough tiles for the 256-row variant, ragged last tile
 ])
 def test_project_matches_oracle(sel, rows, hidden, out_f, head_dim, bias):
     _run(sel, rows, hidden, out_f, head_dim, bias)
