@@ -201,6 +201,25 @@ def time_oracle(w, seconds: float, max_runs: int = 1000):
     return value, desc, el, runs
 
 
+def whole_job(local_total_ms: float, tokens_per_rank: int, world: int, device):
+    """The job's time is its slowest rank's: the max of the ranks' timed totals
+    (an all-reduce when world > 1), and the whole-job rate is the tokens of all
+    ranks over that time, in M/s. Returns (time_ms, rate)."""
+    total_ms = local_total_ms
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    return total_ms, tokens_per_rank * world / (total_ms / 1e3) / 1e6
+
+
+def rank_seed(base_seed: int, rank: int) -> int:
+    """Each rank draws its own batch (replicas: the same shapes, other values)."""
+    return base_seed + 1000 * rank
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -260,7 +279,7 @@ def run_ours(args):
     warm = args.warmup if args.warmup is not None else warm_d
     alg = algorithmic(w)
 
-    xd = inputs.make_torch(w, dev, seed=w.seed + 1000 * rank)
+    xd = inputs.make_torch(w, dev, seed=rank_seed(w.seed, rank))
     so_h, to_h = w.seq_offsets(), w.text_offsets()
     kk_h = None if w.keep_k is None else np.asarray(w.keep_k, np.int32)
     kk_d = None if kk_h is None else torch.from_numpy(kk_h).to(dev)
@@ -354,13 +373,7 @@ def run_ours(args):
 
     per_step_ms = np.array([e[0].elapsed_time(e[3]) for e in ev])
     st = np.array([[e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2]), e[2].elapsed_time(e[3])] for e in ev_stage])
-    total_ms = float(per_step_ms.sum())
-    if world > 1:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    tokens_all = w.total_vis * steps * world
-    value = tokens_all / (total_ms / 1e3) / 1e6
+    total_ms, value = whole_job(float(per_step_ms.sum()), w.total_vis * steps, world, dev)
 
     pk = peaks()
     score_us = float(st[:, 0].mean() * 1e3)
