@@ -310,16 +310,21 @@ def run_ours(args):
             raise select.LitevlmError(rc, L.litevlm_select_last_error(h).decode())
 
     def step(q, k, so_d, to_d, hidden_srcs=None):
+        """One step: scores, top-k, gather; returns the kernels it launched."""
         call(L.litevlm_select_score(h, w.batch, q.data_ptr(), to_d.data_ptr(), c_to_h, k.data_ptr(),
                                     so_d.data_ptr(), c_so_h, xd["q_scale"], xd["k_scale"], scores.data_ptr(), sp))
+        n = L.litevlm_select_last_launches(h)
         call(L.litevlm_select_topk(h, w.batch, scores.data_ptr(), so_d.data_ptr(), c_so_h, c_kk_d, c_kk_h, ratio,
                                    kept.data_ptr(), off_d.data_ptr(), off_h.ctypes.data, sp))
+        n += L.litevlm_select_last_launches(h)
         call(L.litevlm_select_compact(h, total_kept, kept.data_ptr(), w.total_vis, n_t,
                                       hidden_srcs if hidden_srcs is not None else c_src, c_dst, c_rb, sp))
+        return n + L.litevlm_select_last_launches(h)
 
     q, k, so_d, to_d = xd["q"], xd["k"], xd["seq_offsets"], xd["text_offsets"]
+    launches_per_step = 0
     for _ in range(warm):
-        step(q, k, so_d, to_d)
+        launches_per_step = step(q, k, so_d, to_d)
     sel.check_device()
 
     # L2: flush between timed steps unless the step's inputs are larger than L2
@@ -331,7 +336,6 @@ def run_ours(args):
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
     ev_stage = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
     plan = sel.score_plan(to_h, so_h)
-    launches_per_step = 3  # score (fold inside), top-k, gather
 
     if world > 1:
         dist.barrier()

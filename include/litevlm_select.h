@@ -111,6 +111,11 @@ litevlm_status_t litevlm_select_destroy(litevlm_select_t handle);
  * failed create in this thread. */
 const char* litevlm_select_last_error(litevlm_select_t handle);
 
+/* Number of kernels the last call on this handle enqueued (0 after an error
+ * or a call with nothing to do); for counting launches (the score call runs
+ * one kernel, two with the full key set). */
+int32_t litevlm_select_last_launches(litevlm_select_t handle);
+
 /* Static description of a status code. */
 const char* litevlm_status_string(litevlm_status_t status);
 
@@ -287,6 +292,7 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t handle, int64_t total_k
                                         int64_t src_rows, int32_t num_tensors,
                                         const void* const* src, void* const* dst, const int64_t* row_bytes,
                                         litevlm_stream_t stream);
+
 
 /*
  * Prefill sequence splice: the shortened LLM input after token selection

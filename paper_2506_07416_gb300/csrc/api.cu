@@ -38,6 +38,7 @@ struct litevlm_select {
     std::vector<int> tiles_desc;  // scratch of the planner for batches above 4096 requests (host)
     lvs::TopkShape topk_shape;    // per-request sizes passed to the top-k kernel by value
     std::string last_error;
+    int32_t last_launches = 0;  // kernels the last call on this handle enqueued
 };
 
 namespace {
@@ -230,6 +231,8 @@ const char* litevlm_select_last_error(litevlm_select_t h)
     return h ? h->last_error.c_str() : g_create_error.c_str();
 }
 
+int32_t litevlm_select_last_launches(litevlm_select_t h) { return h ? h->last_launches : 0; }
+
 litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm_select_t* out)
 {
     g_create_error.clear();
@@ -359,6 +362,7 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, co
 {
     if (!h || !plan) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     ScoreShape sh;
     const litevlm_status_t s = check_score_shape(h, batch, text_offsets_h, seq_offsets_h, &sh);
     if (s != LITEVLM_OK) return s;
@@ -487,6 +491,7 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
             ? lvs::launch_score_resident(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream)
             : lvs::launch_score(tm_q, tm_k, p, plan, batch, row_bytes, fp8, mrows, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "score launch");
+    h->last_launches = ctx ? 2 : 1;
     return LITEVLM_OK;
 }
 }  // namespace
@@ -499,6 +504,7 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     return score_impl(h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h,
                       q_scale, k_scale, scores, nullptr, stream);
 }
@@ -513,19 +519,22 @@ litevlm_status_t litevlm_select_score_full_keys(litevlm_select_t h, int32_t batc
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     const CtxKeys ctx{k_sys, sys_offsets_d, sys_offsets_h, k_text};
     return score_impl(h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h,
                       q_scale, k_scale, scores, &ctx, stream);
 }
 
-litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const float* scores,
-                                     const int32_t* seq_offsets_d, const int32_t* seq_offsets_h,
-                                     const int32_t* keep_k_d, const int32_t* keep_k_h, float keep_ratio,
-                                     int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
-                                     litevlm_stream_t stream)
+namespace {
+// Host half of the top-k: validation from the host mirrors, out_offsets_h, and
+// the per-request sizes the kernels take by value (h->topk_shape). *run is
+// false when there is nothing to launch (batch 0).
+litevlm_status_t topk_prepare(litevlm_select_t h, int32_t batch, const float* scores, const int32_t* seq_offsets_d,
+                              const int32_t* seq_offsets_h, const int32_t* keep_k_d, const int32_t* keep_k_h,
+                              float keep_ratio, int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
+                              int* max_n_out, int64_t* total_k_out, int64_t* tot_n_out, bool* run)
 {
-    if (!h) return LITEVLM_ERR_INVALID_ARG;
-    h->last_error.clear();
+    *run = false;
     if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
     if (batch > h->cfg.max_batch) return fail(h, LITEVLM_ERR_WORKSPACE, "batch exceeds max_batch");
     if ((keep_k_d == nullptr) != (keep_k_h == nullptr))
@@ -569,9 +578,34 @@ litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const fl
         sh.k[b] = off[(size_t)b + 1] - off[(size_t)b];
         sh.out0[b] = off[(size_t)b];
     }
+    *max_n_out = max_n;
+    *total_k_out = total_k;
+    *tot_n_out = tot_n;
+    *run = true;
+    return LITEVLM_OK;
+}
+}  // namespace
+
+litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const float* scores,
+                                     const int32_t* seq_offsets_d, const int32_t* seq_offsets_h,
+                                     const int32_t* keep_k_d, const int32_t* keep_k_h, float keep_ratio,
+                                     int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
+                                     litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    h->last_launches = 0;
+    int max_n = 0;
+    int64_t total_k = 0, tot_n = 0;
+    bool run = false;
+    const litevlm_status_t s = topk_prepare(h, batch, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h,
+                                            keep_ratio, kept_idx, out_offsets_d, out_offsets_h, &max_n, &total_k,
+                                            &tot_n, &run);
+    if (s != LITEVLM_OK || !run) return s;
     const cudaError_t e = lvs::launch_topk(batch, scores, seq_offsets_d, keep_k_d, keep_ratio, kept_idx,
-                                           out_offsets_d, max_n, sh, (cudaStream_t)stream);
+                                           out_offsets_d, max_n, h->topk_shape, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "topk launch");
+    h->last_launches = 1;
     return LITEVLM_OK;
 }
 
@@ -581,6 +615,7 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t h, int64_t total_kept, 
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     if (total_kept < 0 || src_rows < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "sizes must be >= 0");
     if (num_tensors < 1 || num_tensors > lvs::kMaxGatherTensors)
         return fail(h, LITEVLM_ERR_INVALID_ARG, "num_tensors must be in [1, 8]");
@@ -602,6 +637,7 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t h, int64_t total_kept, 
     const cudaError_t e =
         lvs::launch_compact(total_kept, kept_idx, src_rows, g, vec16, h->err_d, h->num_sms, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "compact launch");
+    h->last_launches = 1;
     return LITEVLM_OK;
 }
 
@@ -617,6 +653,7 @@ litevlm_status_t litevlm_select_splice(litevlm_select_t h, int32_t batch, const 
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
     if (batch > h->cfg.max_batch) return fail(h, LITEVLM_ERR_WORKSPACE, "batch exceeds max_batch");
     if (row_bytes <= 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "row_bytes must be > 0");
@@ -665,6 +702,7 @@ litevlm_status_t litevlm_select_splice(litevlm_select_t h, int32_t batch, const 
     a.err = h->err_d;
     const cudaError_t e = lvs::launch_splice(a, max_rows, vec16, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "splice launch");
+    h->last_launches = 1;
     return LITEVLM_OK;
 }
 
@@ -676,6 +714,7 @@ litevlm_status_t litevlm_select_views(litevlm_select_t h, int32_t batch, int32_t
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     if (batch < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
     if (num_views < 1 || num_views > lvs::kMaxViews)
         return fail(h, LITEVLM_ERR_INVALID_ARG, "num_views must be in [1, 64]");
@@ -709,6 +748,7 @@ litevlm_status_t litevlm_select_views(litevlm_select_t h, int32_t batch, int32_t
     a.seq_offsets = seq_offsets;
     cudaError_t e = lvs::launch_views(a, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "views launch");
+    h->last_launches = 1;
     if (seq_offsets_h) {
         e = cudaMemcpyAsync(seq_offsets_h, seq_offsets, sizeof(int32_t) * ((size_t)batch + 1), cudaMemcpyDeviceToHost,
                             (cudaStream_t)stream);
@@ -723,6 +763,7 @@ litevlm_status_t litevlm_select_fold_norm(litevlm_select_t h, int32_t out_featur
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     if (out_features <= 0 || hidden <= 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "sizes must be > 0");
     if (!w || !gamma || !w_folded) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
     const cudaError_t e = lvs::launch_fold_norm(static_cast<const __nv_bfloat16*>(w), gamma,
@@ -730,6 +771,7 @@ litevlm_status_t litevlm_select_fold_norm(litevlm_select_t h, int32_t out_featur
                                                 (int64_t)out_features * hidden, hidden, h->num_sms,
                                                 (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "fold_norm launch");
+    h->last_launches = 1;
     return LITEVLM_OK;
 }
 
@@ -738,6 +780,7 @@ litevlm_status_t litevlm_select_rope_table(litevlm_select_t h, int32_t max_posit
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     if (max_positions <= 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "max_positions must be > 0");
     if (head_dim != 64 && head_dim != 128) return fail(h, LITEVLM_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
     if (!(rope_base > 1.f) || isinf(rope_base)) return fail(h, LITEVLM_ERR_INVALID_ARG, "rope_base must be > 1");
@@ -749,6 +792,7 @@ litevlm_status_t litevlm_select_rope_table(litevlm_select_t h, int32_t max_posit
     for (int j = 0; j < a.half; ++j) a.inv_freq[j] = (float)pow((double)rope_base, -2.0 * j / (double)head_dim);
     const cudaError_t e = lvs::launch_rope_table(a, h->num_sms, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "rope_table launch");
+    h->last_launches = 1;
     return LITEVLM_OK;
 }
 
@@ -759,6 +803,7 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
+    h->last_launches = 0;
     if (rows < 0 || rows > 65535LL * 128) return fail(h, LITEVLM_ERR_INVALID_ARG, "rows must be in [0, 65535 * 128]");
     if (hidden <= 0 || hidden % 8 != 0)
         return fail(h, LITEVLM_ERR_INVALID_ARG, "hidden must be a positive multiple of 8 (16-byte rows)");
@@ -795,6 +840,7 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
     p.wait_budget = lvs::kWaitBudgetCycles;
     const cudaError_t e = lvs::launch_proj(tm_x, tm_w, p, bm, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "project launch");
+    h->last_launches = 1;
     return LITEVLM_OK;
 }
 

@@ -146,6 +146,7 @@ cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, 
                         float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, const TopkShape& shape,
                         cudaStream_t stream);
 
+
 // compact.cu
 constexpr int kMaxGatherTensors = 8;
 struct GatherArgs {

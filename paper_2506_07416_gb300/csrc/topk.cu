@@ -193,100 +193,16 @@ __global__ void __launch_bounds__(kTopkThreads)
 }
 
 
-// ---------------------------------------------------------------------------
-// Register-resident variant for requests of at most kTopkThreads * KPT tokens.
-// Thread t holds the keys of tokens j = e * kTopkThreads + t (e < KPT), so the
-// loads are coalesced and "round e, warp w, lane l" is index order. The radix
-// select starts below the bits that every key of the request shares (one
-// min/max reduction finds them) and stops as soon as the bin holding the k-th
-// key is taken whole. Every warp finds the selected digit from the shared
-// histogram by itself, so a pass costs one barrier; histograms rotate over
-// three buffers so a buffer is cleared two passes after it was last read.
-// Output positions come from per-(round, warp) ballot counts.
-
-template <int KPT>
-__global__ void __launch_bounds__(kTopkThreads)
-    topk_reg_kernel(const float* __restrict__ scores, const int32_t* __restrict__ seq_off,
-                    const int32_t* __restrict__ keep_k, float ratio, int32_t* __restrict__ kept_idx,
-                    int32_t* __restrict__ out_off, const __grid_constant__ TopkShape sh)
+// The k largest keys of one request (0 < k < N), held KPT per thread by one CTA
+// of kTopkThreads threads (token j = e * kTopkThreads + tid), with the request's
+// smallest and largest key lo_k / hi_k. Calls emit(pos, j) once per kept token,
+// pos = its place among the kept tokens in index order (0 .. k-1). hist and cnt
+// are shared memory; hist[0] and hist[1] must be zero on entry.
+template <int KPT, class Emit>
+__device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, int k, uint32_t lo_k, uint32_t hi_k,
+                                            uint32_t (*hist)[256], int (*cnt)[kTopkWarps], Emit emit)
 {
-    __shared__ uint32_t hist[3][256];
-    __shared__ uint32_t wmin[kTopkWarps], wmax[kTopkWarps];
-    __shared__ int cnt[KPT][kTopkWarps];
-    __shared__ long long s_base;
-
-    const int b = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    // sizes in the parameters (read before the wait: they are not produced on
-    // the device), so the scores are the kernel's first global loads
-    const bool by_value = sh.n > 0;
-    int n0 = 0, N = 0, k_v = 0, out0_v = 0;
-    if (by_value) {
-        n0 = sh.n0[b];
-        N = sh.len[b];
-        k_v = sh.k[b];
-        out0_v = sh.out0[b];
-    }
-    griddep_wait();
-    griddep_launch_dependents();
-    if (!by_value) {
-        n0 = seq_off[b];
-        N = seq_off[b + 1] - n0;
-    }
-
-    uint32_t key[KPT];
-#pragma unroll
-    for (int e = 0; e < KPT; ++e) {
-        const int j = e * kTopkThreads + tid;
-        key[e] = j < N ? order_key(__ldcg(scores + n0 + j)) : 0u;
-    }
-
-    // output base = sum of k over earlier requests
-    long long part = 0;
-    if (!by_value)
-        for (int bb = tid; bb < b; bb += kTopkThreads) part += keep_count(seq_off, keep_k, ratio, bb);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
-    if (tid == 0) s_base = by_value ? (long long)out0_v : 0;
-    __syncthreads();
-    if (lane == 0 && part) atomicAdd(reinterpret_cast<unsigned long long*>(&s_base), (unsigned long long)part);
-    const int k = by_value ? k_v : keep_count(seq_off, keep_k, ratio, b);
-
-    // key range of the request (padding slots take part only through valid keys)
-    uint32_t lo_k = 0xFFFFFFFFu, hi_k = 0u;
-#pragma unroll
-    for (int e = 0; e < KPT; ++e) {
-        if (e * kTopkThreads + tid < N) {
-            lo_k = min(lo_k, key[e]);
-            hi_k = max(hi_k, key[e]);
-        }
-    }
-    lo_k = __reduce_min_sync(0xffffffffu, lo_k);
-    hi_k = __reduce_max_sync(0xffffffffu, hi_k);
-    if (lane == 0) {
-        wmin[warp] = lo_k;
-        wmax[warp] = hi_k;
-    }
-    for (int i = tid; i < 2 * 256; i += kTopkThreads) (&hist[0][0])[i] = 0u;
-    __syncthreads();
-    const long long out_base = s_base;
-    if (tid == 0) {
-        out_off[b + 1] = (int32_t)(out_base + k);
-        if (b == 0) out_off[0] = 0;
-    }
-    if (k <= 0 || N <= 0) return;
-    int32_t* dst = kept_idx + out_base;
-    if (k >= N) {
-        for (int j = tid; j < N; j += kTopkThreads) dst[j] = n0 + j;
-        return;
-    }
-    lo_k = wmin[0];
-    hi_k = wmax[0];
-#pragma unroll
-    for (int w = 1; w < kTopkWarps; ++w) {
-        lo_k = min(lo_k, wmin[w]);
-        hi_k = max(hi_k, wmax[w]);
-    }
 
     // ---- radix select below the common high bits
     const uint32_t diff = lo_k ^ hi_k;
@@ -400,9 +316,106 @@ __global__ void __launch_bounds__(kTopkThreads)
         const int before_w = __shfl_sync(0xffffffffu, v, (warp + kTopkWarps - 1) % kTopkWarps);
         const int tot_e = __shfl_sync(0xffffffffu, v, kTopkWarps - 1);
         const uint32_t bal = __ballot_sync(0xffffffffu, (keep >> e) & 1u);
-        if ((keep >> e) & 1u) dst[run + (warp ? before_w : 0) + __popc(bal & lt_mask)] = n0 + e * kTopkThreads + tid;
+        if ((keep >> e) & 1u) emit(run + (warp ? before_w : 0) + __popc(bal & lt_mask), e * kTopkThreads + tid);
         run += tot_e;
     }
+}
+
+// ---------------------------------------------------------------------------
+// Register-resident variant for requests of at most kTopkThreads * KPT tokens.
+// Thread t holds the keys of tokens j = e * kTopkThreads + t (e < KPT), so the
+// loads are coalesced and "round e, warp w, lane l" is index order. The radix
+// select starts below the bits that every key of the request shares (one
+// min/max reduction finds them) and stops as soon as the bin holding the k-th
+// key is taken whole. Every warp finds the selected digit from the shared
+// histogram by itself, so a pass costs one barrier; histograms rotate over
+// three buffers so a buffer is cleared two passes after it was last read.
+// Output positions come from per-(round, warp) ballot counts.
+
+template <int KPT>
+__global__ void __launch_bounds__(kTopkThreads)
+    topk_reg_kernel(const float* __restrict__ scores, const int32_t* __restrict__ seq_off,
+                    const int32_t* __restrict__ keep_k, float ratio, int32_t* __restrict__ kept_idx,
+                    int32_t* __restrict__ out_off, const __grid_constant__ TopkShape sh)
+{
+    __shared__ uint32_t hist[3][256];
+    __shared__ uint32_t wmin[kTopkWarps], wmax[kTopkWarps];
+    __shared__ int cnt[KPT][kTopkWarps];
+    __shared__ long long s_base;
+
+    const int b = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // sizes in the parameters (read before the wait: they are not produced on
+    // the device), so the scores are the kernel's first global loads
+    const bool by_value = sh.n > 0;
+    int n0 = 0, N = 0, k_v = 0, out0_v = 0;
+    if (by_value) {
+        n0 = sh.n0[b];
+        N = sh.len[b];
+        k_v = sh.k[b];
+        out0_v = sh.out0[b];
+    }
+    griddep_wait();
+    griddep_launch_dependents();
+    if (!by_value) {
+        n0 = seq_off[b];
+        N = seq_off[b + 1] - n0;
+    }
+
+    uint32_t key[KPT];
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) {
+        const int j = e * kTopkThreads + tid;
+        key[e] = j < N ? order_key(__ldcg(scores + n0 + j)) : 0u;
+    }
+
+    // output base = sum of k over earlier requests
+    long long part = 0;
+    if (!by_value)
+        for (int bb = tid; bb < b; bb += kTopkThreads) part += keep_count(seq_off, keep_k, ratio, bb);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
+    if (tid == 0) s_base = by_value ? (long long)out0_v : 0;
+    __syncthreads();
+    if (lane == 0 && part) atomicAdd(reinterpret_cast<unsigned long long*>(&s_base), (unsigned long long)part);
+    const int k = by_value ? k_v : keep_count(seq_off, keep_k, ratio, b);
+
+    // key range of the request (padding slots take part only through valid keys)
+    uint32_t lo_k = 0xFFFFFFFFu, hi_k = 0u;
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) {
+        if (e * kTopkThreads + tid < N) {
+            lo_k = min(lo_k, key[e]);
+            hi_k = max(hi_k, key[e]);
+        }
+    }
+    lo_k = __reduce_min_sync(0xffffffffu, lo_k);
+    hi_k = __reduce_max_sync(0xffffffffu, hi_k);
+    if (lane == 0) {
+        wmin[warp] = lo_k;
+        wmax[warp] = hi_k;
+    }
+    for (int i = tid; i < 2 * 256; i += kTopkThreads) (&hist[0][0])[i] = 0u;
+    __syncthreads();
+    const long long out_base = s_base;
+    if (tid == 0) {
+        out_off[b + 1] = (int32_t)(out_base + k);
+        if (b == 0) out_off[0] = 0;
+    }
+    if (k <= 0 || N <= 0) return;
+    int32_t* dst = kept_idx + out_base;
+    if (k >= N) {
+        for (int j = tid; j < N; j += kTopkThreads) dst[j] = n0 + j;
+        return;
+    }
+    lo_k = wmin[0];
+    hi_k = wmax[0];
+#pragma unroll
+    for (int w = 1; w < kTopkWarps; ++w) {
+        lo_k = min(lo_k, wmin[w]);
+        hi_k = max(hi_k, wmax[w]);
+    }
+    select_kept<KPT>(key, N, k, lo_k, hi_k, hist, cnt, [&](int pos, int j) { dst[pos] = n0 + j; });
 }
 
 }  // namespace

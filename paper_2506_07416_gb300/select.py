@@ -47,6 +47,8 @@ def _load():
     lib.litevlm_select_destroy.argtypes = [P]
     lib.litevlm_select_last_error.argtypes = [P]
     lib.litevlm_select_last_error.restype = ctypes.c_char_p
+    lib.litevlm_select_last_launches.argtypes = [P]
+    lib.litevlm_select_last_launches.restype = ctypes.c_int32
     lib.litevlm_status_string.argtypes = [ctypes.c_int]
     lib.litevlm_status_string.restype = ctypes.c_char_p
     lib.litevlm_select_score.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P]
@@ -74,7 +76,8 @@ EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_la
            "litevlm_status_string", "litevlm_select_score", "litevlm_select_topk", "litevlm_select_compact",
            "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc",
            "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views",
-           "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project"]
+           "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project",
+           "litevlm_select_last_launches"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
