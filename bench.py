@@ -38,7 +38,7 @@ UNIT = "M visual tokens/s"
 DEFAULTS = {"single": (3000, 50), "highres": (2000, 30), "fp8_ragged": (200, 10), "sweep": (20, 3)}
 KERNEL_SOURCES = ["paper_2506_07416_gb300/csrc/score_tc.cu", "paper_2506_07416_gb300/csrc/score_res.cu",
                   "paper_2506_07416_gb300/csrc/pipe.cuh", "paper_2506_07416_gb300/csrc/ptx.cuh",
-                  "paper_2506_07416_gb300/csrc/internal.h"]
+                  "paper_2506_07416_gb300/csrc/score.h"]
 
 
 def parse_args():
