@@ -31,7 +31,8 @@
 //
 // Warp roles (320 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
 // MMA issuer, warps 2..9 = epilogue in two warpgroups (TMEM lane quadrant =
-// warp % 4); warpgroup g takes the tiles that land in TMEM buffer g of a pass.
+// warp % 4); the contractions of both passes cycle through four 128-column
+// TMEM buffers and warpgroup g takes every other one.
 // Every wait is bounded (clock budget); on expiry the kernel sets the error
 // word, drains its own copies and MMAs, frees TMEM and returns.
 
@@ -135,8 +136,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const uint32_t bar0 = base + L::OFF_BAR;
     auto BAR = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
-    const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + QBUF, T1_FULL = Q_EMPTY + QBUF,
-              T1_EMPTY = T1_FULL + 2, T2_FULL = T1_EMPTY + 2, T2_EMPTY = T2_FULL + 2, STATS = T2_EMPTY + 2,
+    // U_FULL / U_EMPTY: a ring of four 128-column TMEM buffers shared by the
+    // contractions of both passes, in issue order (unit u uses buffer u % 4)
+    const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + QBUF, U_FULL = Q_EMPTY + QBUF,
+              U_EMPTY = U_FULL + 4, STATS = U_EMPTY + 4,
               DRAIN = STATS + kStatSlots;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
@@ -156,10 +159,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(BAR(Q_EMPTY + i), 1);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(BAR(T1_FULL + i), 1);
-            mbar_init(BAR(T1_EMPTY + i), 4);   // one arrival per warp of the consuming warpgroup
-            mbar_init(BAR(T2_FULL + i), 1);
-            mbar_init(BAR(T2_EMPTY + i), 4);
+            mbar_init(BAR(U_FULL + i), 1);
+            mbar_init(BAR(U_EMPTY + i), 4);   // one arrival per warp of the consuming warpgroup
+            mbar_init(BAR(U_FULL + 2 + i), 1);
+            mbar_init(BAR(U_EMPTY + 2 + i), 4);
         }
         for (int i = 0; i < kStatSlots; ++i) mbar_init(BAR(STATS + i), csize);
         mbar_init(BAR(DRAIN), 1);
@@ -235,7 +238,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (mt > 0) {
                 const uint32_t idesc1 = idesc_make(MROWS, 128, FMT);
                 const uint32_t idesc2 = idesc_make(128, (uint32_t)n2, FMT);
-                uint32_t ks = 0, kph = 0, t1i = 0, t2i = 0;
+                uint32_t ks = 0, kph = 0, ui = 0;
                 bool ok = true;
                 for (int s = 0; s <= hpg && ok; ++s) {
                     for (int pass = 0; pass < 2 && ok; ++pass) {
@@ -250,15 +253,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t qaddr = base + L::OFF_Q + qb * L::Q_BYTES;
                         for (int t = tile_begin; t < tile_end; ++t) {
                             if (!wait_phase(BAR(K_FULL + ks), kph, ctl)) { ok = false; break; }
-                            const uint32_t tb = pass == 0 ? (t1i & 1) : (t2i & 1);
-                            const uint32_t tph = pass == 0 ? ((t1i >> 1) & 1) : ((t2i >> 1) & 1);
-                            if (!wait_phase(BAR((pass == 0 ? T1_EMPTY : T2_EMPTY) + tb), tph ^ 1, ctl)) {
+                            const uint32_t ub = ui & 3, uph = (ui >> 2) & 1;
+                            if (!wait_phase(BAR(U_EMPTY + ub), uph ^ 1, ctl)) {
                                 ok = false;
                                 break;
                             }
                             tc_fence_after();
                             const uint32_t kaddr = base + L::OFF_K + ks * L::TILE_BYTES;
-                            const uint32_t d = tmem + (pass == 0 ? 0u : 256u) + tb * 128u;
+                            const uint32_t d = tmem + ub * 128u;
 #pragma unroll
                             for (int st = 0; st < KSTEPS; ++st) {
                                 const uint32_t koff = (st >> 2) * (kTileRows * 128) + (st & 3) * 32;
@@ -273,9 +275,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     else mma_f16(d, kd, qd, idesc2, st > 0);
                                 }
                             }
-                            mma_commit(BAR((pass == 0 ? T1_FULL : T2_FULL) + tb));
+                            mma_commit(BAR(U_FULL + ub));
                             mma_commit(BAR(K_EMPTY + ks));
-                            if (pass == 0) ++t1i; else ++t2i;
+                            ++ui;
                             if (++ks == kStages) { ks = 0; kph ^= 1; }
                         }
                         if (pass == 1 && ok) mma_commit(BAR(Q_EMPTY + qb));  // last reader of Q(hs)
@@ -291,9 +293,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        // Two warpgroups (warps 2-5 and 6-9). The two TMEM buffers of each pass
-        // alternate from tile to tile; warpgroup g takes the tiles that land in
-        // buffer g, so both work at once. Control flow is identical within a
+        // Two warpgroups (warps 2-5 and 6-9). The contractions of both passes
+        // cycle through four TMEM buffers in issue order; warpgroup g takes the
+        // units u with u % 2 == g (buffers g and g + 2), so each has one buffer
+        // being filled while it reads the other. Control flow is identical within a
         // warpgroup (named barriers); after an abort every wait returns at once
         // and the steps run out.
         const int quad = warp & 3;
@@ -306,17 +309,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int phalf = MROWS == 128 ? 0 : (lane >> 4);
         const bool p1_live = MROWS == 128 ? (quad * 32 < T) : (quad * 16 < T);
         for (int tl = wg; tl < mt; tl += 2) acc_s[tl * kTileRows + vrow] = 0.f;
-        uint32_t t1i = 0, t2i = 0;
+        uint32_t ui = 0;  // contraction units in issue order (both passes)
         for (int s = 0; s <= hpg; ++s) {
             if (s < hpg) {
                 // ---- pass 1 of head s: online row statistics over this warpgroup's tiles
                 float m = -INFINITY, l = 0.f;
-                for (int t = tile_begin; t < tile_end; ++t, ++t1i) {
-                    const uint32_t tb = t1i & 1;
-                    if ((int)tb != wg) continue;
-                    wait_phase(BAR(T1_FULL + tb), (t1i >> 1) & 1, ctl);
+                for (int t = tile_begin; t < tile_end; ++t, ++ui) {
+                    const uint32_t ub = ui & 3;
+                    if ((int)(ui & 1) != wg) continue;
+                    wait_phase(BAR(U_FULL + ub), (ui >> 2) & 1, ctl);
                     tc_fence_after();
-                    const uint32_t ta = tmem + lane_off + tb * 128u;
+                    const uint32_t ta = tmem + lane_off + ub * 128u;
                     // 32 columns at a time: M = 64 -> this thread's half of the row
                     // (columns 64 * phalf + [0, 64)); M = 128 -> the whole row
                     constexpr int NH = MROWS == 128 ? 4 : 2;
@@ -331,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (hh == NH - 1) {
                             tc_fence_before();
                             __syncwarp();
-                            if (lane == 0) mbar_arrive(BAR(T1_EMPTY + tb));
+                            if (lane == 0) mbar_arrive(BAR(U_EMPTY + ub));
                         }
                         if (p1_live) {
                             const int valid = N - t * kTileRows - (MROWS == 128 ? 0 : phalf * 64) - hh * 32;
@@ -388,12 +391,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 named_bar_sync(1, 256);
                 // ---- pass 2 of head s-1: per-visual-token sums of probabilities
-                for (int t = tile_begin; t < tile_end; ++t, ++t2i) {
-                    const uint32_t tb = t2i & 1;
-                    if ((int)tb != wg) continue;
-                    wait_phase(BAR(T2_FULL + tb), (t2i >> 1) & 1, ctl);
+                for (int t = tile_begin; t < tile_end; ++t, ++ui) {
+                    const uint32_t ub = ui & 3;
+                    if ((int)(ui & 1) != wg) continue;
+                    wait_phase(BAR(U_FULL + ub), (ui >> 2) & 1, ctl);
                     tc_fence_after();
-                    const uint32_t ta = tmem + lane_off + 256u + tb * 128u;
+                    const uint32_t ta = tmem + lane_off + ub * 128u;
                     float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
                     for (int hh = 0; hh < MROWS / 32; ++hh) {
@@ -420,7 +423,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(BAR(T2_EMPTY + tb));
+                    if (lane == 0) mbar_arrive(BAR(U_EMPTY + ub));
                     acc_s[(t - tile_begin) * kTileRows + vrow] += (a0 + a1) + (a2 + a3);
                 }
             }
