@@ -27,6 +27,7 @@ struct litevlm_select {
     float* ctx_stats = nullptr; // [max_total_text][Hq]: normaliser terms of system + causal text keys
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     int res_capacity[2][17];  // resident score kernel: CTAs at once per cluster size, by pass-1 rows (64/128); -1 unknown
+    int tc_capacity[2][17];   // the same for the re-read score kernel
     // last score-kernel choices, keyed by a hash of the batch shape (planning walks every plan)
     struct PlanMemo {
         uint64_t key = 0;
@@ -150,7 +151,10 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* se
     const double unit_s = 1.17e-6, hbm_bytes_per_s = 6.8e12;
     const double tile_bytes = (double)lvs::kTileRows * row_bytes;
     double tc_cost = 0.0;
-    ScoreChoice best{false, lvs::plan_score(bt, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, h->num_sms, &tc_cost)};
+    int* tcap = h->tc_capacity[mrows == 64 ? 0 : 1];
+    for (int cl = 1; cl <= lvs::kMaxCluster; ++cl)
+        if (tcap[cl] < 0) tcap[cl] = lvs::tc_cluster_capacity(row_bytes, fp8, mrows, cl);
+    ScoreChoice best{false, lvs::plan_score(bt, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, tcap, &tc_cost)};
     double best_cost = 1.6 * tc_cost;
     const int max_tiles = batch > 0 ? td[0] : 0;
     const int kflags = c.flags & ~LITEVLM_FLAG_QUERY_LAST_TOKEN;
@@ -260,6 +264,8 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
     litevlm_select* h = new (std::nothrow) litevlm_select();
     if (!h) return fail(nullptr, LITEVLM_ERR_CUDA, "out of host memory");
     h->cfg = *c;
+    for (auto& row : h->tc_capacity)
+        for (int& v : row) v = -1;
     for (auto& row : h->res_capacity)
         for (int& v : row) v = -1;
     cudaError_t e = cudaGetDevice(&h->device);
@@ -893,6 +899,7 @@ struct NoAllocDevice {
     int32_t* tickets = nullptr;
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     int res_capacity[3][2][17];  // by kernel family (bf16 d=128, bf16 d=64, e4m3), as in the handle
+    int tc_capacity[3][2][17];
     litevlm_select::PlanMemo plan_memo[3][4];
     int plan_memo_next[3] = {0, 0, 0};
 };
@@ -935,6 +942,9 @@ litevlm_status_t noalloc_setup(int dev, NoAllocDevice& d)
     d.tickets = static_cast<int32_t*>(tp);
     d.encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     for (auto& fam : d.res_capacity)
+        for (auto& row : fam)
+            for (int& v : row) v = -1;
+    for (auto& fam : d.tc_capacity)
         for (auto& row : fam)
             for (int& v : row) v = -1;
     d.ready = true;
@@ -991,7 +1001,10 @@ extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, in
         h.n_counters = (size_t)kNoAllocTickets;
         h.encode = d.encode;
         for (int r = 0; r < 2; ++r)
-            for (int c = 0; c < 17; ++c) h.res_capacity[r][c] = d.res_capacity[fam][r][c];
+            for (int c = 0; c < 17; ++c) {
+                h.res_capacity[r][c] = d.res_capacity[fam][r][c];
+                h.tc_capacity[r][c] = d.tc_capacity[fam][r][c];
+            }
         for (int k = 0; k < 4; ++k) h.plan_memo[k] = d.plan_memo[fam][k];
         h.plan_memo_next = d.plan_memo_next[fam];
     }
@@ -1023,7 +1036,10 @@ extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, in
         std::lock_guard<std::mutex> lock(g_noalloc_mutex);
         NoAllocDevice& d = g_noalloc[dev];
         for (int r = 0; r < 2; ++r)
-            for (int c = 0; c < 17; ++c) d.res_capacity[fam][r][c] = h.res_capacity[r][c];
+            for (int c = 0; c < 17; ++c) {
+                d.res_capacity[fam][r][c] = h.res_capacity[r][c];
+                d.tc_capacity[fam][r][c] = h.tc_capacity[r][c];
+            }
         for (int k = 0; k < 4; ++k) d.plan_memo[fam][k] = h.plan_memo[k];
         d.plan_memo_next[fam] = h.plan_memo_next;
     }

@@ -98,7 +98,10 @@ double makespan(const BatchTiles& bt, int g, int slots, const Cost& cost)
     return mx;
 }
 
-ScorePlan plan_score(const BatchTiles& bt, int hq, int hkv, int tile_bytes, int num_sms, double* cost_out);
+// cap_by_cluster[c]: CTAs of the re-read kernel resident at once with clusters of c (<= 0: unusable)
+ScorePlan plan_score(const BatchTiles& bt, int hq, int hkv, int tile_bytes, const int* cap_by_cluster,
+                     double* cost_out);
+int tc_cluster_capacity(int row_bytes, bool fp8, int mrows, int cluster);
 cudaError_t launch_score(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
                          const ScorePlan& plan, int batch, int row_bytes, bool fp8, int mrows, cudaStream_t stream);
 bool score_shape_supported(int head_dim, bool fp8);

@@ -453,17 +453,50 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int ROW_BYTES, bool FP8, int MROWS>
+cudaError_t tc_prepare(int cluster)
+{
+    auto kern = score_tc_kernel<ROW_BYTES, FP8, MROWS>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         SmemLayout<ROW_BYTES, MROWS>::ALLOC);
+    if (e == cudaSuccess && cluster > 8) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return e;
+}
+
+// CTAs resident at once with clusters of `cluster` CTAs (occupancy query)
+template <int ROW_BYTES, bool FP8, int MROWS>
+int tc_capacity(int cluster)
+{
+    if (tc_prepare<ROW_BYTES, FP8, MROWS>(cluster) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cluster * 64, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = SmemLayout<ROW_BYTES, MROWS>::ALLOC;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, score_tc_kernel<ROW_BYTES, FP8, MROWS>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return n * cluster;
+}
+
+template <int ROW_BYTES, bool FP8, int MROWS>
 cudaError_t launch_variant(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p,
                            const ScorePlan& plan, int batch, cudaStream_t stream)
 {
     auto kern = score_tc_kernel<ROW_BYTES, FP8, MROWS>;
     const int smem = SmemLayout<ROW_BYTES, MROWS>::ALLOC;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = tc_prepare<ROW_BYTES, FP8, MROWS>(plan.cluster);
     if (e != cudaSuccess) return e;
-    if (plan.cluster > 8) {
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-        if (e != cudaSuccess) return e;
-    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(plan.cluster * plan.groups * batch), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
@@ -482,6 +515,14 @@ cudaError_t launch_variant(const CUtensorMap& tm_q, const CUtensorMap& tm_k, con
 
 }  // namespace
 
+int tc_cluster_capacity(int row_bytes, bool fp8, int mrows, int cluster)
+{
+    if (fp8) return mrows == 64 ? tc_capacity<128, true, 64>(cluster) : tc_capacity<128, true, 128>(cluster);
+    if (row_bytes == 256)
+        return mrows == 64 ? tc_capacity<256, false, 64>(cluster) : tc_capacity<256, false, 128>(cluster);
+    return mrows == 64 ? tc_capacity<128, false, 64>(cluster) : tc_capacity<128, false, 128>(cluster);
+}
+
 bool score_shape_supported(int head_dim, bool fp8)
 {
     if (fp8) return head_dim == 128;
@@ -490,18 +531,8 @@ bool score_shape_supported(int head_dim, bool fp8)
 
 // CTAs of one cluster size that run at once with one CTA per SM (GPC packing
 // on a 152-SM GB300: 1, 2 -> 152; 4 -> 144; 8 -> 120; 16 -> 112).
-static int cluster_capacity(int c, int num_sms)
-{
-    switch (c) {
-    case 1:
-    case 2: return num_sms;
-    case 4: return num_sms * 144 / 152;
-    case 8: return num_sms * 120 / 152;
-    default: return num_sms * 112 / 152;
-    }
-}
-
-ScorePlan plan_score(const BatchTiles& bt, int hq, int hkv, int tile_bytes, int num_sms, double* cost_out)
+ScorePlan plan_score(const BatchTiles& bt, int hq, int hkv, int tile_bytes, const int* cap_by_cluster,
+                     double* cost_out)
 {
     ScorePlan best{1, 1, 1};
     double best_cost = 1e300;
@@ -512,11 +543,12 @@ ScorePlan plan_score(const BatchTiles& bt, int hq, int hkv, int tile_bytes, int 
     }
     const int G = hq / hkv;
     for (int pass = 0; pass < 2 && best_cost >= 1e299; ++pass) {
-        for (int c = 1; c <= kMaxCluster; c *= 2) {
+        for (int c = 1; c <= kMaxCluster; ++c) {
             const int tpc = (max_tiles + c - 1) / c;
             if (tpc > kMaxTilesPerCta) continue;
-            if (c > 1 && (c / 2) >= max_tiles) break;  // idle ranks only
-            const int cap = cluster_capacity(c, num_sms);
+            if (c > 1 && (c - 1) * tpc >= max_tiles) continue;  // an idle rank on the largest request
+            const int cap = cap_by_cluster[c];
+            if (cap < c) continue;
             for (int g = 1; g <= hq; ++g) {
                 if (hq % g) continue;
                 const long long ctas = (long long)bt.n * c * g;
