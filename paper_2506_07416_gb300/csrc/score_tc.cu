@@ -22,7 +22,9 @@
 //           into TMEM; one epilogue thread per visual token adds
 //           sum_i 2^(s_ij * c - b_hi) to its running score.
 // Software pipeline with one head of look-ahead: pass 1 of head s+1 runs while
-// the statistics of head s travel across the cluster, then pass 2 of head s.
+// the statistics of head s travel across the cluster, then pass 2 of head s
+// (a CTA that is its own cluster has nothing to wait for and runs the two
+// passes of each head back to back).
 // The K tiles stream through a TMA ring for both passes (the pass-2 re-read of
 // a CTA's few tiles is normally served by L2). Scores are summed over the heads
 // of the group in shared memory; with one head group they are final, with
@@ -133,6 +135,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int G = p.hq / p.hkv;
     const int hpg = p.heads_per_group;
     const float cl = p.c_log2;
+    // Pass 2 of a head follows pass 1 of the next head (lag 1), so the
+    // statistics exchange of the cluster overlaps a contraction; a CTA without
+    // peers needs no exchange and runs both passes of a head in turn (lag 0),
+    // which halves the K tiles that must stay in L2 for the re-read.
+    const int lag = csize > 1 ? 1 : 0;
 
     const uint32_t bar0 = base + L::OFF_BAR;
     auto BAR = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
@@ -207,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (++ks == kStages) { ks = 0; kph ^= 1; }
                 }
             };
-            for (int s = 0; s <= hpg && ok; ++s) {
+            for (int s = 0; s < hpg + lag && ok; ++s) {
                 if (s < hpg) {
                     const int h = hg * hpg + s;
                     const int qb = s % QBUF;
@@ -220,7 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ++q_issued[qb];
                     load_tiles(h / G);
                 }
-                if (s >= 1 && ok) load_tiles((hg * hpg + s - 1) / G);
+                if (s >= lag && ok) load_tiles((hg * hpg + s - lag) / G);
             }
             // drain: the last load of every slot lands before the CTA leaves
             // (these waits ignore the abort flag)
@@ -240,11 +247,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t idesc2 = idesc_make(128, (uint32_t)n2, FMT);
                 uint32_t ks = 0, kph = 0, ui = 0;
                 bool ok = true;
-                for (int s = 0; s <= hpg && ok; ++s) {
+                for (int s = 0; s < hpg + lag && ok; ++s) {
                     for (int pass = 0; pass < 2 && ok; ++pass) {
                         if (pass == 0 && s >= hpg) continue;
-                        if (pass == 1 && s < 1) continue;
-                        const int hs = pass == 0 ? s : s - 1;  // head of this unit
+                        if (pass == 1 && s < lag) continue;
+                        const int hs = pass == 0 ? s : s - lag;  // head of this unit
                         const int qb = hs % QBUF;
                         if (pass == 0) {
                             if (!wait_phase(BAR(Q_FULL + qb), (hs / QBUF) & 1, ctl)) { ok = false; break; }
@@ -310,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool p1_live = MROWS == 128 ? (quad * 32 < T) : (quad * 16 < T);
         for (int tl = wg; tl < mt; tl += 2) acc_s[tl * kTileRows + vrow] = 0.f;
         uint32_t ui = 0;  // contraction units in issue order (both passes)
-        for (int s = 0; s <= hpg; ++s) {
+        for (int s = 0; s < hpg + lag; ++s) {
             if (s < hpg) {
                 // ---- pass 1 of head s: online row statistics over this warpgroup's tiles
                 float m = -INFINITY, l = 0.f;
@@ -374,9 +381,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
-            if (s >= 1) {
+            if (s >= lag) {
                 // ---- merge the cluster's statistics of head s-1
-                const int hs = s - 1;
+                const int hs = s - lag;
                 const int slot = hs % kStatSlots;
                 float* b2 = b2_s + (hs & 1) * kMaxText;
                 if (wg == 0) {
