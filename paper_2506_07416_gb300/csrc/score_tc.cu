@@ -31,10 +31,10 @@
 // several the CTAs write partial rows and the last CTA of the request to finish
 // (atomic ticket) adds them in a fixed order.
 //
-// Warp roles (320 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
-// MMA issuer, warps 2..9 = epilogue in two warpgroups (TMEM lane quadrant =
+// Warp roles (448 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
+// MMA issuer, warps 2..13 = epilogue in three warpgroups (TMEM lane quadrant =
 // warp % 4); the contractions of both passes cycle through four 128-column
-// TMEM buffers and warpgroup g takes every other one.
+// TMEM buffers and warpgroup g takes units u with u % 3 == g.
 // Every wait is bounded (clock budget); on expiry the kernel sets the error
 // word, drains its own copies and MMAs, frees TMEM and returns.
 
@@ -48,7 +48,9 @@ namespace lvs {
 
 namespace {
 
-constexpr int kThreads = 320;
+constexpr int kEpiWG = 3;                    // epilogue warpgroups
+constexpr int kEpiThreads = 128 * kEpiWG;
+constexpr int kThreads = 64 + kEpiThreads;
 constexpr int kStatSlots = 4;  // stats of heads s-3..s may be live across the cluster
 
 // Shared-memory plan. The ring gets whatever is left of the 227 KB after the
@@ -64,7 +66,8 @@ struct SmemLayout {
     // Q(s+2) load while pass 2 of head s is still reading Q(s).
     static constexpr int QBUF = MROWS == 64 ? 3 : 2;
     static constexpr int FIXED = QBUF * Q_BYTES + kMaxTilesPerCta * kTileRows * 4 + kStatSlots * kMaxText * 8 +
-                                 2 * kMaxText * 4 + kMaxText * 8 + kMaxTilesPerCta * 4 + 512 + 64 + 1024;
+                                 2 * kMaxText * 4 + (kEpiWG - 1) * kMaxText * 8 + kMaxTilesPerCta * 4 + 512 + 64 +
+                                 1024;
     static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
     static constexpr int kStages = STAGES_FIT > 10 ? 10 : STAGES_FIT;
     static constexpr int OFF_K = 0;
@@ -72,8 +75,8 @@ struct SmemLayout {
     static constexpr int OFF_ACC = OFF_Q + QBUF * Q_BYTES;
     static constexpr int OFF_STATS = OFF_ACC + kMaxTilesPerCta * kTileRows * 4;
     static constexpr int OFF_B2 = OFF_STATS + kStatSlots * kMaxText * 8;
-    static constexpr int OFF_XS = OFF_B2 + 2 * kMaxText * 4;      // [128] float2: warpgroup 1's row statistics
-    static constexpr int OFF_FLAGS = OFF_XS + kMaxText * 8;       // [32] int, fold flags
+    static constexpr int OFF_XS = OFF_B2 + 2 * kMaxText * 4;  // [kEpiWG - 1][128] float2: other warpgroups' row stats
+    static constexpr int OFF_FLAGS = OFF_XS + (kEpiWG - 1) * kMaxText * 8;  // [32] int, fold flags
     static constexpr int OFF_BAR = OFF_FLAGS + kMaxTilesPerCta * 4;
     // k_full[S], k_empty[S], q_full[QBUF], q_empty[QBUF], t1_full[2], t1_empty[2],
     // t2_full[2], t2_empty[2], stats[4], drain
@@ -300,14 +303,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        // Two warpgroups (warps 2-5 and 6-9). The contractions of both passes
-        // cycle through four TMEM buffers in issue order; warpgroup g takes the
-        // units u with u % 2 == g (buffers g and g + 2), so each has one buffer
-        // being filled while it reads the other. Control flow is identical within a
+        // Three warpgroups (warps 2-5, 6-9, 10-13). The contractions of both
+        // passes cycle through four TMEM buffers in issue order; warpgroup g
+        // takes the units u with u % 3 == g, in order, so while one warpgroup
+        // reads a buffer the others' units are being filled. A unit's buffer
+        // was last used by unit u - 4, which belongs to another warpgroup and
+        // comes earlier in that warpgroup's order, so no wait is circular. Control flow is identical within a
         // warpgroup (named barriers); after an abort every wait returns at once
         // and the steps run out.
         const int quad = warp & 3;
-        const int wg = (warp - 2) >> 2;                       // 0 or 1
+        const int wg = (warp - 2) >> 2;                       // 0 .. kEpiWG - 1
         const int et = threadIdx.x - 64;                      // 0..255
         const int vrow = quad * 32 + lane;                    // pass 2: TMEM lane = visual token in tile
         const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
@@ -315,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int prow = MROWS == 128 ? quad * 32 + lane : quad * 16 + (lane & 15);
         const int phalf = MROWS == 128 ? 0 : (lane >> 4);
         const bool p1_live = MROWS == 128 ? (quad * 32 < T) : (quad * 16 < T);
-        for (int tl = wg; tl < mt; tl += 2) acc_s[tl * kTileRows + vrow] = 0.f;
+        for (int tl = wg; tl < mt; tl += kEpiWG) acc_s[tl * kTileRows + vrow] = 0.f;
         uint32_t ui = 0;  // contraction units in issue order (both passes)
         for (int s = 0; s < hpg + lag; ++s) {
             if (s < hpg) {
@@ -323,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 float m = -INFINITY, l = 0.f;
                 for (int t = tile_begin; t < tile_end; ++t, ++ui) {
                     const uint32_t ub = ui & 3;
-                    if ((int)(ui & 1) != wg) continue;
+                    if ((int)(ui % kEpiWG) != wg) continue;
                     wait_phase(BAR(U_FULL + ub), (ui >> 2) & 1, ctl);
                     tc_fence_after();
                     const uint32_t ta = tmem + lane_off + ub * 128u;
@@ -361,15 +366,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 // ---- merge the warpgroups, publish (m, l) of head s to the cluster
                 const bool writer = MROWS == 128 || lane < 16;
-                if (wg == 1 && writer) xs_s[prow] = make_float2(m, l);
-                named_bar_sync(1, 256);
+                if (wg > 0 && writer) xs_s[(wg - 1) * kMaxText + prow] = make_float2(m, l);
+                named_bar_sync(1, kEpiThreads);
                 if (wg == 0) {
                     if (writer) {
-                        const float2 o = xs_s[prow];
-                        const float mm = fmaxf(m, o.x);
-                        if (mm != -INFINITY) {
-                            l = (l > 0.f ? l * ex2((m - mm) * cl) : 0.f) + (o.y > 0.f ? o.y * ex2((o.x - mm) * cl) : 0.f);
-                            m = mm;
+#pragma unroll
+                        for (int o_wg = 1; o_wg < kEpiWG; ++o_wg) {  // fixed order: deterministic
+                            const float2 o = xs_s[(o_wg - 1) * kMaxText + prow];
+                            const float mm = fmaxf(m, o.x);
+                            if (mm != -INFINITY) {
+                                l = (l > 0.f ? l * ex2((m - mm) * cl) : 0.f) +
+                                    (o.y > 0.f ? o.y * ex2((o.x - mm) * cl) : 0.f);
+                                m = mm;
+                            }
                         }
                         stats_s[(s % kStatSlots) * kMaxText + prow] = make_float2(m, l);
                     }
@@ -396,11 +405,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         b2[et] = INFINITY;
                     }
                 }
-                named_bar_sync(1, 256);
+                named_bar_sync(1, kEpiThreads);
                 // ---- pass 2 of head s-1: per-visual-token sums of probabilities
                 for (int t = tile_begin; t < tile_end; ++t, ++ui) {
                     const uint32_t ub = ui & 3;
-                    if ((int)(ui & 1) != wg) continue;
+                    if ((int)(ui % kEpiWG) != wg) continue;
                     wait_phase(BAR(U_FULL + ub), (ui >> 2) & 1, ctl);
                     tc_fence_after();
                     const uint32_t ta = tmem + lane_off + ub * 128u;
@@ -435,10 +444,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-        named_bar_sync(1, 256);  // every tile's sums are in acc_s
+        named_bar_sync(1, kEpiThreads);  // every tile's sums are in acc_s
         // ---- results
         const float denom = (float)p.hq * (float)T;
-        for (int tl = wg; tl < mt; tl += 2) {
+        for (int tl = wg; tl < mt; tl += kEpiWG) {
             const int j = (tile_begin + tl) * kTileRows + vrow;
             if (j < N) {
                 const float a = acc_s[tl * kTileRows + vrow];
@@ -446,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
             }
         }
-        if (multi) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 256, 1, fold_flags);
+        if (multi) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, kEpiThreads, 1, fold_flags);
         tc_fence_before();
     }
 
