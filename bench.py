@@ -55,6 +55,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="bounded CPU work for the oracle baseline")
     ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--measure-fp8-peak", action="store_true",
+                    help="time a cuBLASLt e4m3 GEMM (torch._scaled_mm) and print its TFLOP/s, nothing else")
     return ap.parse_args()
 
 
@@ -679,8 +681,36 @@ def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept):
                    "into one of two device buffers on a copy stream, kept indices + offsets copied back"}
 
 
+def measure_fp8_peak(n: int = 8192, reps: int = 50):
+    """Dense e4m3 x e4m3 -> bf16 GEMM throughput of the library GEMM (cuBLASLt
+    through torch._scaled_mm), n x n x n, the e4m3 counterpart of the measured
+    bf16 peak. Inputs far larger than L2 are not needed for a compute-bound GEMM."""
+    import torch
+    dev = torch.device("cuda")
+    g = torch.Generator(device=dev).manual_seed(0)
+    a = torch.randn((n, n), generator=g, device=dev).to(torch.float8_e4m3fn)
+    b = torch.randn((n, n), generator=g, device=dev).to(torch.float8_e4m3fn).t()  # column-major operand
+    one = torch.ones((), device=dev)
+    for _ in range(5):
+        torch._scaled_mm(a, b, scale_a=one, scale_b=one, out_dtype=torch.bfloat16)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        torch._scaled_mm(a, b, scale_a=one, scale_b=one, out_dtype=torch.bfloat16)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    tf = 2.0 * n ** 3 / (ms * 1e-3) / 1e12
+    print(json.dumps({"fp8_e4m3_tflops": tf, "n": n, "ms_per_gemm": ms, "library": "cuBLASLt via torch._scaled_mm",
+                      "bf16_tflops_measured": peaks()["bf16_tflops"]}), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
+    if args.measure_fp8_peak:
+        return measure_fp8_peak()
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)
