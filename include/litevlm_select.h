@@ -295,6 +295,26 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t handle, int64_t total_k
 
 
 /*
+ * Scores and top-k in one call: the outputs of litevlm_select_score (scores)
+ * followed by litevlm_select_topk on them, with the arguments of those two
+ * calls. When the score launch splits the heads of a request over several
+ * CTAs, the top-k kernel adds the head-group partial rows itself (in the same
+ * order as the score kernel would, so the scores are bit-identical) instead of
+ * the score kernel's ticketed fold, which shortens the critical path of small
+ * batches. It does so when batch <= 256, N_b <= 8192 and head groups x the
+ * largest N_b <= 32768 (the partial values one top-k CTA reads); otherwise it
+ * runs the two calls unchanged.
+ */
+litevlm_status_t litevlm_select_score_topk(litevlm_select_t handle, int32_t batch,
+                                           const void* q_text, const int32_t* text_offsets_d,
+                                           const int32_t* text_offsets_h, const void* k_vis,
+                                           const int32_t* seq_offsets_d, const int32_t* seq_offsets_h,
+                                           float q_scale, float k_scale, float* scores,
+                                           const int32_t* keep_k_d, const int32_t* keep_k_h, float keep_ratio,
+                                           int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
+                                           litevlm_stream_t stream);
+
+/*
  * Prefill sequence splice: the shortened LLM input after token selection
  * (Design section: the LLM prefills only the kept visual tokens with the
  * prompt). Request b's output rows are its S_b system rows, then its k_b kept

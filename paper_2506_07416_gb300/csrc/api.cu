@@ -395,8 +395,10 @@ struct CtxKeys {
 litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_text, const int32_t* text_offsets_d,
                             const int32_t* text_offsets_h, const void* k_vis, const int32_t* seq_offsets_d,
                             const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
-                            const CtxKeys* ctx, litevlm_stream_t stream)
+                            const CtxKeys* ctx, litevlm_stream_t stream, bool allow_defer = false,
+                            int* deferred_groups = nullptr)
 {
+    if (deferred_groups) *deferred_groups = 0;
     const litevlm_select_config_t& c = h->cfg;
     const bool fp8 = c.qk_dtype == LITEVLM_FP8_E4M3;
     ScoreShape sh;
@@ -455,6 +457,11 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
     p.slot_cols = (max_t + 15) & ~15;
     p.query_last = (c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
     p.extra = nullptr;
+    // the top-k CTA of a request reads groups x N_b partial values: worth it
+    // for small requests (it saves the score kernel's ticketed fold), not for
+    // long ones with many groups
+    p.defer_fold = allow_defer && plan.groups > 1 && (int64_t)plan.groups * sh.max_n <= 32768;
+    if (p.defer_fold && deferred_groups) *deferred_groups = plan.groups;
     if (ctx) {
         lvs::CtxArgs ca{};
         ca.q = static_cast<const uint8_t*>(q_text);
@@ -578,6 +585,8 @@ litevlm_status_t topk_prepare(litevlm_select_t h, int32_t batch, const float* sc
         for (int32_t b = 0; b <= batch; ++b) out_offsets_h[b] = off[(size_t)b];
     lvs::TopkShape& sh = h->topk_shape;
     sh.n = batch <= lvs::kTopkShapeMax ? batch : 0;
+    sh.partials = nullptr;
+    sh.groups = 0;
     for (int32_t b = 0; b < sh.n; ++b) {
         sh.n0[b] = seq_offsets_h[b];
         sh.len[b] = seq_offsets_h[b + 1] - seq_offsets_h[b];
@@ -608,10 +617,54 @@ litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const fl
                                             keep_ratio, kept_idx, out_offsets_d, out_offsets_h, &max_n, &total_k,
                                             &tot_n, &run);
     if (s != LITEVLM_OK || !run) return s;
-    const cudaError_t e = lvs::launch_topk(batch, scores, seq_offsets_d, keep_k_d, keep_ratio, kept_idx,
-                                           out_offsets_d, max_n, h->topk_shape, (cudaStream_t)stream);
+    // scores are only read (no deferred fold here)
+    const cudaError_t e = lvs::launch_topk(batch, const_cast<float*>(scores), seq_offsets_d, keep_k_d, keep_ratio,
+                                           kept_idx, out_offsets_d, max_n, h->topk_shape, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "topk launch");
     h->last_launches = 1;
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_score_topk(litevlm_select_t h, int32_t batch, const void* q_text,
+                                           const int32_t* text_offsets_d, const int32_t* text_offsets_h,
+                                           const void* k_vis, const int32_t* seq_offsets_d,
+                                           const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
+                                           const int32_t* keep_k_d, const int32_t* keep_k_h, float keep_ratio,
+                                           int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
+                                           litevlm_stream_t stream)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    h->last_launches = 0;
+    int max_n = 0;
+    int64_t total_k = 0, tot_n = 0;
+    bool run = false;
+    litevlm_status_t s = topk_prepare(h, batch, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h,
+                                      keep_ratio, kept_idx, out_offsets_d, out_offsets_h, &max_n, &total_k, &tot_n,
+                                      &run);
+    if (s != LITEVLM_OK) return s;
+    // the top-k kernel can take over the head-group fold when it holds the
+    // request's keys in registers and has the sizes by value
+    const bool can_defer = h->topk_shape.n == batch && max_n <= 16 * 512;
+    int groups = 0;
+    s = score_impl(h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h, q_scale,
+                   k_scale, scores, nullptr, stream, can_defer, &groups);
+    if (s != LITEVLM_OK || !run) return s;
+    lvs::TopkShape& sh = h->topk_shape;
+    if (groups > 0) {
+        const bool last_only = (h->cfg.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
+        sh.partials = h->partials;
+        sh.groups = groups;
+        sh.total_vis = tot_n;
+        for (int32_t b = 0; b < batch; ++b) {
+            const int t = text_offsets_h[b + 1] - text_offsets_h[b];
+            sh.denom[b] = (float)h->cfg.num_q_heads * (float)(last_only && t > 0 ? 1 : t);
+        }
+    }
+    const cudaError_t e = lvs::launch_topk(batch, scores, seq_offsets_d, keep_k_d, keep_ratio, kept_idx,
+                                           out_offsets_d, max_n, sh, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "topk launch");
+    h->last_launches = 2;
     return LITEVLM_OK;
 }
 

@@ -41,8 +41,15 @@ struct TopkShape {
     int32_t len[kTopkShapeMax];     // N_b
     int32_t k[kTopkShapeMax];       // k_b
     int32_t out0[kTopkShapeMax];    // sum of k over earlier requests
+    // Deferred fold (partials != null): the scores are the sum over `groups`
+    // partial rows (stride total_vis, added in group order) divided by denom[b];
+    // the kernel writes them to `scores` and selects on them.
+    const float* partials;
+    int32_t groups;
+    int64_t total_vis;
+    float denom[kTopkShapeMax];
 };
-cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,
+cudaError_t launch_topk(int batch, float* scores, const int32_t* seq_off, const int32_t* keep_k,
                         float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, const TopkShape& shape,
                         cudaStream_t stream);
 

@@ -30,6 +30,7 @@ struct ScoreLaunch {
     int32_t slot_cols;        // resident kernel: TMEM columns per slot (T rounded up to 16, max over batch)
     int32_t res_nb;           // resident kernel: TMEM head buffers, 1 or 2 (2: heads overlap)
     int32_t query_last;       // 1: only the last text token of each request is a query
+    int32_t defer_fold;       // 1 (with groups > 1): leave the group partials; the top-k kernel adds them
     float c_log2;             // q_scale * k_scale / sqrt(d) * log2(e)
     long long wait_budget;
     // [sum T][Hq] normaliser terms of the system and causal text keys (unit of

@@ -455,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
             }
         }
-        if (multi) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, kEpiThreads, 1, fold_flags);
+        if (multi && !p.defer_fold) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, kEpiThreads, 1, fold_flags);
         tc_fence_before();
     }
 

@@ -332,9 +332,9 @@ __device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, i
 // three buffers so a buffer is cleared two passes after it was last read.
 // Output positions come from per-(round, warp) ballot counts.
 
-template <int KPT>
+template <int KPT, bool DEFER>
 __global__ void __launch_bounds__(kTopkThreads)
-    topk_reg_kernel(const float* __restrict__ scores, const int32_t* __restrict__ seq_off,
+    topk_reg_kernel(float* __restrict__ scores, const int32_t* __restrict__ seq_off,
                     const int32_t* __restrict__ keep_k, float ratio, int32_t* __restrict__ kept_idx,
                     int32_t* __restrict__ out_off, const __grid_constant__ TopkShape sh)
 {
@@ -363,10 +363,43 @@ __global__ void __launch_bounds__(kTopkThreads)
     }
 
     uint32_t key[KPT];
+    if constexpr (DEFER) {  // launched only with the sizes by value and the partials
+        // the score kernel's last step: the head-group partials, added in group
+        // order and divided once, as its own fold would
+        const float den = sh.denom[b];
+        float sum[KPT];
 #pragma unroll
-    for (int e = 0; e < KPT; ++e) {
-        const int j = e * kTopkThreads + tid;
-        key[e] = j < N ? order_key(__ldcg(scores + n0 + j)) : 0u;
+        for (int e = 0; e < KPT; ++e) sum[e] = 0.f;
+        constexpr int QG = KPT <= 4 ? 8 : (KPT <= 8 ? 4 : 2);  // loads in flight per key, within the registers
+        for (int g0 = 0; g0 < sh.groups; g0 += QG) {
+            float v[KPT][QG];
+#pragma unroll
+            for (int e = 0; e < KPT; ++e) {
+                const int j = e * kTopkThreads + tid;
+#pragma unroll
+                for (int q = 0; q < QG; ++q)
+                    v[e][q] = (j < N && g0 + q < sh.groups)
+                                  ? __ldcg(sh.partials + (int64_t)(g0 + q) * sh.total_vis + n0 + j) : 0.f;
+            }
+#pragma unroll
+            for (int e = 0; e < KPT; ++e)
+#pragma unroll
+                for (int q = 0; q < QG; ++q)
+                    if (g0 + q < sh.groups) sum[e] += v[e][q];
+        }
+#pragma unroll
+        for (int e = 0; e < KPT; ++e) {
+            const int j = e * kTopkThreads + tid;
+            const float sc = sum[e] / den;
+            if (j < N) scores[n0 + j] = sc;
+            key[e] = j < N ? order_key(sc) : 0u;
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < KPT; ++e) {
+            const int j = e * kTopkThreads + tid;
+            key[e] = j < N ? order_key(__ldcg(scores + n0 + j)) : 0u;
+        }
     }
 
     // output base = sum of k over earlier requests
@@ -437,17 +470,22 @@ cudaError_t launch_pdl(void (*kern)(Args...), unsigned grid, unsigned block, siz
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
-cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, const int32_t* keep_k,
+cudaError_t launch_topk(int batch, float* scores, const int32_t* seq_off, const int32_t* keep_k,
                         float keep_ratio, int32_t* kept_idx, int32_t* out_off, int max_n, const TopkShape& shape,
                         cudaStream_t stream)
 {
     if (batch <= 0) return cudaSuccess;
     // requests up to 16 keys per thread: registers only
     if (max_n <= 16 * kTopkThreads) {
-        auto kern = max_n <= 2 * kTopkThreads   ? topk_reg_kernel<2>
-                    : max_n <= 4 * kTopkThreads ? topk_reg_kernel<4>
-                    : max_n <= 8 * kTopkThreads ? topk_reg_kernel<8>
-                                                : topk_reg_kernel<16>;
+        const bool defer = shape.partials != nullptr && shape.n == batch;
+        auto kern = defer ? (max_n <= 2 * kTopkThreads   ? topk_reg_kernel<2, true>
+                             : max_n <= 4 * kTopkThreads ? topk_reg_kernel<4, true>
+                             : max_n <= 8 * kTopkThreads ? topk_reg_kernel<8, true>
+                                                         : topk_reg_kernel<16, true>)
+                          : (max_n <= 2 * kTopkThreads   ? topk_reg_kernel<2, false>
+                             : max_n <= 4 * kTopkThreads ? topk_reg_kernel<4, false>
+                             : max_n <= 8 * kTopkThreads ? topk_reg_kernel<8, false>
+                                                         : topk_reg_kernel<16, false>);
         return launch_pdl(kern, (unsigned)batch, kTopkThreads, 0, stream, scores, seq_off, keep_k, keep_ratio,
                           kept_idx, out_off, shape);
     }
@@ -455,8 +493,8 @@ cudaError_t launch_topk(int batch, const float* scores, const int32_t* seq_off, 
     const size_t smem = (size_t)keys * 4;
     cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(topk_kernel, (unsigned)batch, kTopkThreads, smem, stream, scores, seq_off, keep_k, keep_ratio,
-                      kept_idx, out_off, keys);
+    return launch_pdl(topk_kernel, (unsigned)batch, kTopkThreads, smem, stream, (const float*)scores, seq_off, keep_k,
+                      keep_ratio, kept_idx, out_off, keys);
 }
 
 }  // namespace lvs

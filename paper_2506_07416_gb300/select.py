@@ -59,12 +59,13 @@ def _load():
     lib.litevlm_select_project.argtypes = [P, i64, i32, i32, P, P, P, f32, i32, P, P, i32, P, P]
     lib.litevlm_select_topk.argtypes = [P, i32, P, P, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
+    lib.litevlm_select_score_topk.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
     lib.litevlm_select_score_plan.argtypes = [P, i32, P, P, P]
     lib.litevlm_select_splice.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, P, P, i64, P, P, P, P, P]
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
     for fn in ("create", "destroy", "score", "score_full_keys", "topk", "compact", "check_device", "score_plan",
-               "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project"):
+               "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project", "score_topk"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -77,7 +78,7 @@ EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_la
            "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc",
            "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views",
            "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project",
-           "litevlm_select_last_launches"]
+           "litevlm_select_last_launches", "litevlm_select_score_topk"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -168,6 +169,16 @@ def views(handle: int, batch: int, num_views: int, lexical, logits, tokens_per_v
     _check(LIB.litevlm_select_views(handle, batch, num_views, _ptr(lexical), _ptr(logits), _ptr(tpv), w_lex, w_logit,
                                     threshold, min_views, _ptr(view_mask), _ptr(view_offsets), _ptr(selected_views),
                                     _ptr(seq_offsets), _ptr(seq_offsets_h), _stream_ptr(stream)), handle)
+
+
+def score_topk(handle: int, batch: int, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h,
+               q_scale: float, k_scale: float, scores, keep_k_d, keep_k_h, keep_ratio: float, kept_idx,
+               out_offsets_d, out_offsets_h, stream=None) -> None:
+    to_h, so_h, kk_h = _host_i32(text_offsets_h), _host_i32(seq_offsets_h), _host_i32(keep_k_h)
+    _check(LIB.litevlm_select_score_topk(handle, batch, _ptr(q_text), _ptr(text_offsets_d), _ptr(to_h),
+                                         _ptr(k_vis), _ptr(seq_offsets_d), _ptr(so_h), q_scale, k_scale,
+                                         _ptr(scores), _ptr(keep_k_d), _ptr(kk_h), keep_ratio, _ptr(kept_idx),
+                                         _ptr(out_offsets_d), _ptr(out_offsets_h), _stream_ptr(stream)), handle)
 
 
 def fold_norm(handle: int, out_features: int, hidden: int, w, gamma, w_folded, stream=None) -> None:
@@ -305,6 +316,32 @@ class Selector:
         views(self.handle, batch, nv, lexical, logits, tokens_per_view, w_lex, w_logit, threshold, min_views, mask,
               vo, sv, so, so_h, stream)
         return mask[:batch], vo, sv, so, so_h
+
+    def score_topk(self, q, text_offsets, k, seq_offsets, q_scale=1.0, k_scale=1.0, keep_k=None,
+                   keep_ratio: float = 0.0, text_offsets_h=None, seq_offsets_h=None, stream=None):
+        """Scores and top-k in one call. Returns (scores, kept_idx, out_offsets
+        device, out_offsets host numpy)."""
+        import torch
+        so_h = _host_i32(seq_offsets if seq_offsets_h is None else seq_offsets_h)
+        to_h = _host_i32(text_offsets if text_offsets_h is None else text_offsets_h)
+        batch = len(so_h) - 1
+        kk_h = _host_i32(keep_k)
+        kk_d = None
+        if kk_h is not None:
+            kk_d = keep_k if isinstance(keep_k, torch.Tensor) and keep_k.is_cuda else \
+                torch.from_numpy(kk_h).to(k.device)
+            total = int(kk_h.sum())
+        else:
+            r = float(np.float32(keep_ratio))
+            total = int(sum(min(n, max(0, int(np.floor(r * n)))) for n in np.diff(so_h)))
+        scores = torch.empty(max(1, int(so_h[-1])), dtype=torch.float32, device=k.device)
+        kept = torch.empty(max(total, 1), dtype=torch.int32, device=k.device)
+        off_d = torch.empty(batch + 1, dtype=torch.int32, device=k.device)
+        off_h = np.zeros(batch + 1, np.int32)
+        score_topk(self.handle, batch, q, text_offsets, to_h, k, seq_offsets, so_h, q_scale, k_scale, scores, kk_d,
+                   kk_h, keep_ratio, kept, off_d, off_h, stream)
+        self._keep_alive = kk_d
+        return scores[:int(so_h[-1])], kept[:int(off_h[-1])], off_d, off_h
 
     def fold_norm(self, w, gamma, stream=None):
         """bf16 W * gamma (per input column) for project()."""
