@@ -554,7 +554,7 @@ def run_project(w, xd, sel, dev, stream, steps, pk):
     y = torch.empty((rows, O), dtype=torch.bfloat16, device=dev)
     L = select.LIB
     args = (sel.handle, rows, H, O, x.data_ptr(), wf.data_ptr(), None, 1e-6, d, pos.data_ptr(), table.data_ptr(),
-            rows + 64, y.data_ptr(), stream.cuda_stream)
+            rows + 64, 0.0, y.data_ptr(), stream.cuda_stream)
     n = max(3, min(steps, 50))
     res = {}
     def ours():

@@ -228,10 +228,16 @@ litevlm_status_t litevlm_select_views(litevlm_select_t handle, int32_t batch, in
  * j pairs with j + head_dim/2, (y1, y2) -> (y1 cos - y2 sin, y2 cos + y1 sin)
  * with (cos, sin) = table[positions[r]][j]. One tcgen05 contraction per
  * 128 x 256 (or 128) output tile; the row scale, bias and rotation are applied
- * to the fp32 accumulator, which is rounded once to bf16.
+ * to the fp32 accumulator, which is rounded once: to bf16, or, when
+ * out_scale > 0, to the e4m3 code of y / out_scale (round to nearest even,
+ * saturating to +-448: a static per-tensor scale as FP8 post-training
+ * quantisation calibrates it; the e4m3 score path takes out_scale as q_scale /
+ * k_scale).
  *   rows             0 .. 65535 * 128 token rows; hidden a multiple of 8; out_features a multiple of 128
- *   x                device bf16 [rows, hidden];  y device bf16 [rows, out_features]
- *                    (= [rows, heads, head_dim], the layout litevlm_select_score reads)
+ *   x                device bf16 [rows, hidden];  y device [rows, out_features] bf16, or
+ *                    e4m3 codes when out_scale > 0 (= [rows, heads, head_dim], the layout
+ *                    litevlm_select_score reads)
+ *   out_scale        0: bf16 output; > 0 (finite): e4m3 output of y / out_scale
  *   bias             device float [out_features] or NULL
  *   eps              >= 0
  *   head_dim         0 (no rotation), 64 or 128
@@ -250,7 +256,8 @@ litevlm_status_t litevlm_select_project(litevlm_select_t handle, int64_t rows, i
                                         int32_t out_features, const void* x, const void* w_folded,
                                         const float* bias, float eps, int32_t head_dim,
                                         const int32_t* positions, const float* rope_table,
-                                        int32_t max_positions, void* y, litevlm_stream_t stream);
+                                        int32_t max_positions, float out_scale, void* y,
+                                        litevlm_stream_t stream);
 
 /*
  * Per-request top-k (Results section, ratio r of visual tokens kept; Table 1).

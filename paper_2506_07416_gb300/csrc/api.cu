@@ -858,7 +858,7 @@ litevlm_status_t litevlm_select_rope_table(litevlm_select_t h, int32_t max_posit
 litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_t hidden, int32_t out_features,
                                         const void* x, const void* w_folded, const float* bias, float eps,
                                         int32_t head_dim, const int32_t* positions, const float* rope_table,
-                                        int32_t max_positions, void* y, litevlm_stream_t stream)
+                                        int32_t max_positions, float out_scale, void* y, litevlm_stream_t stream)
 {
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
@@ -871,6 +871,8 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
     if (head_dim != 0 && head_dim != 64 && head_dim != 128)
         return fail(h, LITEVLM_ERR_UNSUPPORTED, "head_dim must be 0 (no rotation), 64 or 128");
     if (!(eps >= 0.f) || isinf(eps)) return fail(h, LITEVLM_ERR_INVALID_ARG, "eps must be finite and >= 0");
+    if (!(out_scale >= 0.f) || isinf(out_scale))
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "out_scale must be 0 (bf16 output) or finite and > 0 (e4m3)");
     if (rows == 0) return LITEVLM_OK;
     if (!x || !w_folded || !y) return fail(h, LITEVLM_ERR_INVALID_ARG, "a device pointer is NULL");
     if (!aligned16(x) || !aligned16(w_folded) || !aligned16(y))
@@ -894,7 +896,9 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
     p.bias = bias;
     p.positions = positions;
     p.rope = reinterpret_cast<const float2*>(rope_table);
-    p.y = static_cast<__nv_bfloat16*>(y);
+    p.y = out_scale > 0.f ? nullptr : static_cast<__nv_bfloat16*>(y);
+    p.y8 = out_scale > 0.f ? static_cast<uint8_t*>(y) : nullptr;
+    p.out_inv_scale = out_scale > 0.f ? 1.f / out_scale : 0.f;
     p.err = h->err_d;
     p.wait_budget = lvs::kWaitBudgetCycles;
     const cudaError_t e = lvs::launch_proj(tm_x, tm_w, p, bm, (cudaStream_t)stream);

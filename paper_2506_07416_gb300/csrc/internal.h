@@ -105,7 +105,9 @@ struct ProjArgs {
     const float* bias;        // [O] or null
     const int32_t* positions; // [rows] (head_dim > 0)
     const float2* rope;       // [max_positions][head_dim / 2] (cos, sin)
-    __nv_bfloat16* y;         // [rows, O]
+    __nv_bfloat16* y;         // [rows, O] bf16 output, or
+    uint8_t* y8;              // [rows, O] e4m3 codes of y * out_inv_scale (null: bf16 output)
+    float out_inv_scale;
     int32_t* err;
     long long wait_budget;
 };

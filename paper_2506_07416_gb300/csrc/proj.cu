@@ -23,6 +23,8 @@
 
 #include <math.h>
 
+#include <cuda_fp8.h>
+
 #include "internal.h"
 #include "pipe.cuh"
 #include "ptx.cuh"
@@ -58,7 +60,36 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-// scale, bias, rotation and bf16 store of columns [c_begin, c_end) of one
+// two e4m3 codes (round to nearest even, saturating to +-448)
+__device__ __forceinline__ uint32_t pack_e4m3(float lo, float hi)
+{
+    return (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(lo, hi), __NV_SATFINITE, __NV_E4M3);
+}
+
+// 32 consecutive outputs of one row from 16 value pairs: bf16 (64 bytes), or
+// e4m3 codes of y / scale (32 bytes) when the call asked for e4m3
+__device__ __forceinline__ void store_pairs(const ProjArgs& p, int64_t elem, const float2 (&y)[16])
+{
+    if (p.y8) {
+        uint32_t o[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            o[q] = pack_e4m3(y[2 * q].x * p.out_inv_scale, y[2 * q].y * p.out_inv_scale) |
+                   (pack_e4m3(y[2 * q + 1].x * p.out_inv_scale, y[2 * q + 1].y * p.out_inv_scale) << 16);
+        uint4* d = reinterpret_cast<uint4*>(p.y8 + elem);
+        d[0] = make_uint4(o[0], o[1], o[2], o[3]);
+        d[1] = make_uint4(o[4], o[5], o[6], o[7]);
+    } else {
+        uint32_t o[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) o[q] = pack_bf16(y[q].x, y[q].y);
+        uint4* d = reinterpret_cast<uint4*>(p.y + elem);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) d[q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+    }
+}
+
+// scale, bias, rotation and store (bf16 or e4m3) of columns [c_begin, c_end) of one
 // accumulator row (this thread's); the range holds whole heads
 __device__ __forceinline__ void proj_store_row(const ProjArgs& p, uint32_t ta, int64_t grow, int n0, int c_begin,
                                                int c_end, bool live, float sc)
@@ -71,7 +102,7 @@ __device__ __forceinline__ void proj_store_row(const ProjArgs& p, uint32_t ta, i
             pos = 0;
         }
     }
-    __nv_bfloat16* yrow = p.y + grow * (int64_t)p.out_features + n0;
+    const int64_t row0 = grow * (int64_t)p.out_features + n0;  // element index of this tile's first column
     if (p.head_dim > 0) {
         const int half = p.head_dim / 2;
         const float2* cs_row = p.rope + (int64_t)pos * half;
@@ -82,29 +113,24 @@ __device__ __forceinline__ void proj_store_row(const ProjArgs& p, uint32_t ta, i
                 tmem_ld32(ta + (uint32_t)(h0 + half + c), v2);
                 tmem_wait_ld();
                 if (live) {
-                    uint32_t o1[16], o2[16];
+                    float2 a[16], b[16];
 #pragma unroll
-                    for (int j = 0; j < 32; j += 2) {
-                        float a[2], b[2];
-#pragma unroll
-                        for (int e = 0; e < 2; ++e) {
-                            const int col1 = n0 + h0 + c + j + e;
-                            const float y1 = fmaf(v1[j + e], sc, p.bias ? p.bias[col1] : 0.f);
-                            const float y2 = fmaf(v2[j + e], sc, p.bias ? p.bias[col1 + half] : 0.f);
-                            const float2 cs = cs_row[c + j + e];
-                            a[e] = y1 * cs.x - y2 * cs.y;
-                            b[e] = y2 * cs.x + y1 * cs.y;
+                    for (int j = 0; j < 32; ++j) {
+                        const int col1 = n0 + h0 + c + j;
+                        const float y1 = fmaf(v1[j], sc, p.bias ? p.bias[col1] : 0.f);
+                        const float y2 = fmaf(v2[j], sc, p.bias ? p.bias[col1 + half] : 0.f);
+                        const float2 cs = cs_row[c + j];
+                        const float r1 = y1 * cs.x - y2 * cs.y, r2 = y2 * cs.x + y1 * cs.y;
+                        if (j & 1) {
+                            a[j / 2].y = r1;
+                            b[j / 2].y = r2;
+                        } else {
+                            a[j / 2].x = r1;
+                            b[j / 2].x = r2;
                         }
-                        o1[j / 2] = pack_bf16(a[0], a[1]);
-                        o2[j / 2] = pack_bf16(b[0], b[1]);
                     }
-                    uint4* d1 = reinterpret_cast<uint4*>(yrow + h0 + c);
-                    uint4* d2 = reinterpret_cast<uint4*>(yrow + h0 + half + c);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        d1[q] = make_uint4(o1[4 * q], o1[4 * q + 1], o1[4 * q + 2], o1[4 * q + 3]);
-                        d2[q] = make_uint4(o2[4 * q], o2[4 * q + 1], o2[4 * q + 2], o2[4 * q + 3]);
-                    }
+                    store_pairs(p, row0 + h0 + c, a);
+                    store_pairs(p, row0 + h0 + half + c, b);
                 }
             }
         }
@@ -114,14 +140,12 @@ __device__ __forceinline__ void proj_store_row(const ProjArgs& p, uint32_t ta, i
             tmem_ld32(ta + (uint32_t)c, v);
             tmem_wait_ld();
             if (live) {
-                uint32_t o[16];
+                float2 o[16];
 #pragma unroll
                 for (int j = 0; j < 32; j += 2)
-                    o[j / 2] = pack_bf16(fmaf(v[j], sc, p.bias ? p.bias[n0 + c + j] : 0.f),
-                                         fmaf(v[j + 1], sc, p.bias ? p.bias[n0 + c + j + 1] : 0.f));
-                uint4* d = reinterpret_cast<uint4*>(yrow + c);
-#pragma unroll
-                for (int q = 0; q < 4; ++q) d[q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                    o[j / 2] = make_float2(fmaf(v[j], sc, p.bias ? p.bias[n0 + c + j] : 0.f),
+                                           fmaf(v[j + 1], sc, p.bias ? p.bias[n0 + c + j + 1] : 0.f));
+                store_pairs(p, row0 + c, o);
             }
         }
     }

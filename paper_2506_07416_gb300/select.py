@@ -56,7 +56,7 @@ def _load():
     lib.litevlm_select_views.argtypes = [P, i32, i32, P, P, P, f32, f32, f32, i32, P, P, P, P, P, P]
     lib.litevlm_select_fold_norm.argtypes = [P, i32, i32, P, P, P, P]
     lib.litevlm_select_rope_table.argtypes = [P, i32, i32, f32, P, P]
-    lib.litevlm_select_project.argtypes = [P, i64, i32, i32, P, P, P, f32, i32, P, P, i32, P, P]
+    lib.litevlm_select_project.argtypes = [P, i64, i32, i32, P, P, P, f32, i32, P, P, i32, f32, P, P]
     lib.litevlm_select_topk.argtypes = [P, i32, P, P, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_score_topk.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P, P, f32, P, P, P, P]
@@ -192,9 +192,9 @@ def rope_table(handle: int, max_positions: int, head_dim: int, rope_base: float,
 
 
 def project(handle: int, rows: int, hidden: int, out_features: int, x, w_folded, bias, eps: float, head_dim: int,
-            positions, table, max_positions: int, y, stream=None) -> None:
+            positions, table, max_positions: int, y, stream=None, out_scale: float = 0.0) -> None:
     _check(LIB.litevlm_select_project(handle, rows, hidden, out_features, _ptr(x), _ptr(w_folded), _ptr(bias), eps,
-                                      head_dim, _ptr(positions), _ptr(table), max_positions, _ptr(y),
+                                      head_dim, _ptr(positions), _ptr(table), max_positions, out_scale, _ptr(y),
                                       _stream_ptr(stream)), handle)
 
 
@@ -357,15 +357,17 @@ class Selector:
         return t
 
     def project(self, x, w_folded, bias=None, eps: float = 1e-6, head_dim: int = 0, positions=None, table=None,
-                out=None, stream=None):
-        """y = RoPE(RMS-scale(x) . w_folded^T + bias), bf16 [rows, out_features]."""
+                out=None, stream=None, out_scale: float = 0.0):
+        """y = RoPE(RMS-scale(x) . w_folded^T + bias): bf16 [rows, out_features],
+        or uint8 e4m3 codes of y / out_scale when out_scale > 0."""
         import torch
         rows, hidden = x.shape
         out_f = w_folded.shape[0]
         if out is None:
-            out = torch.empty((rows, out_f), dtype=torch.bfloat16, device=x.device)
+            out = torch.empty((rows, out_f), dtype=torch.uint8 if out_scale > 0 else torch.bfloat16,
+                              device=x.device)
         project(self.handle, rows, hidden, out_f, x, w_folded, bias, eps, head_dim, positions, table,
-                0 if table is None else table.shape[0], out, stream)
+                0 if table is None else table.shape[0], out, stream, out_scale)
         return out
 
     def topk(self, scores, seq_offsets, keep_k=None, keep_ratio: float = 0.0, seq_offsets_h=None, kept_idx=None,

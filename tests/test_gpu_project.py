@@ -129,3 +129,66 @@ def test_projection_feeds_the_scores(sel):
     o = oracle.score(qo.reshape(T, hq, d), ko.reshape(N, hq, d), so, to, hq, hq, d, "bf16")
     assert_scores_close(sc, o, "e4m3")
     s.close()
+
+
+def _e4m3_decode(codes_u8, scale):
+    return torch.from_numpy(codes_u8).view(torch.float8_e4m3fn).float().numpy().astype(np.float64) * scale
+
+
+def test_project_e4m3_output(sel):
+    """e4m3 output under a static per-tensor scale: the codes decode to the
+    oracle's y within the e4m3 rounding (at most 1/16 relative for normal
+    values) plus a small absolute term for the subnormal range; with a scale
+    too small, values saturate at +-448 * scale instead of overflowing."""
+    rows, H, O, d = 300, 1024, 512, 128
+    x, g, w, b, pos = inputs.projection_numpy(rows, H, O, seed=13, bias=True, max_position=2048)
+    wf = sel.fold_norm(_bf16_dev(w), torch.from_numpy(g).cuda())
+    table = sel.rope_table(2048, d, 1e6)
+    oy = oracle.project(x, g, 1e-6, w, b, d, pos, 1e6)
+    scale = float(np.abs(oy).max()) / 448.0
+    y8 = sel.project(_bf16_dev(x), wf, torch.from_numpy(b).cuda(), 1e-6, d, torch.from_numpy(pos).cuda(), table,
+                     out_scale=scale)
+    sel.check_device()
+    assert y8.dtype == torch.uint8
+    gy = _e4m3_decode(y8.cpu().numpy(), scale)
+    rms = float(np.sqrt(np.mean(oy * oy)))
+    bad = np.abs(gy - oy) > 0.0625 * np.abs(oy) + 0.02 * rms
+    assert not bad.any(), int(bad.sum())
+    small = scale / 8
+    y8 = sel.project(_bf16_dev(x), wf, torch.from_numpy(b).cuda(), 1e-6, d, torch.from_numpy(pos).cuda(), table,
+                     out_scale=small)
+    gs = _e4m3_decode(y8.cpu().numpy(), small)
+    assert np.all(np.isfinite(gs)) and np.abs(gs).max() <= 448 * small * (1 + 1e-6)
+    big = np.abs(oy) > 448 * small * 1.1
+    assert np.all(np.abs(gs[big]) == 448 * small)
+
+
+def test_e4m3_projection_feeds_the_e4m3_scores(sel):
+    """x -> e4m3 q, k (static scales) -> the e4m3 score kernel, against the
+    oracle chain (fp64 projection, the same scales, torch's e4m3 rounding, the
+    e4m3 score oracle); the two codes may differ by one e4m3 rounding, so the
+    scores agree to the e4m3 tolerance."""
+    from gpu_util import assert_scores_close
+    from paper_2506_07416_gb300 import select
+    H, hq, d, N, T = 512, 8, 128, 700, 40
+    xv, g, wk, _, _ = inputs.projection_numpy(N, H, hq * d, seed=21)
+    xt, _, wq, _, _ = inputs.projection_numpy(T, H, hq * d, seed=22)
+    pos_v = (16 + np.arange(N)).astype(np.int32)
+    pos_t = (16 + N + np.arange(T)).astype(np.int32)
+    ko = oracle.project(xv, g, 1e-6, wk, None, d, pos_v, 1e6)
+    qo = oracle.project(xt, g, 1e-6, wq, None, d, pos_t, 1e6)
+    ks, qs = float(np.abs(ko).max()) / 448.0, float(np.abs(qo).max()) / 448.0
+    table = sel.rope_table(2048, d, 1e6)
+    gk = sel.project(_bf16_dev(xv), sel.fold_norm(_bf16_dev(wk), torch.from_numpy(g).cuda()), None, 1e-6, d,
+                     torch.from_numpy(pos_v).cuda(), table, out_scale=ks)
+    gq = sel.project(_bf16_dev(xt), sel.fold_norm(_bf16_dev(wq), torch.from_numpy(g).cuda()), None, 1e-6, d,
+                     torch.from_numpy(pos_t).cuda(), table, out_scale=qs)
+    so, to = np.array([0, N], np.int32), np.array([0, T], np.int32)
+    s = select.Selector(1, N, T, hq, hq, d, "e4m3")
+    sc = s.score(gq.view(T, hq, d), torch.from_numpy(to).cuda(), gk.view(N, hq, d), torch.from_numpy(so).cuda(),
+                 q_scale=qs, k_scale=ks, seq_offsets_h=so, text_offsets_h=to).cpu().numpy()
+    s.check_device()
+    enc = lambda a, sc_: torch.from_numpy((a / sc_).astype(np.float32)).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    o = oracle.score(enc(qo, qs).reshape(T, hq, d), enc(ko, ks).reshape(N, hq, d), so, to, hq, hq, d, "e4m3", qs, ks)
+    assert_scores_close(sc, o, "e4m3")
+    s.close()
