@@ -125,7 +125,13 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const int b = p.order_n > 0 ? (int)p.order[req_i] : req_i;
     const int hg = item - req_i * p.groups;
 
-    griddep_wait();
+    // With the full-key-set terms (p.extra, written by the kernel launched just
+    // before this one) only the threads that read them wait for that kernel,
+    // right before the read: this kernel's other inputs come from kernels that
+    // had completed before that one passed its own wait, so the visual-key work
+    // overlaps it. Every CTA still waits before it exits, so this grid never
+    // completes ahead of that one.
+    if (!p.extra) griddep_wait();
     griddep_launch_dependents();
     // The request's offsets are loaded here and first used after the setup
     // below (barriers, TMEM, cluster barrier), so their latency overlaps it.
@@ -201,6 +207,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                            (tpc > 0 && (tpc - 1) * p.slot_cols + span > buf_cols) ||
                            tpc > (nb == 2 ? kBufSlots : kResMaxSlots) || (int)csize * p.slot_cols > L::RECV_COLS;
     if (bad_shape || N <= 0) {
+        if (p.extra) griddep_wait();
         if (bad_shape && threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
         tc_fence_before();
         __syncthreads();
@@ -480,7 +487,10 @@ __global__ void __launch_bounds__(kResThreads, 1)
                         if (v2.y > 0.f) Ls += v2.y * ex2((v2.x - M) * cl);
                     }
                     float b = fmaf(M, cl, __log2f(Ls));
-                    if (p.extra) b = log2_add(b, p.extra[(int64_t)(t0 + col) * p.hq + hg * hpg + s]);
+                    if (p.extra) {
+                        griddep_wait();
+                        b = log2_add(b, p.extra[(int64_t)(t0 + col) * p.hq + hg * hpg + s]);
+                    }
                     float mloc = smax[wt];  // this CTA's column max: the e values' reference
 #pragma unroll
                     for (int q = 1; q < 4; ++q) mloc = fmaxf(mloc, smax[q * 64 + wt]);
@@ -574,6 +584,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         tc_fence_after();
         tmem_dealloc(tmem, kResTmemCols);
     }
+    if (p.extra) griddep_wait();  // returns at once for threads that already waited
     cluster_sync_all();
 }
 

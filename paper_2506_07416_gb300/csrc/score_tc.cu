@@ -114,7 +114,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int b = p.order_n > 0 ? (int)p.order[req_i] : req_i;
     const int hg = item - req_i * p.groups;
 
-    griddep_wait();
+    // With the full-key-set terms (p.extra, written by the kernel launched just
+    // before this one) only the threads that read them wait for that kernel,
+    // right before the read: this kernel's other inputs come from kernels that
+    // had completed before that one passed its own wait, so the visual-key work
+    // overlaps it. Every CTA still waits before it exits, so this grid never
+    // completes ahead of that one.
+    if (!p.extra) griddep_wait();
     griddep_launch_dependents();
     const int n0 = p.seq_off[b];
     const int N = p.seq_off[b + 1] - n0;
@@ -124,11 +130,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool multi = p.groups > 1;
     // Uniform for the whole cluster (same request). With several head groups
     // every CTA must still take its fold ticket, so only shape errors return.
-    if (T > MROWS || (N > 0 && T <= 0)) {
-        if (threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
+    if (T > MROWS || (N > 0 && T <= 0) || N <= 0) {
+        if (p.extra) griddep_wait();
+        if (N > 0 && threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
         return;
     }
-    if (N <= 0) return;
     const int n_tiles = (N + kTileRows - 1) / kTileRows;
     const int tpc = (n_tiles + (int)csize - 1) / (int)csize;
     const int tile_begin = min(n_tiles, (int)rank * tpc);
@@ -399,7 +405,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     wait_phase_cluster(BAR(STATS + slot), (uint32_t)(hs / kStatSlots) & 1u, ctl);
                     if (et < T) {
                         float bm = merge_cluster_row(base + L::OFF_STATS + (uint32_t)(slot * kMaxText + et) * 8u, csize, cl);
-                        if (p.extra) bm = log2_add(bm, p.extra[(int64_t)(t0 + et) * p.hq + hg * hpg + hs]);
+                        if (p.extra) {
+                            griddep_wait();
+                            bm = log2_add(bm, p.extra[(int64_t)(t0 + et) * p.hq + hg * hpg + hs]);
+                        }
                         b2[et] = bm;
                     } else {
                         b2[et] = INFINITY;
@@ -465,6 +474,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         tmem_dealloc(tmem, 512);
     }
+    if (p.extra) griddep_wait();  // returns at once for threads that already waited
     cluster_sync_all();  // peers are done reading this CTA's statistics
 }
 
