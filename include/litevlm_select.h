@@ -32,8 +32,9 @@
  *     a call returns after enqueueing. Host-side validation happens before any
  *     work is enqueued; on error nothing is enqueued.
  *   - The *_h offset arrays must hold the same values as their *_d mirrors;
- *     they are read on the host for validation and sizing only. Mirrors that
- *     disagree are undefined behaviour.
+ *     they are read on the host for validation and sizing, and for small
+ *     batches the kernels take them by value (launch parameters) instead of
+ *     loading the device arrays. Mirrors that disagree are undefined behaviour.
  *   - Every function returns a status and never aborts the process. The text
  *     of the last error of a handle is available from litevlm_select_last_error.
  *   - A handle is used by one host thread and one stream at a time.

@@ -482,6 +482,14 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
         if (ce != cudaSuccess) return cuda_fail(h, ce, "context-key statistics launch");
         p.extra = h->ctx_stats;
     }
+    p.nv = 0;
+    if (batch <= lvs::kOffsetsByValue) {
+        for (int32_t b = 0; b <= batch; ++b) {
+            p.so_v[b] = seq_offsets_h[b];
+            p.to_v[b] = text_offsets_h[b];
+        }
+        p.nv = batch;
+    }
     // clusters are launched largest request first (stable: ties keep index order)
     p.order_n = 0;
     if (batch > 1 && batch <= lvs::kOrderMax) {

@@ -47,9 +47,6 @@ __device__ __forceinline__ void cp_async_wait_all()
     asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
-// generic-proxy shared-memory writes -> visible to the tensor core (async proxy)
-__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-
 // Byte offset of 16-byte piece u of row r in a K-major tile of `rows` rows
 // stored as 128-byte swizzled blocks along d ([ROW_BYTES / 128][rows][128 B],
 // 8-row groups of 1024 bytes, piece c of row r at c ^ (r % 8)).
@@ -155,7 +152,7 @@ __global__ void __launch_bounds__(kCtxThreads) ctx_stats_kernel(const CtxArgs a)
             cp_async16(sB + sw128_offset(r, u, kCtxKeys), src, bytes);
         }
         cp_async_wait_all();
-        fence_proxy_async_smem();
+        fence_proxy_async_shared();  // the copies' writes -> visible to the tensor core
         __syncthreads();
         if (threadIdx.x == 0) {
             tc_fence_after();

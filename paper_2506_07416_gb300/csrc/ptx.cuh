@@ -43,6 +43,13 @@ __device__ __forceinline__ void fence_mbar_init_cluster()
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
 
+// orders this thread's earlier shared-memory writes (generic proxy) before its
+// later bulk-copy operations (async proxy)
+__device__ __forceinline__ void fence_proxy_async_shared()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 __device__ __forceinline__ void mbar_arrive(uint32_t bar)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
@@ -105,6 +112,17 @@ __device__ __forceinline__ uint32_t cluster_nctarank()
 }
 
 // all threads of all CTAs of the cluster; every thread of a warp must execute it
+// the two halves of cluster_sync_all, for a barrier whose wait is deferred
+__device__ __forceinline__ void cluster_arrive()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_wait()
+{
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void cluster_sync_all()
 {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");

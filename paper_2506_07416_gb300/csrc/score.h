@@ -14,6 +14,7 @@ constexpr int kMaxText = 128;            // text tokens per request handled by t
 constexpr int kMaxTilesPerCta = 32;      // score tiles one CTA may own
 constexpr int kMaxCluster = 16;
 constexpr int kOrderMax = 2048;          // batches up to this size are launched largest request first
+constexpr int kOffsetsByValue = 64;      // batches up to this size carry their offsets in the launch parameters
 
 struct ScoreLaunch {
     const int32_t* seq_off;   // device [batch+1]
@@ -36,6 +37,13 @@ struct ScoreLaunch {
     // [sum T][Hq] normaliser terms of the system and causal text keys (unit of
     // the merged statistic b, from ctx_stats.cu), or null: visual keys only
     const float* extra;
+    // nv > 0 (batches of at most kOffsetsByValue requests): the seq / text
+    // offsets by value, equal to seq_off / text_off (the host mirrors), so a
+    // CTA knows its tiles without a global load and its first copies go out as
+    // soon as its setup is done. nv == 0: read seq_off / text_off.
+    int32_t nv;
+    int32_t so_v[kOffsetsByValue + 1];
+    int32_t to_v[kOffsetsByValue + 1];
     // Cluster k of the 1-D grid serves item k: request order[k / groups] (the
     // requests from the largest to the smallest, so the hardware starts the
     // biggest clusters first and fills in with small ones), head group

@@ -98,6 +98,36 @@ __device__ __forceinline__ float transpose_sum32(float (&x)[32], int lane)
     return x[0];
 }
 
+// What a CTA serves of its request: the text rows, the tile range, and whether
+// the shape fits the kernel's buffers (uniform over the cluster).
+struct ResShape {
+    int N, t0, T, n2, n_tiles, tile_begin, mt, nb;
+    bool bad;
+};
+
+template <int RECV_COLS>
+__device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int n1, int tq, int t1, uint32_t rank,
+                                              uint32_t csize, int mrows)
+{
+    ResShape r;
+    r.N = n1 - n0;
+    r.t0 = p.query_last && t1 > tq ? t1 - 1 : tq;  // last-token queries: one row
+    r.T = t1 - r.t0;
+    r.n2 = (r.T + 15) & ~15;
+    r.n_tiles = (r.N + kTileRows - 1) / kTileRows;
+    const int tpc = r.N > 0 ? (r.n_tiles + (int)csize - 1) / (int)csize : 0;
+    // Shape errors are caught on the host; this only keeps the kernel within its buffers.
+    const int span = p.slot_cols / 2 + 32 * ((p.slot_cols / 2 + 31) / 32);  // columns the epilogue reads per slot
+    r.nb = p.res_nb == 2 ? 2 : 1;
+    const int buf_cols = r.nb == 2 ? kBufCols : kResTmemCols;
+    r.bad = r.T > mrows || r.n2 > p.slot_cols || (r.N > 0 && r.T <= 0) ||
+            (tpc > 0 && (tpc - 1) * p.slot_cols + span > buf_cols) ||
+            tpc > (r.nb == 2 ? kBufSlots : kResMaxSlots) || (int)csize * p.slot_cols > RECV_COLS;
+    r.tile_begin = min(r.n_tiles, (int)rank * tpc);
+    r.mt = min(r.n_tiles, r.tile_begin + tpc) - r.tile_begin;
+    return r;
+}
+
 template <int ROW_BYTES, bool FP8, int MROWS>
 __global__ void __launch_bounds__(kResThreads, 1)
     score_res_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -133,12 +163,14 @@ __global__ void __launch_bounds__(kResThreads, 1)
     // completes ahead of that one.
     if (!p.extra) griddep_wait();
     griddep_launch_dependents();
-    // The request's offsets are loaded here and first used after the setup
-    // below (barriers, TMEM, cluster barrier), so their latency overlaps it.
-    const int n0 = p.seq_off[b];
-    const int n1 = p.seq_off[b + 1];
-    const int tq = p.text_off[b];
-    const int t1 = p.text_off[b + 1];
+    // The request's offsets: by value for small batches; otherwise loaded here
+    // and first used after the setup below (barriers, TMEM, cluster barrier),
+    // so their latency overlaps it.
+    const bool byv = p.nv > 0;
+    const int n0 = byv ? p.so_v[b] : p.seq_off[b];
+    const int n1 = byv ? p.so_v[b + 1] : p.seq_off[b + 1];
+    const int tq = byv ? p.to_v[b] : p.text_off[b];
+    const int t1 = byv ? p.to_v[b + 1] : p.text_off[b + 1];
     const bool multi = p.groups > 1;
     const int G = p.hq / p.hkv;
     const int hpg = p.heads_per_group;
@@ -188,24 +220,18 @@ __global__ void __launch_bounds__(kResThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    cluster_sync_all();
+    // Cluster barrier, split: every thread arrives now (after its CTA's barriers
+    // exist) and waits only before its first access to a peer's shared memory
+    // (the epilogue, below) or before the final barrier (producer, MMA warp),
+    // so the first copies and contractions do not wait for the slowest CTA of
+    // the cluster to get here.
+    cluster_arrive();
     const uint32_t tmem = *tmem_slot;
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
-    const int N = n1 - n0;
-    const int t0 = p.query_last && t1 > tq ? t1 - 1 : tq;  // last-token queries: one row
-    const int T = t1 - t0;
-    const int n2 = (T + 15) & ~15;
-    const int n_tiles = (N + kTileRows - 1) / kTileRows;
-    const int tpc = N > 0 ? (n_tiles + (int)csize - 1) / (int)csize : 0;
-    // Uniform for the whole cluster (same request). Shape errors are caught on
-    // the host; this only keeps the kernel within its buffers.
-    const int span = p.slot_cols / 2 + 32 * ((p.slot_cols / 2 + 31) / 32);  // columns the epilogue reads per slot
-    const int nb = p.res_nb == 2 ? 2 : 1;
-    const int buf_cols = nb == 2 ? kBufCols : kResTmemCols;
-    const bool bad_shape = T > MROWS || n2 > p.slot_cols || (N > 0 && T <= 0) ||
-                           (tpc > 0 && (tpc - 1) * p.slot_cols + span > buf_cols) ||
-                           tpc > (nb == 2 ? kBufSlots : kResMaxSlots) || (int)csize * p.slot_cols > L::RECV_COLS;
+    const ResShape shp = res_shape<L::RECV_COLS>(p, n0, n1, tq, t1, rank, csize, MROWS);
+    const int N = shp.N, t0 = shp.t0, T = shp.T, n2 = shp.n2, nb = shp.nb;
+    const bool bad_shape = shp.bad;  // uniform for the whole cluster (same request)
     if (bad_shape || N <= 0) {
         if (p.extra) griddep_wait();
         if (bad_shape && threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
@@ -215,12 +241,13 @@ __global__ void __launch_bounds__(kResThreads, 1)
             tc_fence_after();
             tmem_dealloc(tmem, kResTmemCols);
         }
+        cluster_wait();
         cluster_sync_all();
         return;
     }
-    const int tile_begin = min(n_tiles, (int)rank * tpc);
-    const int tile_end = min(n_tiles, tile_begin + tpc);
-    const int mt = tile_end - tile_begin;
+    const int tile_begin = shp.tile_begin;
+    const int tile_end = tile_begin + shp.mt;
+    const int mt = shp.mt;
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
@@ -261,6 +288,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 if (q_issued[s] > 0) wait_phase(BAR(Q_FULL + s), (uint32_t)(q_issued[s] - 1) & 1u, drain_ctl);
         }
         __syncwarp();
+        cluster_wait();
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
@@ -302,8 +330,10 @@ __global__ void __launch_bounds__(kResThreads, 1)
             wait_phase(BAR(DRAIN), 0, drain_ctl);
         }
         __syncwarp();
+        cluster_wait();
     } else {
         // ------------------------------------------------------------ epilogue (2 warpgroups)
+        cluster_wait();  // the peers' barriers and buffers exist before any statistics go out
         // Control flow is identical for every thread of a warpgroup (named
         // barriers); after an abort every wait returns at once. Warp-synchronous
         // instructions (tcgen05.ld, redux.sync, shuffles) run under branches

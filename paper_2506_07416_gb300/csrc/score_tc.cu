@@ -122,10 +122,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     // completes ahead of that one.
     if (!p.extra) griddep_wait();
     griddep_launch_dependents();
-    const int n0 = p.seq_off[b];
-    const int N = p.seq_off[b + 1] - n0;
-    const int t1 = p.text_off[b + 1];
-    const int t0 = p.query_last && t1 > p.text_off[b] ? t1 - 1 : p.text_off[b];  // last-token queries: one row
+    // the request's offsets: by value for small batches (no global load)
+    const bool byv = p.nv > 0;
+    const int n0 = byv ? p.so_v[b] : p.seq_off[b];
+    const int N = (byv ? p.so_v[b + 1] : p.seq_off[b + 1]) - n0;
+    const int tq = byv ? p.to_v[b] : p.text_off[b];
+    const int t1 = byv ? p.to_v[b + 1] : p.text_off[b + 1];
+    const int t0 = p.query_last && t1 > tq ? t1 - 1 : tq;  // last-token queries: one row
     const int T = t1 - t0;
     const bool multi = p.groups > 1;
     // Uniform for the whole cluster (same request). With several head groups
@@ -196,7 +199,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    cluster_sync_all();  // every CTA's barriers exist before any remote arrival
+    // Cluster barrier, split: every thread arrives now (its CTA's barriers
+    // exist) and waits only before its first remote arrival (the epilogue) or
+    // before the final barrier (producer, MMA warp), so the first copies and
+    // contractions do not wait for the slowest CTA of the cluster.
+    cluster_arrive();
     const uint32_t tmem = *tmem_slot;
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
@@ -248,6 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (q_issued[s] > 0) wait_phase(BAR(Q_FULL + s), (uint32_t)(q_issued[s] - 1) & 1u, drain_ctl);
         }
         __syncwarp();
+        cluster_wait();
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
@@ -307,8 +315,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             wait_phase(BAR(DRAIN), 0, drain_ctl);
         }
         __syncwarp();
+        cluster_wait();
     } else {
         // ------------------------------------------------------------ epilogue
+        cluster_wait();  // the peers' barriers and buffers exist before any statistics go out
         // Three warpgroups (warps 2-5, 6-9, 10-13). The contractions of both
         // passes cycle through four TMEM buffers in issue order; warpgroup g
         // takes the units u with u % 3 == g, in order, so while one warpgroup

@@ -370,7 +370,7 @@ __global__ void __launch_bounds__(kTopkThreads)
         float sum[KPT];
 #pragma unroll
         for (int e = 0; e < KPT; ++e) sum[e] = 0.f;
-        constexpr int QG = KPT <= 4 ? 8 : (KPT <= 8 ? 4 : 2);  // loads in flight per key, within the registers
+        constexpr int QG = KPT <= 4 ? 16 : (KPT <= 8 ? 4 : 2);  // loads in flight per key, within the registers
         for (int g0 = 0; g0 < sh.groups; g0 += QG) {
             float v[KPT][QG];
 #pragma unroll
