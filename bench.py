@@ -311,16 +311,17 @@ def run_ours(args):
         if rc != 0:
             raise select.LitevlmError(rc, L.litevlm_select_last_error(h).decode())
 
-    def step(q, k, so_d, to_d, hidden_srcs=None):
+    def step(q, k, so_d, to_d, hidden_srcs=None, s_ptr=None):
         """One step: scores and top-k (one call: the top-k kernel adds the
         head-group partials), then the gather; returns the kernels launched."""
+        st_ = sp if s_ptr is None else s_ptr
         call(L.litevlm_select_score_topk(h, w.batch, q.data_ptr(), to_d.data_ptr(), c_to_h, k.data_ptr(),
                                          so_d.data_ptr(), c_so_h, xd["q_scale"], xd["k_scale"], scores.data_ptr(),
                                          c_kk_d, c_kk_h, ratio, kept.data_ptr(), off_d.data_ptr(),
-                                         off_h.ctypes.data, sp))
+                                         off_h.ctypes.data, st_))
         n = L.litevlm_select_last_launches(h)
         call(L.litevlm_select_compact(h, total_kept, kept.data_ptr(), w.total_vis, n_t,
-                                      hidden_srcs if hidden_srcs is not None else c_src, c_dst, c_rb, sp))
+                                      hidden_srcs if hidden_srcs is not None else c_src, c_dst, c_rb, st_))
         return n + L.litevlm_select_last_launches(h)
 
     q, k, so_d, to_d = xd["q"], xd["k"], xd["seq_offsets"], xd["text_offsets"]
@@ -408,7 +409,10 @@ def run_ours(args):
            "project": run_project(w, xd, sel, dev, stream, steps, pk)}
 
     # end to end through the public API with host buffers
-    e2e = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept)
+    e2e = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel)
+    e2e["copy_all_inputs"] = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel,
+                                     gather_from_host=False)
+    e2e["eager"] = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, graph=False)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -617,17 +621,32 @@ def run_views(w, sel, dev, stream, steps):
             "mean_views_selected": sel_views / max(1, w.batch)}
 
 
-def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept):
-    """Host buffers in, selection out, through the C-ABI: every step copies its
-    inputs (q, K, offsets and the gathered tensors, packed in one pinned host
+def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, gather_from_host=True, graph=True):
+    """Host buffers in, selection out, through the C-ABI, all inside the timed
+    region: every step copies q, K and the offsets (packed in one pinned host
     buffer) to the device, runs the three calls, and reads the kept indices and
-    offsets back into pinned host memory, all inside the timed region. Inputs are
-    double-buffered on the device and copied on a second stream, so the copy of
-    step i + 1 overlaps the kernels of step i (the way a serving loop would run
-    it); each step's kernels wait for its own copy."""
+    offsets back into pinned host memory. Inputs are double-buffered on the
+    device and copied on a second stream, so the copy of step i + 1 overlaps the
+    kernels of step i (the way a serving loop would run it); each step's kernels
+    wait for its own copy.
+
+    The gathered tensors other than K (hidden states, V) stay in pinned host
+    memory and the gather reads only their kept rows through the device view
+    (litevlm_select_host_view), so only those rows cross the host link
+    (gather_from_host=True). With gather_from_host=False they are copied whole
+    with the other inputs every step. h2d_bytes_per_step counts what crosses
+    the link either way.
+
+    graph=True: the calls of 8 consecutive steps (copies, the C-ABI calls with
+    their kernels, result copies, and the events between the two streams) are
+    captured once into a CUDA graph, which the timed loop replays, so the host
+    issues one launch per 8 steps instead of about fifteen API calls per step.
+    The device work is the same as in the eager loop (graph=False), whose time
+    is bound by the host's issue rate on small workloads."""
     import torch
-    names = ["q", "k", "seq_offsets", "text_offsets"] + [n for n in w.gather if n not in ("k",)]
-    sizes = {n: xd[n].numel() * xd[n].element_size() for n in names}
+    host_gather = [n for n in w.gather if n != "k"] if gather_from_host else []
+    names = ["q", "k", "seq_offsets", "text_offsets"] + [n for n in w.gather if n != "k" and n not in host_gather]
+    sizes = {n: xd[n].numel() * xd[n].element_size() for n in names + host_gather}
     offs, tot = {}, 0
     for n in names:
         offs[n] = tot
@@ -635,51 +654,89 @@ def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept):
     host = torch.empty(tot, dtype=torch.uint8).pin_memory()
     for n in names:
         host[offs[n]:offs[n] + sizes[n]].copy_(xd[n].contiguous().view(-1).view(torch.uint8).cpu())
+    # the host-resident gather sources and their device views
+    resident = {n: xd[n].cpu().pin_memory() for n in host_gather}
+    resident_view = {n: sel.host_view(resident[n]) for n in host_gather}
     bufs = [torch.empty(tot, dtype=torch.uint8, device=dev) for _ in range(2)]
 
     def views(buf):
         return {n: buf[offs[n]:offs[n] + sizes[n]].view(xd[n].dtype).view(xd[n].shape) for n in names}
 
     dv = [views(b) for b in bufs]
-    c_srcs = [(ctypes.c_void_p * len(w.gather))(*[d[n].data_ptr() for n in w.gather]) for d in dv]
+    c_srcs = [(ctypes.c_void_p * len(w.gather))(*[resident_view[n] if n in resident_view else d[n].data_ptr()
+                                                  for n in w.gather]) for d in dv]
     res_h = torch.empty(kept.numel() + off_d.numel(), dtype=torch.int32).pin_memory()
     nk = kept.numel()
     steps = args.e2e_steps if args.e2e_steps is not None else max(3, min(200, (args.steps or DEFAULTS[w.name][0])))
     copy_stream = torch.cuda.Stream(device=dev)
     copied = [torch.cuda.Event() for _ in range(2)]
     used = [torch.cuda.Event() for _ in range(2)]
-    h2d = tot
+    h2d = tot + sum(total_kept * (sizes[n] // xd[n].shape[0]) for n in host_gather)
     d2h = res_h.numel() * 4
 
-    def one(i):
+    def one(i, st, wait_used=True):
         sl = i & 1
         with torch.cuda.stream(copy_stream):
-            copy_stream.wait_event(used[sl])      # the kernels of step i - 2 are done with this buffer
+            if wait_used:
+                copy_stream.wait_event(used[sl])  # the kernels of step i - 2 are done with this buffer
             bufs[sl].copy_(host, non_blocking=True)
             copied[sl].record(copy_stream)
-        stream.wait_event(copied[sl])
+        st.wait_event(copied[sl])
         d = dv[sl]
-        step(d["q"], d["k"], d["seq_offsets"], d["text_offsets"], c_srcs[sl])
-        used[sl].record(stream)
-        res_h[:nk].copy_(kept, non_blocking=True)
-        res_h[nk:].copy_(off_d, non_blocking=True)
+        step(d["q"], d["k"], d["seq_offsets"], d["text_offsets"], c_srcs[sl], st.cuda_stream)
+        used[sl].record(st)
+        with torch.cuda.stream(st):
+            res_h[:nk].copy_(kept, non_blocking=True)
+            res_h[nk:].copy_(off_d, non_blocking=True)
 
     for i in range(4):
-        one(i)
+        one(i, stream)
     torch.cuda.synchronize()
+    per_graph = 8
+    g = None
+    if graph:
+        cap = torch.cuda.Stream(device=dev)
+        cap.wait_stream(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap, capture_error_mode="relaxed"):
+            fork = torch.cuda.Event()
+            fork.record(cap)
+            copy_stream.wait_event(fork)  # the copy stream joins the capture
+            for i in range(per_graph):
+                # steps 0 and 1 of a replay follow the previous replay in stream order
+                one(i, cap, wait_used=i >= 2)
+            cap.wait_stream(copy_stream)  # and leaves it
+        torch.cuda.synchronize()
+        steps = max(per_graph, (steps + per_graph - 1) // per_graph * per_graph)
+        g.replay()
+        torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     copy_stream.wait_event(e0)
-    for i in range(steps):
-        one(i)
+    if g is not None:
+        with torch.cuda.stream(stream):
+            for _ in range(steps // per_graph):
+                g.replay()
+    else:
+        for i in range(steps):
+            one(i, stream)
     stream.wait_stream(copy_stream)
     e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
+    if host_gather:
+        api = ("litevlm_select_score_topk + compact" + (" (8 steps captured into a CUDA graph, replayed)" if g else "")
+               + "; each step copies q, K and the offsets from one pinned host "
+               "buffer into one of two device buffers on a copy stream; the gather reads the kept rows of "
+               + ", ".join(host_gather) + " straight from pinned host memory (litevlm_select_host_view); "
+               "kept indices + offsets copied back")
+    else:
+        api = ("litevlm_select_score_topk + compact" + (" (8 steps captured into a CUDA graph, replayed)" if g else "")
+               + "; each step's inputs (gathered tensors included) copied from "
+               "one pinned host buffer into one of two device buffers on a copy stream, kept indices + offsets "
+               "copied back")
     return {"value": w.total_vis * steps / (ms / 1e3) / 1e6, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "steps": steps, "ms_per_step": ms / steps,
-            "api": "litevlm_select_score/topk/compact; each step's inputs copied from one pinned host buffer "
-                   "into one of two device buffers on a copy stream, kept indices + offsets copied back"}
+            "d2h_bytes_per_step": int(d2h), "steps": steps, "ms_per_step": ms / steps, "api": api}
 
 
 def measure_fp8_peak(n: int = 8192, reps: int = 50):

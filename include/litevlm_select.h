@@ -289,7 +289,10 @@ litevlm_status_t litevlm_select_topk(litevlm_select_t handle, int32_t batch, con
  *   src_rows     rows of every source tensor (sum N_b)
  *   num_tensors  1..8 tensors gathered with the same index list
  *   src, dst     HOST arrays of num_tensors DEVICE pointers; src[t] is
- *                [src_rows, row_bytes[t]], dst[t] is [total_kept, row_bytes[t]]
+ *                [src_rows, row_bytes[t]], dst[t] is [total_kept, row_bytes[t]].
+ *                A src[t] may be the device view of pinned host memory
+ *                (litevlm_select_host_view): the kernel then reads the kept
+ *                rows over the host link, and no other row crosses it.
  *   row_bytes    HOST array of num_tensors row sizes in bytes (> 0)
  * dst[t][r] = src[t][kept_idx[r]] byte for byte. Rows whose size and pointers are
  * 16-byte aligned move with 128-bit loads and stores; others byte by byte.
@@ -300,6 +303,23 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t handle, int64_t total_k
                                         int64_t src_rows, int32_t num_tensors,
                                         const void* const* src, void* const* dst, const int64_t* row_bytes,
                                         litevlm_stream_t stream);
+
+/*
+ * Device view of pinned host memory, so that the gather can take its source
+ * rows straight from the host (only the kept rows then cross the host link:
+ * the score reads every K row, the gather only the kept hidden / K / V rows).
+ *   host         HOST pointer into memory from cudaHostAlloc / cudaMallocHost
+ *                (or registered with cudaHostRegister as mapped)
+ *   device_view  out: the address a kernel uses for `host`
+ *                (cudaHostGetDevicePointer; the same address where the host
+ *                and the device share one address space)
+ * LITEVLM_ERR_INVALID_ARG if the runtime gives the memory no device address
+ * (memory that is neither pinned nor mapped, on a system whose GPU does not use
+ * the host's page tables); nothing is enqueued. The view stays valid while the
+ * memory stays pinned; the caller keeps the host data unchanged until the
+ * gather that reads it has finished.
+ */
+litevlm_status_t litevlm_select_host_view(litevlm_select_t handle, const void* host, void** device_view);
 
 
 /*

@@ -931,6 +931,21 @@ litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_
     return LITEVLM_OK;
 }
 
+litevlm_status_t litevlm_select_host_view(litevlm_select_t h, const void* host, void** device_view)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (!host || !device_view) return fail(h, LITEVLM_ERR_INVALID_ARG, "host and device_view must not be NULL");
+    void* d = nullptr;
+    const cudaError_t e = cudaHostGetDevicePointer(&d, const_cast<void*>(host), 0);
+    if (e != cudaSuccess || !d) {
+        (void)cudaGetLastError();  // not sticky: leave no error behind for the next call
+        return fail(h, LITEVLM_ERR_INVALID_ARG, "the runtime gives this host memory no device address");
+    }
+    *device_view = d;
+    return LITEVLM_OK;
+}
+
 }  // extern "C"
 
 // ----------------------------------------------------------------------------

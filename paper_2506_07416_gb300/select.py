@@ -61,11 +61,12 @@ def _load():
     lib.litevlm_select_compact.argtypes = [P, i64, P, i64, i32, P, P, P, P]
     lib.litevlm_select_score_topk.argtypes = [P, i32, P, P, P, P, P, P, f32, f32, P, P, P, f32, P, P, P, P]
     lib.litevlm_select_check_device.argtypes = [P, P]
+    lib.litevlm_select_host_view.argtypes = [P, P, ctypes.POINTER(P)]
     lib.litevlm_select_score_plan.argtypes = [P, i32, P, P, P]
     lib.litevlm_select_splice.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, P, P, i64, P, P, P, P, P]
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
     for fn in ("create", "destroy", "score", "score_full_keys", "topk", "compact", "check_device", "score_plan",
-               "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project", "score_topk"):
+               "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project", "score_topk", "host_view"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -78,7 +79,7 @@ EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_la
            "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc",
            "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views",
            "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project",
-           "litevlm_select_last_launches", "litevlm_select_score_topk"]
+           "litevlm_select_last_launches", "litevlm_select_score_topk", "litevlm_select_host_view"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -225,6 +226,13 @@ def splice(handle: int, batch: int, sys_rows, sys_offsets_d, sys_offsets_h, vis_
                                      _ptr(txt_rows), _ptr(text_offsets_d), _ptr(to), int(row_bytes), _ptr(out_rows),
                                      _ptr(out_offsets_d), _ptr(out_offsets_h), _ptr(position_ids),
                                      _stream_ptr(stream)), handle)
+
+
+def host_view(handle: int, host_ptr: int) -> int:
+    """litevlm_select_host_view: the device address of pinned host memory."""
+    out = ctypes.c_void_p()
+    _check(LIB.litevlm_select_host_view(handle, host_ptr, ctypes.byref(out)), handle)
+    return int(out.value)
 
 
 def check_device(handle: int, stream=None) -> None:
@@ -397,14 +405,22 @@ class Selector:
         return kept_idx[:int(off_h[-1])], out_offsets, off_h
 
     def compact(self, kept_idx, total_kept: int, srcs: Sequence, dsts: Optional[List] = None, stream=None):
+        """Gathers the kept rows of each source into the device. A source in
+        pinned host memory is read through its device view, so only its kept
+        rows cross the host link."""
         import torch
         rows = [s.shape[0] for s in srcs]
         if dsts is None:
-            dsts = [torch.empty((max(total_kept, 0),) + tuple(s.shape[1:]), dtype=s.dtype, device=s.device)
+            dsts = [torch.empty((max(total_kept, 0),) + tuple(s.shape[1:]), dtype=s.dtype, device=kept_idx.device)
                     for s in srcs]
         rb = [s[0].numel() * s.element_size() if s.shape[0] else 1 for s in srcs]
-        compact(self.handle, total_kept, kept_idx, min(rows) if rows else 0, srcs, dsts, rb, stream)
+        src_ptrs = [self.host_view(s) if s.device.type == "cpu" else s for s in srcs]
+        compact(self.handle, total_kept, kept_idx, min(rows) if rows else 0, src_ptrs, dsts, rb, stream)
         return dsts
+
+    def host_view(self, t) -> int:
+        """Device address of a pinned host tensor (or host pointer)."""
+        return host_view(self.handle, _ptr(t))
 
     def splice(self, sys_rows, sys_offsets, vis_rows, seq_offsets, kept_idx, kept_offsets, txt_rows, text_offsets,
                stream=None):

@@ -259,6 +259,36 @@ def test_compact_out_of_range_index_is_reported(sel):
     s.check_device()  # the word was cleared
 
 
+@pytest.mark.parametrize("row_bytes", [4096, 112, 6])
+def test_compact_from_pinned_host_memory_bit_exact(sel, row_bytes):
+    """Sources in pinned host memory are read through their device view: the
+    gathered rows are the source rows byte for byte, next to a device source
+    gathered with the same indices."""
+    w = _case("g", 1, 1, 128, "bf16", [8], [1])
+    s = _selector(sel, w)
+    rng = np.random.default_rng(5)
+    rows = 3000
+    src_np = rng.integers(0, 256, size=(rows, row_bytes), dtype=np.uint8)
+    host = torch.from_numpy(src_np).pin_memory()
+    dev_src = host.cuda()
+    idx_np = np.sort(rng.choice(rows, 907, replace=False)).astype(np.int32)
+    idx = torch.from_numpy(idx_np).cuda()
+    from_host, from_dev = s.compact(idx, len(idx_np), [host, dev_src])
+    s.check_device()
+    np.testing.assert_array_equal(from_host.cpu().numpy(), src_np[idx_np])
+    np.testing.assert_array_equal(from_dev.cpu().numpy(), src_np[idx_np])
+
+
+def test_host_view_argument_errors(sel):
+    w = _case("g", 1, 1, 128, "bf16", [8], [1])
+    s = _selector(sel, w)
+    with pytest.raises(sel.LitevlmError) as e:
+        s.host_view(0)
+    assert e.value.name == "INVALID_ARG"
+    host = torch.zeros(64, dtype=torch.uint8).pin_memory()
+    assert s.host_view(host) != 0
+
+
 # ----------------------------------------------------------------------------- whole path
 
 def test_tiny_whole_path(sel):
