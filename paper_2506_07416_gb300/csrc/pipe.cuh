@@ -73,13 +73,20 @@ __device__ __forceinline__ void row_stats_update(const float* v, int valid, floa
     const float mc = m_new * cl;
     float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
     if (valid >= NV) {
+        // packed pairs: the same per-column fma and sums, half the instructions
+        const float2 cl2 = make_float2(cl, cl), nmc2 = make_float2(-mc, -mc);
+        float2 s01 = make_float2(0.f, 0.f), s23 = make_float2(0.f, 0.f);
 #pragma unroll
         for (int c = 0; c < NV; c += 4) {
-            s0 += ex2(fmaf(v[c], cl, -mc));
-            s1 += ex2(fmaf(v[c + 1], cl, -mc));
-            s2 += ex2(fmaf(v[c + 2], cl, -mc));
-            s3 += ex2(fmaf(v[c + 3], cl, -mc));
+            const float2 x01 = ffma2(make_float2(v[c], v[c + 1]), cl2, nmc2);
+            const float2 x23 = ffma2(make_float2(v[c + 2], v[c + 3]), cl2, nmc2);
+            s01 = fadd2(s01, make_float2(ex2(x01.x), ex2(x01.y)));
+            s23 = fadd2(s23, make_float2(ex2(x23.x), ex2(x23.y)));
         }
+        s0 = s01.x;
+        s1 = s01.y;
+        s2 = s23.x;
+        s3 = s23.y;
     } else {
 #pragma unroll
         for (int c = 0; c < NV; c += 4) {

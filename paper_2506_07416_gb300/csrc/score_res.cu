@@ -356,7 +356,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         float* accw = acc_s + wg * kResMaxSlots * kTileRows;
         float* ssum = scr_sum + wg * 4 * 64;
         float* b2w = b2_s + wg * 64;                   // weight of column c_begin + c, 0 for c >= h2 or >= T
-        float* mcw = mc_s + wg * 64;                   // CTA column max * c of column c_begin + c
+        float* mcw = mc_s + wg * 64;                   // -(CTA column max * c) of column c_begin + c
         const uint32_t recv_base = base + L::OFF_RECV;
         const uint32_t tcol = tmem + lane_off;
         for (int tl = 0; tl < mt; ++tl) accw[tl * kTileRows + vrow] = 0.f;
@@ -431,7 +431,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     float m = smax[32 * ch + wt];
 #pragma unroll
                     for (int q = 1; q < 4; ++q) m = fmaxf(m, smax[q * 64 + 32 * ch + wt]);
-                    mcw[32 * ch + wt] = m * cl;  // columns past cw: garbage, never used
+                    mcw[32 * ch + wt] = -(m * cl);  // columns past cw: garbage, never used
                 }
                 named_bar_sync(wg_bar, 128);
             }
@@ -456,21 +456,26 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     tmem_ld32(ta, v);
                     tmem_wait_ld();
                     const bool ok = lane_valid(tl);
+                    const float2 cl2 = make_float2(cl, cl);
 #pragma unroll
                     for (int c = 0; c < 32; c += 4) {
                         const float4 m4 = *reinterpret_cast<const float4*>(mcw + 32 * ch + c);
-                        const float e0 = ok ? ex2(fmaf(v[c], cl, -m4.x)) : 0.f;
-                        const float e1 = ok ? ex2(fmaf(v[c + 1], cl, -m4.y)) : 0.f;
-                        const float e2 = ok ? ex2(fmaf(v[c + 2], cl, -m4.z)) : 0.f;
-                        const float e3 = ok ? ex2(fmaf(v[c + 3], cl, -m4.w)) : 0.f;
+                        const float2 x01 = ffma2(make_float2(v[c], v[c + 1]), cl2, make_float2(m4.x, m4.y));
+                        const float2 x23 = ffma2(make_float2(v[c + 2], v[c + 3]), cl2, make_float2(m4.z, m4.w));
+                        const float e0 = ok ? ex2(x01.x) : 0.f;
+                        const float e1 = ok ? ex2(x01.y) : 0.f;
+                        const float e2 = ok ? ex2(x23.x) : 0.f;
+                        const float e3 = ok ? ex2(x23.y) : 0.f;
                         v[c] = e0;
                         v[c + 1] = e1;
                         v[c + 2] = e2;
                         v[c + 3] = e3;
-                        sm[c] += e0;
-                        sm[c + 1] += e1;
-                        sm[c + 2] += e2;
-                        sm[c + 3] += e3;
+                        const float2 s01 = fadd2(make_float2(sm[c], sm[c + 1]), make_float2(e0, e1));
+                        const float2 s23 = fadd2(make_float2(sm[c + 2], sm[c + 3]), make_float2(e2, e3));
+                        sm[c] = s01.x;
+                        sm[c + 1] = s01.y;
+                        sm[c + 2] = s23.x;
+                        sm[c + 3] = s23.y;
                     }
                     tmem_st_cols(ta, v, cw);
                 }
@@ -550,28 +555,20 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     tmem_wait_ld();  // va: slot tl
                     if (last) release(buf, tl);
                     if (tl + 1 < mt) tmem_ld32(tbuf + (uint32_t)((tl + 1) * scols) + col0, vb);
-                    float a0 = 0.f, a1 = 0.f;
+                    float2 a01 = make_float2(0.f, 0.f);
 #pragma unroll
-                    for (int c = 0; c < 32; c += 2) {
-                        if (c < cw) {
-                            a0 = fmaf(va[c], wv[c], a0);
-                            a1 = fmaf(va[c + 1], wv[c + 1], a1);
-                        }
-                    }
-                    accw[tl * kTileRows + vrow] += a0 + a1;
+                    for (int c = 0; c < 32; c += 2)
+                        if (c < cw) a01 = ffma2(make_float2(va[c], va[c + 1]), make_float2(wv[c], wv[c + 1]), a01);
+                    accw[tl * kTileRows + vrow] += a01.x + a01.y;
                     if (tl + 1 < mt) {
                         tmem_wait_ld();  // vb: slot tl + 1
                         if (last) release(buf, tl + 1);
                         if (tl + 2 < mt) tmem_ld32(tbuf + (uint32_t)((tl + 2) * scols) + col0, va);
-                        a0 = a1 = 0.f;
+                        a01 = make_float2(0.f, 0.f);
 #pragma unroll
-                        for (int c = 0; c < 32; c += 2) {
-                            if (c < cw) {
-                                a0 = fmaf(vb[c], wv[c], a0);
-                                a1 = fmaf(vb[c + 1], wv[c + 1], a1);
-                            }
-                        }
-                        accw[(tl + 1) * kTileRows + vrow] += a0 + a1;
+                        for (int c = 0; c < 32; c += 2)
+                            if (c < cw) a01 = ffma2(make_float2(vb[c], vb[c + 1]), make_float2(wv[c], wv[c + 1]), a01);
+                        accw[(tl + 1) * kTileRows + vrow] += a01.x + a01.y;
                     }
                 }
             }

@@ -419,9 +419,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                             griddep_wait();
                             bm = log2_add(bm, p.extra[(int64_t)(t0 + et) * p.hq + hg * hpg + hs]);
                         }
-                        b2[et] = bm;
+                        b2[et] = -bm;  // stored negated: the fma addend of pass 2
                     } else {
-                        b2[et] = INFINITY;
+                        b2[et] = -INFINITY;
                     }
                 }
                 named_bar_sync(1, kEpiThreads);
@@ -432,7 +432,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     wait_phase(BAR(U_FULL + ub), (ui >> 2) & 1, ctl);
                     tc_fence_after();
                     const uint32_t ta = tmem + lane_off + ub * 128u;
-                    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+                    float2 a01 = make_float2(0.f, 0.f), a23 = make_float2(0.f, 0.f);
+                    const float2 cl2 = make_float2(cl, cl);
 #pragma unroll
                     for (int hh = 0; hh < MROWS / 32; ++hh) {
                         const int c0 = hh * 32;
@@ -447,10 +448,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                                     for (int e = 0; e < 16; e += 4) {
                                         const float4 bb = *reinterpret_cast<const float4*>(b2 + c0 + k * 16 + e);
-                                        a0 += ex2(fmaf(v[k * 16 + e], cl, -bb.x));
-                                        a1 += ex2(fmaf(v[k * 16 + e + 1], cl, -bb.y));
-                                        a2 += ex2(fmaf(v[k * 16 + e + 2], cl, -bb.z));
-                                        a3 += ex2(fmaf(v[k * 16 + e + 3], cl, -bb.w));
+                                        const float2 x01 = ffma2(make_float2(v[k * 16 + e], v[k * 16 + e + 1]), cl2,
+                                                                 make_float2(bb.x, bb.y));
+                                        const float2 x23 = ffma2(make_float2(v[k * 16 + e + 2], v[k * 16 + e + 3]),
+                                                                 cl2, make_float2(bb.z, bb.w));
+                                        a01 = fadd2(a01, make_float2(ex2(x01.x), ex2(x01.y)));
+                                        a23 = fadd2(a23, make_float2(ex2(x23.x), ex2(x23.y)));
                                     }
                                 }
                             }
@@ -459,7 +462,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(BAR(U_EMPTY + ub));
-                    acc_s[(t - tile_begin) * kTileRows + vrow] += (a0 + a1) + (a2 + a3);
+                    acc_s[(t - tile_begin) * kTileRows + vrow] += (a01.x + a01.y) + (a23.x + a23.y);
                 }
             }
         }
