@@ -53,11 +53,11 @@ __device__ __forceinline__ void row_stats_update(const float* v, int valid, floa
     float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
     if (valid >= NV) {
 #pragma unroll
-        for (int c = 0; c < NV; c += 4) {
-            mx0 = fmaxf(mx0, v[c]);
-            mx1 = fmaxf(mx1, v[c + 1]);
-            mx2 = fmaxf(mx2, v[c + 2]);
-            mx3 = fmaxf(mx3, v[c + 3]);
+        for (int c = 0; c < NV; c += 8) {
+            mx0 = fmax3(mx0, v[c], v[c + 1]);
+            mx1 = fmax3(mx1, v[c + 2], v[c + 3]);
+            mx2 = fmax3(mx2, v[c + 4], v[c + 5]);
+            mx3 = fmax3(mx3, v[c + 6], v[c + 7]);
         }
     } else {
 #pragma unroll

@@ -42,6 +42,14 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b)
     return r;
 }
 
+// three-input maximum (one instruction)
+__device__ __forceinline__ float fmax3(float a, float b, float c)
+{
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
 __device__ __forceinline__ float ex2(float x)
 {
     float y;
