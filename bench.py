@@ -87,6 +87,36 @@ def algorithmic(w):
             "compact_bytes": compact_bytes, "kept": ks, "row_total": row_total}
 
 
+def stage_rooflines(alg, stage_us, step_us, pk, dtype):
+    """Roofline of each stage and of the whole step.
+
+    A stage's roofline time is the slower of its FLOPs at the tensor peak and
+    its algorithmic bytes at the HBM peak. `frac` = roofline time / measured
+    time. The step's roofline is the sum over the three stages, against the
+    measured step time (events at step boundaries). The e4m3 tensor peak is
+    the measured bf16 peak times the nominal 2:1 ratio of the two."""
+    hbm = pk["hbm_gbs"] * 1e9
+    tensor = pk["bf16_tflops"] * 1e12 * (1.0 if dtype == "bf16" else 2.0)
+    work = {"score": (alg["score_flops"], alg["score_bytes"]), "topk": (0, alg["topk_bytes"]),
+            "compact": (0, alg["compact_bytes"])}
+    out = {}
+    total = 0.0
+    for name, (flops, nbytes) in work.items():
+        t_flops, t_bytes = flops / tensor * 1e6, nbytes / hbm * 1e6
+        roof_us = max(t_flops, t_bytes)
+        total += roof_us
+        measured = float(stage_us[name])
+        out[name] = {"bound": "tensor" if t_flops > t_bytes else "hbm", "algorithmic_bytes": int(nbytes),
+                     "flops": int(flops), "roofline_us": roof_us, "measured_us": measured,
+                     "frac": roof_us / measured if measured > 0 else None}
+    out["step"] = {"roofline_us": total, "measured_us": float(step_us),
+                   "frac": total / step_us if step_us > 0 else None}
+    out["peaks"] = {"hbm_gbs": pk["hbm_gbs"], "tensor_tflops": tensor / 1e12,
+                    "source": pk["source"] + (" (bf16 burst)" if dtype == "bf16" else
+                                              " (bf16 burst x 2, the nominal e4m3 ratio)")}
+    return out
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -437,6 +467,7 @@ def run_ours(args):
                        "score_launch": {"kernel": select.KERNELS.get(plan[0]), "cluster": plan[1],
                                         "tiles_per_cta": plan[2], "head_groups": plan[3]}},
             "stages_p50_us": stage_us,
+            "stages_roofline": stage_rooflines(alg, stage_us, float(np.median(per_step_ms) * 1e3), pk, w.dtype),
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "next": nxt,
             "gpu_launches": launches_per_step * steps, "clocks": clocks,
             "wall_s": wall}
