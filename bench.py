@@ -637,9 +637,16 @@ def run_views(w, sel, dev, stream, steps):
             mask.data_ptr(), vo.data_ptr(), sv.data_ptr(), so.data_ptr(), None, stream.cuda_stream)
     for _ in range(3):
         assert L.litevlm_select_views(*args) == 0
+    n = max(3, min(steps, 200))
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    # the kernel takes a few microseconds, less than the host needs per call: a
+    # spin on the GPU (about 50 us per call) lets the host queue every call
+    # first, so each event pair brackets GPU work only, not host gaps
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(100_000 * n)
     ts = []
-    for _ in range(max(3, min(steps, 200))):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for e0, e1 in evs:
         e0.record(stream)
         assert L.litevlm_select_views(*args) == 0
         e1.record(stream)
