@@ -1,7 +1,8 @@
 // Per-request top-k of the visual-token scores (Results section, "Visual Token
 // Compression": a ratio r of the visual tokens is kept; Table 1 token counts).
 //
-// One CTA per request. Scores become order-preserving 32-bit keys (NaN -> 0,
+// One CTA per request (512 threads; the register kernel below takes 1024 on
+// requests of 2049 to 8192 tokens). Scores become order-preserving 32-bit keys (NaN -> 0,
 // the lowest key; -0 and +0 the same key), an MSB-first radix select (4 passes
 // of 8 bits, warp-aggregated shared-memory histograms) finds the k-th largest
 // key K* and how many keys equal to K* must be taken, then one pass over the
@@ -20,7 +21,8 @@ namespace lvs {
 
 namespace {
 
-constexpr int kTopkThreads = 512;
+constexpr int kTopkThreads = 512;      // the shared-memory kernel; register kernel up to 2048 tokens
+constexpr int kTopkWideThreads = 1024; // register kernel, 2049 .. 8192 tokens
 constexpr int kTopkWarps = kTopkThreads / 32;
 
 __device__ __forceinline__ uint32_t order_key(float f)
@@ -194,14 +196,15 @@ __global__ void __launch_bounds__(kTopkThreads)
 
 
 // The k largest keys of one request (0 < k < N), held KPT per thread by one CTA
-// of kTopkThreads threads (token j = e * kTopkThreads + tid), with the request's
+// of NT threads (token j = e * NT + tid), with the request's
 // smallest and largest key lo_k / hi_k. Calls emit(pos, j) once per kept token,
 // pos = its place among the kept tokens in index order (0 .. k-1). hist and cnt
 // are shared memory; hist[0] and hist[1] must be zero on entry.
-template <int KPT, class Emit>
+template <int KPT, int NT, class Emit>
 __device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, int k, uint32_t lo_k, uint32_t hi_k,
-                                            uint32_t (*hist)[256], int (*cnt)[kTopkWarps], Emit emit)
+                                            uint32_t (*hist)[256], int (*cnt)[NT / 32], Emit emit)
 {
+    constexpr int NW = NT / 32;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
     // ---- radix select below the common high bits
@@ -218,7 +221,7 @@ __device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, i
         uint32_t* h = hist[pass % 3];
 #pragma unroll
         for (int e = 0; e < KPT; ++e) {
-            if (e * kTopkThreads + tid < N && (key[e] & mask) == prefix) atomicAdd(&h[(key[e] >> lo) & dmask], 1u);
+            if (e * NT + tid < N && (key[e] & mask) == prefix) atomicAdd(&h[(key[e] >> lo) & dmask], 1u);
         }
         if (tid < 256) hist[(pass + 1) % 3][tid] = 0u;
         __syncthreads();
@@ -264,7 +267,7 @@ __device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, i
     uint32_t gt = 0, eq = 0;
 #pragma unroll
     for (int e = 0; e < KPT; ++e) {
-        const bool valid = e * kTopkThreads + tid < N;
+        const bool valid = e * NT + tid < N;
         const uint32_t m = key[e] & mask;
         gt |= (uint32_t)(valid && m > prefix) << e;
         eq |= (uint32_t)(valid && m == prefix) << e;
@@ -283,14 +286,14 @@ __device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, i
         keep = gt;
 #pragma unroll
         for (int e = 0; e < KPT; ++e) {
-            int v = lane < kTopkWarps ? cnt[e][lane] : 0;
+            int v = lane < NW ? cnt[e][lane] : 0;
 #pragma unroll
-            for (int o = 1; o < kTopkWarps; o <<= 1) {
+            for (int o = 1; o < NW; o <<= 1) {
                 const int y = __shfl_up_sync(0xffffffffu, v, o);
                 if (lane >= o) v += y;
             }
-            const int before_w = __shfl_sync(0xffffffffu, v, (warp + kTopkWarps - 1) % kTopkWarps);
-            const int tot_e = __shfl_sync(0xffffffffu, v, kTopkWarps - 1);
+            const int before_w = __shfl_sync(0xffffffffu, v, (warp + NW - 1) % NW);
+            const int tot_e = __shfl_sync(0xffffffffu, v, NW - 1);
             const uint32_t bal = __ballot_sync(0xffffffffu, (eq >> e) & 1u);
             const int rank = run + (warp ? before_w : 0) + __popc(bal & lt_mask);
             if (((eq >> e) & 1u) && rank < remaining) keep |= 1u << e;
@@ -307,23 +310,23 @@ __device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, i
     int run = 0;
 #pragma unroll
     for (int e = 0; e < KPT; ++e) {
-        int v = lane < kTopkWarps ? cnt[e][lane] : 0;
+        int v = lane < NW ? cnt[e][lane] : 0;
 #pragma unroll
-        for (int o = 1; o < kTopkWarps; o <<= 1) {
+        for (int o = 1; o < NW; o <<= 1) {
             const int y = __shfl_up_sync(0xffffffffu, v, o);
             if (lane >= o) v += y;
         }
-        const int before_w = __shfl_sync(0xffffffffu, v, (warp + kTopkWarps - 1) % kTopkWarps);
-        const int tot_e = __shfl_sync(0xffffffffu, v, kTopkWarps - 1);
+        const int before_w = __shfl_sync(0xffffffffu, v, (warp + NW - 1) % NW);
+        const int tot_e = __shfl_sync(0xffffffffu, v, NW - 1);
         const uint32_t bal = __ballot_sync(0xffffffffu, (keep >> e) & 1u);
-        if ((keep >> e) & 1u) emit(run + (warp ? before_w : 0) + __popc(bal & lt_mask), e * kTopkThreads + tid);
+        if ((keep >> e) & 1u) emit(run + (warp ? before_w : 0) + __popc(bal & lt_mask), e * NT + tid);
         run += tot_e;
     }
 }
 
 // ---------------------------------------------------------------------------
-// Register-resident variant for requests of at most kTopkThreads * KPT tokens.
-// Thread t holds the keys of tokens j = e * kTopkThreads + t (e < KPT), so the
+// Register-resident variant for requests of at most NT * KPT tokens.
+// Thread t holds the keys of tokens j = e * NT + t (e < KPT), so the
 // loads are coalesced and "round e, warp w, lane l" is index order. The radix
 // select starts below the bits that every key of the request shares (one
 // min/max reduction finds them) and stops as soon as the bin holding the k-th
@@ -332,15 +335,16 @@ __device__ __forceinline__ void select_kept(const uint32_t (&key)[KPT], int N, i
 // three buffers so a buffer is cleared two passes after it was last read.
 // Output positions come from per-(round, warp) ballot counts.
 
-template <int KPT, bool DEFER>
-__global__ void __launch_bounds__(kTopkThreads)
+template <int KPT, bool DEFER, int NT>
+__global__ void __launch_bounds__(NT)
     topk_reg_kernel(float* __restrict__ scores, const int32_t* __restrict__ seq_off,
                     const int32_t* __restrict__ keep_k, float ratio, int32_t* __restrict__ kept_idx,
                     int32_t* __restrict__ out_off, const __grid_constant__ TopkShape sh)
 {
+    constexpr int NW = NT / 32;
     __shared__ uint32_t hist[3][256];
-    __shared__ uint32_t wmin[kTopkWarps], wmax[kTopkWarps];
-    __shared__ int cnt[KPT][kTopkWarps];
+    __shared__ uint32_t wmin[NW], wmax[NW];
+    __shared__ int cnt[KPT][NW];
     __shared__ long long s_base;
 
     const int b = blockIdx.x;
@@ -370,12 +374,13 @@ __global__ void __launch_bounds__(kTopkThreads)
         float sum[KPT];
 #pragma unroll
         for (int e = 0; e < KPT; ++e) sum[e] = 0.f;
-        constexpr int QG = KPT <= 4 ? 16 : (KPT <= 8 ? 4 : 2);  // loads in flight per key, within the registers
+        // loads in flight per key, within the registers (at most 64 registers a thread at 1024 threads)
+        constexpr int QG = NT >= 1024 ? 16 / KPT : (KPT <= 4 ? 16 : (KPT <= 8 ? 4 : 2));
         for (int g0 = 0; g0 < sh.groups; g0 += QG) {
             float v[KPT][QG];
 #pragma unroll
             for (int e = 0; e < KPT; ++e) {
-                const int j = e * kTopkThreads + tid;
+                const int j = e * NT + tid;
 #pragma unroll
                 for (int q = 0; q < QG; ++q)
                     v[e][q] = (j < N && g0 + q < sh.groups)
@@ -389,7 +394,7 @@ __global__ void __launch_bounds__(kTopkThreads)
         }
 #pragma unroll
         for (int e = 0; e < KPT; ++e) {
-            const int j = e * kTopkThreads + tid;
+            const int j = e * NT + tid;
             const float sc = sum[e] / den;
             if (j < N) scores[n0 + j] = sc;
             key[e] = j < N ? order_key(sc) : 0u;
@@ -397,7 +402,7 @@ __global__ void __launch_bounds__(kTopkThreads)
     } else {
 #pragma unroll
         for (int e = 0; e < KPT; ++e) {
-            const int j = e * kTopkThreads + tid;
+            const int j = e * NT + tid;
             key[e] = j < N ? order_key(__ldcg(scores + n0 + j)) : 0u;
         }
     }
@@ -405,7 +410,7 @@ __global__ void __launch_bounds__(kTopkThreads)
     // output base = sum of k over earlier requests
     long long part = 0;
     if (!by_value)
-        for (int bb = tid; bb < b; bb += kTopkThreads) part += keep_count(seq_off, keep_k, ratio, bb);
+        for (int bb = tid; bb < b; bb += NT) part += keep_count(seq_off, keep_k, ratio, bb);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) part += __shfl_down_sync(0xffffffffu, part, o);
     if (tid == 0) s_base = by_value ? (long long)out0_v : 0;
@@ -417,7 +422,7 @@ __global__ void __launch_bounds__(kTopkThreads)
     uint32_t lo_k = 0xFFFFFFFFu, hi_k = 0u;
 #pragma unroll
     for (int e = 0; e < KPT; ++e) {
-        if (e * kTopkThreads + tid < N) {
+        if (e * NT + tid < N) {
             lo_k = min(lo_k, key[e]);
             hi_k = max(hi_k, key[e]);
         }
@@ -428,7 +433,7 @@ __global__ void __launch_bounds__(kTopkThreads)
         wmin[warp] = lo_k;
         wmax[warp] = hi_k;
     }
-    for (int i = tid; i < 2 * 256; i += kTopkThreads) (&hist[0][0])[i] = 0u;
+    for (int i = tid; i < 2 * 256; i += NT) (&hist[0][0])[i] = 0u;
     __syncthreads();
     const long long out_base = s_base;
     if (tid == 0) {
@@ -438,17 +443,12 @@ __global__ void __launch_bounds__(kTopkThreads)
     if (k <= 0 || N <= 0) return;
     int32_t* dst = kept_idx + out_base;
     if (k >= N) {
-        for (int j = tid; j < N; j += kTopkThreads) dst[j] = n0 + j;
+        for (int j = tid; j < N; j += NT) dst[j] = n0 + j;
         return;
     }
-    lo_k = wmin[0];
-    hi_k = wmax[0];
-#pragma unroll
-    for (int w = 1; w < kTopkWarps; ++w) {
-        lo_k = min(lo_k, wmin[w]);
-        hi_k = max(hi_k, wmax[w]);
-    }
-    select_kept<KPT>(key, N, k, lo_k, hi_k, hist, cnt, [&](int pos, int j) { dst[pos] = n0 + j; });
+    lo_k = __reduce_min_sync(0xffffffffu, lane < NW ? wmin[lane] : 0xFFFFFFFFu);
+    hi_k = __reduce_max_sync(0xffffffffu, lane < NW ? wmax[lane] : 0u);
+    select_kept<KPT, NT>(key, N, k, lo_k, hi_k, hist, cnt, [&](int pos, int j) { dst[pos] = n0 + j; });
 }
 
 }  // namespace
@@ -475,18 +475,24 @@ cudaError_t launch_topk(int batch, float* scores, const int32_t* seq_off, const 
                         cudaStream_t stream)
 {
     if (batch <= 0) return cudaSuccess;
-    // requests up to 16 keys per thread: registers only
-    if (max_n <= 16 * kTopkThreads) {
-        const bool defer = shape.partials != nullptr && shape.n == batch;
-        auto kern = defer ? (max_n <= 2 * kTopkThreads   ? topk_reg_kernel<2, true>
-                             : max_n <= 4 * kTopkThreads ? topk_reg_kernel<4, true>
-                             : max_n <= 8 * kTopkThreads ? topk_reg_kernel<8, true>
-                                                         : topk_reg_kernel<16, true>)
-                          : (max_n <= 2 * kTopkThreads   ? topk_reg_kernel<2, false>
-                             : max_n <= 4 * kTopkThreads ? topk_reg_kernel<4, false>
-                             : max_n <= 8 * kTopkThreads ? topk_reg_kernel<8, false>
-                                                         : topk_reg_kernel<16, false>);
+    // registers only: 512 threads up to 2048 tokens, 1024 threads up to 8192
+    // (measured on GB300: the wider CTA halves each thread's chain of loads,
+    // passes and ranks on long requests, and costs more than it saves on short ones)
+    const bool defer = shape.partials != nullptr && shape.n == batch;
+    if (max_n <= 4 * kTopkThreads) {
+        auto kern = defer ? (max_n <= 2 * kTopkThreads ? topk_reg_kernel<2, true, kTopkThreads>
+                                                       : topk_reg_kernel<4, true, kTopkThreads>)
+                          : (max_n <= 2 * kTopkThreads ? topk_reg_kernel<2, false, kTopkThreads>
+                                                       : topk_reg_kernel<4, false, kTopkThreads>);
         return launch_pdl(kern, (unsigned)batch, kTopkThreads, 0, stream, scores, seq_off, keep_k, keep_ratio,
+                          kept_idx, out_off, shape);
+    }
+    if (max_n <= 8 * kTopkWideThreads) {
+        auto kern = defer ? (max_n <= 4 * kTopkWideThreads ? topk_reg_kernel<4, true, kTopkWideThreads>
+                                                           : topk_reg_kernel<8, true, kTopkWideThreads>)
+                          : (max_n <= 4 * kTopkWideThreads ? topk_reg_kernel<4, false, kTopkWideThreads>
+                                                           : topk_reg_kernel<8, false, kTopkWideThreads>);
+        return launch_pdl(kern, (unsigned)batch, kTopkWideThreads, 0, stream, scores, seq_off, keep_k, keep_ratio,
                           kept_idx, out_off, shape);
     }
     const int keys = max_n < kTopkSmemKeys ? max_n : kTopkSmemKeys;
