@@ -341,18 +341,24 @@ def run_ours(args):
         if rc != 0:
             raise select.LitevlmError(rc, L.litevlm_select_last_error(h).decode())
 
-    def step(q, k, so_d, to_d, hidden_srcs=None, s_ptr=None):
-        """One step: scores and top-k (one call: the top-k kernel adds the
-        head-group partials), then the gather; returns the kernels launched."""
-        st_ = sp if s_ptr is None else s_ptr
+    def select_call(q, k, so_d, to_d, s_ptr, kept_t, off_t):
+        """Scores and top-k in one call (the top-k kernel adds the head-group
+        partials); returns the kernels launched."""
         call(L.litevlm_select_score_topk(h, w.batch, q.data_ptr(), to_d.data_ptr(), c_to_h, k.data_ptr(),
                                          so_d.data_ptr(), c_so_h, xd["q_scale"], xd["k_scale"], scores.data_ptr(),
-                                         c_kk_d, c_kk_h, ratio, kept.data_ptr(), off_d.data_ptr(),
-                                         off_h.ctypes.data, st_))
-        n = L.litevlm_select_last_launches(h)
-        call(L.litevlm_select_compact(h, total_kept, kept.data_ptr(), w.total_vis, n_t,
-                                      hidden_srcs if hidden_srcs is not None else c_src, c_dst, c_rb, st_))
-        return n + L.litevlm_select_last_launches(h)
+                                         c_kk_d, c_kk_h, ratio, kept_t.data_ptr(), off_t.data_ptr(),
+                                         off_h.ctypes.data, s_ptr))
+        return L.litevlm_select_last_launches(h)
+
+    def gather_call(kept_t, srcs, s_ptr):
+        call(L.litevlm_select_compact(h, total_kept, kept_t.data_ptr(), w.total_vis, n_t, srcs, c_dst, c_rb, s_ptr))
+        return L.litevlm_select_last_launches(h)
+
+    def step(q, k, so_d, to_d, hidden_srcs=None, s_ptr=None):
+        """One step: scores and top-k, then the gather; returns the kernels launched."""
+        st_ = sp if s_ptr is None else s_ptr
+        n = select_call(q, k, so_d, to_d, st_, kept, off_d)
+        return n + gather_call(kept, hidden_srcs if hidden_srcs is not None else c_src, st_)
 
     q, k, so_d, to_d = xd["q"], xd["k"], xd["seq_offsets"], xd["text_offsets"]
     launches_per_step = 0
@@ -460,10 +466,11 @@ def run_ours(args):
            "project": run_project(w, xd, sel, dev, stream, steps, pk)}
 
     # end to end through the public API with host buffers
-    e2e = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel)
-    e2e["copy_all_inputs"] = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel,
+    calls = (select_call, gather_call)
+    e2e = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel)
+    e2e["copy_all_inputs"] = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel,
                                      gather_from_host=False)
-    e2e["eager"] = run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, graph=False)
+    e2e["eager"] = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel, graph=False)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -682,14 +689,17 @@ def run_views(w, sel, dev, stream, steps):
             "mean_views_selected": sel_views / max(1, w.batch)}
 
 
-def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, gather_from_host=True, graph=True):
+def run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel, gather_from_host=True, graph=True):
     """Host buffers in, selection out, through the C-ABI, all inside the timed
     region: every step copies q, K and the offsets (packed in one pinned host
     buffer) to the device, runs the three calls, and reads the kept indices and
     offsets back into pinned host memory. Inputs are double-buffered on the
     device and copied on a second stream, so the copy of step i + 1 overlaps the
     kernels of step i (the way a serving loop would run it); each step's kernels
-    wait for its own copy.
+    wait for its own copy. The gather of step i runs on a third stream, so it
+    overlaps the scores and top-k of step i + 1; the kept indices and offsets
+    are double-buffered for that, and a step's input buffer is reused only
+    after both its select and its gather are done.
 
     The gathered tensors other than K (hidden states, V) stay in pinned host
     memory and the gather reads only their kept rows through the device view
@@ -729,26 +739,37 @@ def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, gather
     res_h = torch.empty(kept.numel() + off_d.numel(), dtype=torch.int32).pin_memory()
     nk = kept.numel()
     steps = args.e2e_steps if args.e2e_steps is not None else max(3, min(200, (args.steps or DEFAULTS[w.name][0])))
+    select_call, gather_call = calls
+    kept2 = [kept, torch.empty_like(kept)]
+    off2 = [off_d, torch.empty_like(off_d)]
     copy_stream = torch.cuda.Stream(device=dev)
+    gather_stream = torch.cuda.Stream(device=dev)
     copied = [torch.cuda.Event() for _ in range(2)]
-    used = [torch.cuda.Event() for _ in range(2)]
+    selected = [torch.cuda.Event() for _ in range(2)]
+    gathered = [torch.cuda.Event() for _ in range(2)]
     h2d = tot + sum(total_kept * (sizes[n] // xd[n].shape[0]) for n in host_gather)
     d2h = res_h.numel() * 4
 
     def one(i, st, wait_used=True):
         sl = i & 1
         with torch.cuda.stream(copy_stream):
-            if wait_used:
-                copy_stream.wait_event(used[sl])  # the kernels of step i - 2 are done with this buffer
+            if wait_used:  # the select and the gather of step i - 2 are done with this buffer
+                copy_stream.wait_event(selected[sl])
+                copy_stream.wait_event(gathered[sl])
             bufs[sl].copy_(host, non_blocking=True)
             copied[sl].record(copy_stream)
         st.wait_event(copied[sl])
+        if wait_used:
+            st.wait_event(gathered[sl])  # the gather of step i - 2 has read kept2[sl]
         d = dv[sl]
-        step(d["q"], d["k"], d["seq_offsets"], d["text_offsets"], c_srcs[sl], st.cuda_stream)
-        used[sl].record(st)
+        select_call(d["q"], d["k"], d["seq_offsets"], d["text_offsets"], st.cuda_stream, kept2[sl], off2[sl])
+        selected[sl].record(st)
         with torch.cuda.stream(st):
-            res_h[:nk].copy_(kept, non_blocking=True)
-            res_h[nk:].copy_(off_d, non_blocking=True)
+            res_h[:nk].copy_(kept2[sl], non_blocking=True)
+            res_h[nk:].copy_(off2[sl], non_blocking=True)
+        gather_stream.wait_event(selected[sl])
+        gather_call(kept2[sl], c_srcs[sl], gather_stream.cuda_stream)
+        gathered[sl].record(gather_stream)
 
     for i in range(4):
         one(i, stream)
@@ -762,11 +783,13 @@ def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, gather
         with torch.cuda.graph(g, stream=cap, capture_error_mode="relaxed"):
             fork = torch.cuda.Event()
             fork.record(cap)
-            copy_stream.wait_event(fork)  # the copy stream joins the capture
+            copy_stream.wait_event(fork)  # the copy and gather streams join the capture
+            gather_stream.wait_event(fork)
             for i in range(per_graph):
                 # steps 0 and 1 of a replay follow the previous replay in stream order
                 one(i, cap, wait_used=i >= 2)
-            cap.wait_stream(copy_stream)  # and leaves it
+            cap.wait_stream(copy_stream)  # and leave it
+            cap.wait_stream(gather_stream)
         torch.cuda.synchronize()
         steps = max(per_graph, (steps + per_graph - 1) // per_graph * per_graph)
         g.replay()
@@ -774,6 +797,7 @@ def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, gather
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     copy_stream.wait_event(e0)
+    gather_stream.wait_event(e0)
     if g is not None:
         with torch.cuda.stream(stream):
             for _ in range(steps // per_graph):
@@ -782,11 +806,13 @@ def run_e2e(args, w, xd, step, dev, stream, kept, off_d, total_kept, sel, gather
         for i in range(steps):
             one(i, stream)
     stream.wait_stream(copy_stream)
+    stream.wait_stream(gather_stream)
     e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
     if host_gather:
         api = ("litevlm_select_score_topk + compact" + (" (8 steps captured into a CUDA graph, replayed)" if g else "")
+               + "; the gather of step i overlaps the select of step i + 1 (own stream)"
                + "; each step copies q, K and the offsets from one pinned host "
                "buffer into one of two device buffers on a copy stream; the gather reads the kept rows of "
                + ", ".join(host_gather) + " straight from pinned host memory (litevlm_select_host_view); "
