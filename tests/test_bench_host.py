@@ -54,3 +54,23 @@ def test_workload_bounds_match_their_intensity():
         r = bench.stage_rooflines(alg, {"score": 1.0, "topk": 1.0, "compact": 1.0}, 3.0, PK, "bf16")
         assert r["score"]["bound"] == bound
         assert r["topk"]["bound"] == "hbm" and r["compact"]["bound"] == "hbm"
+
+
+@pytest.mark.parametrize("ratio,k", [(0.1, 345), (0.2, 691), (0.3, 1036), (0.5, 1728)])
+def test_sweep_keep_counts_follow_the_floor_reading(ratio, k):
+    # k = floor((double)(float)r * N) with N = 3456: 0.1f * 3456 = 345.6..., 0.2f -> 691.2..., 0.3f -> 1036.8...
+    class A:
+        workload, batch = "sweep", None
+    A.ratio = ratio
+    w = bench.workload_for(A())
+    alg = bench.algorithmic(w)
+    assert alg["kept"] == [k] * 128
+    assert sum(alg["kept"]) == 128 * k
+
+
+def test_batch_option_takes_the_first_requests():
+    class A:
+        workload, ratio, batch = "fp8_ragged", None, 5
+    w = bench.workload_for(A())
+    full = inputs.workload("fp8_ragged")
+    assert w.batch == 5 and list(w.n_vis) == list(full.n_vis[:5]) and list(w.n_txt) == list(full.n_txt[:5])
