@@ -2,15 +2,17 @@
 """Benchmark of the token-selection path (score -> top-k -> gather) on GB300.
 
 One step = one pass of the whole path over one batch of synthetic input:
-litevlm_select_score, litevlm_select_topk and litevlm_select_compact through
-the C-ABI, inputs resident in HBM. Prints ONE JSON line (rank 0).
+litevlm_select_score_topk and litevlm_select_compact through the C-ABI, inputs
+resident in HBM. Prints ONE JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--ratio R]
   python bench.py --impl reference ...   # the CPU oracle, timed on the host cores
 
-Workloads (paper_2506_07416_gb300/inputs.py): single (default; 1 request of
-6 views x 256 = 1536 visual + 64 text tokens, 16 heads x 128, keep 30%),
-highres, fp8_ragged, sweep (128 requests; --ratio 0.1/0.2/0.3/0.5).
+Workloads (paper_2506_07416_gb300/inputs.py): sweep (default; 128 requests x
+(6 views x 576 = 3456 visual + 64 text tokens), 32 heads x 128, hidden 4096,
+keep 30%; --ratio 0.1/0.2/0.3/0.5), single, highres, fp8_ragged. The default
+run also measures the other three workloads and reports each one's full record
+under "workloads" (--workloads none skips them).
 Multi-GPU: one process per GPU (torchrun), each rank runs its own batch
 (weak scaling, no collective on the data path); time = max over ranks.
 """
@@ -35,48 +37,73 @@ sys.path.insert(0, ROOT)
 
 METRIC = "visual tokens scored+selected per sec (M/s), % of HBM/tensor roofline, p50 µs"
 UNIT = "M visual tokens/s"
-DEFAULTS = {"single": (3000, 50), "highres": (2000, 30), "fp8_ragged": (200, 10), "sweep": (20, 3)}
+# (timed steps, warm-up steps) of the headline run; the sub-records of the other workloads take SUB_STEPS
+DEFAULTS = {"single": (3000, 50), "highres": (2000, 30), "fp8_ragged": (200, 10), "sweep": (20, 5)}
+SUB_STEPS = {"single": (500, 20), "highres": (300, 10), "fp8_ragged": (60, 5), "sweep": (10, 3)}
 KERNEL_SOURCES = ["paper_2506_07416_gb300/csrc/score_tc.cu", "paper_2506_07416_gb300/csrc/score_res.cu",
                   "paper_2506_07416_gb300/csrc/pipe.cuh", "paper_2506_07416_gb300/csrc/ptx.cuh",
                   "paper_2506_07416_gb300/csrc/score.h"]
+WORKLOADS = ["sweep", "single", "highres", "fp8_ragged"]
 
 
-def parse_args():
+def parse_args(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=None)
     ap.add_argument("--warmup", type=int, default=None)
-    ap.add_argument("--workload", default="single", choices=["single", "highres", "fp8_ragged", "sweep"])
+    ap.add_argument("--workload", default="sweep", choices=WORKLOADS)
     ap.add_argument("--ratio", type=float, default=None, help="keep ratio override (sweep: 0.1/0.2/0.3/0.5)")
     ap.add_argument("--batch", type=int, default=None, help="use only the first B requests (profiling)")
+    ap.add_argument("--workloads", default="auto",
+                    help="other workloads measured after the headline one, comma-separated, or 'none'; "
+                         "auto: the three others when the headline is the default sweep on one GPU")
     ap.add_argument("--score-kernel", default="auto", choices=["auto", "reread", "resident", "resident_1buf",
                                                                      "resident_2buf"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="bounded CPU work for the oracle baseline")
+    ap.add_argument("--no-next", action="store_true", help="skip the next-row measurements (splice, ...)")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="bounded CPU work for the oracle baseline")
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--measure-fp8-peak", action="store_true",
                     help="time a cuBLASLt e4m3 GEMM (torch._scaled_mm) and print its TFLOP/s, nothing else")
-    return ap.parse_args()
+    return ap.parse_args(argv)
+
+
+def sub_workloads(args, world: int):
+    """The workloads measured after the headline one (full records under "workloads")."""
+    if args.workloads == "none":
+        return []
+    if args.workloads == "auto":
+        if world > 1 or args.workload != "sweep" or args.batch is not None:
+            return []
+        return [n for n in WORKLOADS if n != args.workload]
+    names = [n.strip() for n in args.workloads.split(",") if n.strip()]
+    for n in names:
+        if n not in WORKLOADS:
+            raise SystemExit(f"unknown workload {n!r}")
+    return [n for n in names if n != args.workload]
 
 
 # ----------------------------------------------------------------------------- work accounting
 
-def workload_for(args):
+def workload_for(args, name=None):
     from paper_2506_07416_gb300 import inputs
-    w = inputs.workload(args.workload)
-    if args.ratio is not None:
+    w = inputs.workload(name or args.workload)
+    if name is None and args.ratio is not None:
         from dataclasses import replace
         w = replace(w, keep_ratio=args.ratio, keep_k=None)
-    if args.batch is not None and args.batch < w.batch:
+    if name is None and args.batch is not None and args.batch < w.batch:
         w = inputs.sub_batch(w, list(range(args.batch)))
     return w
 
 
 def algorithmic(w):
-    """Bytes and FLOPs the method itself moves / computes per step (no re-reads)."""
+    """Bytes and FLOPs the method itself moves / computes per step (no re-reads).
+    The kept counts come from the library's own keep-count call."""
+    from paper_2506_07416_gb300 import select
     e = 2 if w.dtype == "bf16" else 1
-    ks = w.keep_counts()
+    off = select.keep_offsets(w.seq_offsets(), w.keep_k, float(w.keep_ratio or 0.0))
+    ks = [int(x) for x in np.diff(off)]
     rb = w.row_bytes()
     row_total = sum(rb[n] for n in w.gather)
     score_bytes = sum(n * w.hkv * w.head_dim * e + t * w.hq * w.head_dim * e + 4 * n for n, t in zip(w.n_vis, w.n_txt))
@@ -147,6 +174,14 @@ def committed_traffic(workload):
     return ent.get("dram_bytes_per_launch")
 
 
+def config_of(w):
+    """The workload as the JSON line names it (the same for both arms)."""
+    return {"workload": f"{w.name}: {w.description}", "batch": w.batch, "visual_tokens": w.total_vis,
+            "text_tokens": w.total_txt, "q_heads": w.hq, "kv_heads": w.hkv, "head_dim": w.head_dim,
+            "keep": (f"ratio {w.keep_ratio}" if w.keep_k is None else "keep_k per request"),
+            "gather": list(w.gather)}
+
+
 # ----------------------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -202,6 +237,14 @@ class ClockSampler:
 
 # ----------------------------------------------------------------------------- CPU oracle
 
+def host_cores() -> int:
+    """Host cores this process may run on."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        return os.cpu_count() or 1
+
+
 def oracle_sample(w):
     """A bounded sample of the workload for the CPU oracle: whole requests."""
     from paper_2506_07416_gb300 import inputs
@@ -211,26 +254,38 @@ def oracle_sample(w):
     return inputs.sub_batch(w, reqs), reqs
 
 
-def time_oracle(w, seconds: float, max_runs: int = 1000):
-    """Runs the oracle (score + top-k + gather) on a bounded sample until about
-    `seconds` of CPU time; returns (M tokens/s, description, runs)."""
+def _oracle_runs(ws, x, seconds: float, threads: int, max_runs: int = 1000):
     import oracle
-    from paper_2506_07416_gb300 import inputs
-    ws, reqs = oracle_sample(w)
-    x = inputs.make_numpy(ws)
-    kk = ws.keep_k
-    ratio = ws.keep_ratio or 0.0
     runs, t0 = 0, time.perf_counter()
     while True:
-        oracle.select(x, ws.hq, ws.hkv, ws.head_dim, ws.dtype, keep_k=kk, keep_ratio=ratio, gather=ws.gather)
+        oracle.select(x, ws.hq, ws.hkv, ws.head_dim, ws.dtype, keep_k=ws.keep_k, keep_ratio=ws.keep_ratio or 0.0,
+                      gather=ws.gather, threads=threads)
         runs += 1
         el = time.perf_counter() - t0
         if el >= seconds or runs >= max_runs:
-            break
-    value = ws.total_vis * runs / el / 1e6
-    desc = (f"{runs} run(s) of the whole path on request(s) {reqs} ({ws.total_vis} visual tokens each run), "
-            f"{el:.1f} s, single thread")
-    return value, desc, el, runs
+            return runs, el
+
+
+def time_oracle(w, seconds: float):
+    """Runs the oracle (score + top-k + gather) on a bounded sample, on all the
+    host cores this process may use (the threaded score, bit-identical to the
+    serial one) for about seconds / 2, and on one thread for about seconds / 2.
+    Returns the cpu_baseline record (value = the all-cores rate)."""
+    from paper_2506_07416_gb300 import inputs
+    ws, reqs = oracle_sample(w)
+    x = inputs.make_numpy(ws)
+    cores = host_cores()
+    runs_n, el_n = _oracle_runs(ws, x, seconds / 2, cores)
+    runs_1, el_1 = _oracle_runs(ws, x, seconds / 2, 1)
+    v_n = ws.total_vis * runs_n / el_n / 1e6
+    v_1 = ws.total_vis * runs_1 / el_1 / 1e6
+    desc = (f"the whole path (fp64 scores, full-sort top-k, row copies) on request(s) {reqs} of the workload "
+            f"({ws.total_vis} visual tokens per run): {runs_n} run(s) in {el_n:.1f} s on {cores} threads "
+            f"(scores threaded over (head, query) rows, then over tokens, in the serial summation order), "
+            f"{runs_1} run(s) in {el_1:.1f} s on one thread")
+    return {"value": v_n, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+            "single_thread": {"value": v_1, "unit": UNIT, "cores": 1, "runs": runs_1, "seconds": el_1},
+            "all_cores": {"value": v_n, "unit": UNIT, "cores": cores, "runs": runs_n, "seconds": el_n}}
 
 
 def whole_job(local_total_ms: float, tokens_per_rank: int, world: int, device):
@@ -253,6 +308,8 @@ def rank_seed(base_seed: int, rank: int) -> int:
 
 
 def run_reference(args):
+    """The reference arm: the CPU oracle as it stands, on the host cores, each
+    step the whole path on a bounded sample of the workload (rank 0 only)."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
@@ -263,24 +320,29 @@ def run_reference(args):
     from paper_2506_07416_gb300 import inputs
     ws, reqs = oracle_sample(w)
     x = inputs.make_numpy(ws)
-    for _ in range(warm):
+    cores = host_cores()
+
+    def one():
         oracle.select(x, ws.hq, ws.hkv, ws.head_dim, ws.dtype, keep_k=ws.keep_k, keep_ratio=ws.keep_ratio or 0.0,
-                      gather=ws.gather)
+                      gather=ws.gather, threads=cores)
+
+    for _ in range(warm):
+        one()
     times = []
     for _ in range(steps):
         t0 = time.perf_counter()
-        oracle.select(x, ws.hq, ws.hkv, ws.head_dim, ws.dtype, keep_k=ws.keep_k, keep_ratio=ws.keep_ratio or 0.0,
-                      gather=ws.gather)
+        one()
         times.append(time.perf_counter() - t0)
     tot = sum(times)
     value = ws.total_vis * steps / tot / 1e6
-    desc = f"each step: the whole path on request(s) {reqs} of the workload ({ws.total_vis} visual tokens)"
+    desc = (f"each step: the whole path on request(s) {reqs} of the workload ({ws.total_vis} visual tokens), "
+            f"scores threaded over {cores} host cores")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": steps, "warmup": warm, "ms_per_step": tot / steps * 1e3,
             "p50_us": statistics.median(times) * 1e6, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name + ": " + w.description, "sample_requests": reqs},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc},
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config_of(w),
+            "sample_requests": reqs,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
     print(json.dumps(line), flush=True)
@@ -293,8 +355,6 @@ def run_ours(args):
     import torch
     import torch.distributed as dist
 
-    from paper_2506_07416_gb300 import inputs, select
-
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
@@ -302,13 +362,56 @@ def run_ours(args):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    stream = torch.cuda.current_stream()
-    sp = stream.cuda_stream
 
     w = workload_for(args)
     steps_d, warm_d = DEFAULTS[w.name]
     steps = args.steps if args.steps is not None else steps_d
     warm = args.warmup if args.warmup is not None else warm_d
+    rec = measure(args, w, steps, warm, dev, rank, world, full=True)
+
+    subs = {}
+    for name in sub_workloads(args, world):
+        ws = workload_for(args, name)
+        s_steps, s_warm = SUB_STEPS[name]
+        r = measure(args, ws, s_steps, max(3, s_warm), dev, rank, world, full=False)
+        subs[name] = {k: r[k] for k in ("value", "unit", "steps", "warmup", "ms_per_step", "p50_us", "p10_us",
+                                        "p90_us", "warm", "dtype", "config", "score_launch", "stages_p50_us",
+                                        "stages_roofline", "roofline", "e2e", "gpu_launches", "clocks", "l2")}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = time_oracle(w, args.cpu_seconds)
+
+    line = {"metric": METRIC, "value": rec["value"], "unit": UNIT, "n_gpus": world, "steps": steps, "warmup": warm,
+            "ms_per_step": rec["ms_per_step"], "p50_us": rec["p50_us"], "p10_us": rec["p10_us"],
+            "p90_us": rec["p90_us"], "warm": rec["warm"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": rec["dtype"],
+            "data": "synthetic (seeded; shapes of the paper's multi-camera workloads)",
+            "config": rec["config"], "l2": rec["l2"],
+            "parallelism": f"replicas x{world}, one batch per GPU, no collective",
+            "score_launch": rec["score_launch"], "stages_p50_us": rec["stages_p50_us"],
+            "stages_roofline": rec["stages_roofline"], "roofline": rec["roofline"], "cpu_baseline": cpu,
+            "e2e": rec["e2e"], "next": rec.get("next"), "workloads": subs or None,
+            "gpu_launches": rec["gpu_launches"], "clocks": rec["clocks"], "wall_s": rec["wall_s"]}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def measure(args, w, steps, warm_steps, dev, rank, world, full):
+    """Times `steps` steps of the path on workload w (after `warm_steps`
+    untimed ones) and returns the record: the whole-job rate, step percentiles,
+    stage times and rooflines, the clocks seen, and the end-to-end figure
+    (full=True: also the e2e variants and the next-row measurements)."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2506_07416_gb300 import inputs, select
+
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
     alg = algorithmic(w)
 
     xd = inputs.make_torch(w, dev, seed=rank_seed(w.seed, rank))
@@ -362,7 +465,7 @@ def run_ours(args):
 
     q, k, so_d, to_d = xd["q"], xd["k"], xd["seq_offsets"], xd["text_offsets"]
     launches_per_step = 0
-    for _ in range(warm):
+    for _ in range(warm_steps):
         launches_per_step = step(q, k, so_d, to_d)
     sel.check_device()
 
@@ -379,7 +482,7 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    clk = ClockSampler(local)
+    clk = ClockSampler(dev.index or 0)
     clk.start()
     time.sleep(0.15)
     wall0 = time.perf_counter()
@@ -413,7 +516,7 @@ def run_ours(args):
     # cold ones when the timed steps flush L2. A GPU spin queued first lets the
     # host enqueue every step before the GPU reaches them, so the events
     # bracket GPU work only.
-    warm = None
+    warm_stats = None
     if flush is not None:
         n_warm = min(steps, 500)
         ev_warm = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -427,9 +530,9 @@ def run_ours(args):
             e1.record(stream)
         torch.cuda.synchronize()
         wt = np.array([a.elapsed_time(b) for a, b in ev_warm]) * 1e3
-        warm = {"p10_us": float(np.percentile(wt, 10)), "p50_us": float(np.median(wt)),
-                "p90_us": float(np.percentile(wt, 90)), "steps": n_warm,
-                "timing": "the same step back to back without the L2 flush, events at step boundaries"}
+        warm_stats = {"p10_us": float(np.percentile(wt, 10)), "p50_us": float(np.median(wt)),
+                      "p90_us": float(np.percentile(wt, 90)), "steps": n_warm,
+                      "timing": "the same step back to back without the L2 flush, events at step boundaries"}
     clocks = clk.stop()
     if world > 1:
         dist.barrier()
@@ -458,55 +561,45 @@ def run_ours(args):
                 "peak_source": pk["source"] + " (burst cuBLAS bf16)",
                 "duration_us": score_us, "duration_source": "mean CUDA-event time of the score call, stage pass"}
 
-    # prefill splice (a next-step row, timed on its own after the step): 32 system rows and
-    # the text rows of every request around its kept visual rows, hidden-size rows
-    nxt = {"splice": run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk),
-           "full_keys": run_full_keys(w, xd, sel, dev, stream, steps, flush, pk),
-           "views": run_views(w, sel, dev, stream, steps),
-           "project": run_project(w, xd, sel, dev, stream, steps, pk)}
+    nxt = None
+    if full and not args.no_next:
+        # next-step rows, each timed on its own after the step: prefill splice
+        # (32 system rows and the text rows of every request around its kept
+        # visual rows), full-key scores, view gating, layer-0 projection
+        nxt = {"splice": run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk),
+               "full_keys": run_full_keys(w, xd, sel, dev, stream, steps, flush, pk),
+               "views": run_views(w, sel, dev, stream, steps),
+               "project": run_project(w, xd, sel, dev, stream, steps, pk)}
 
     # end to end through the public API with host buffers
     calls = (select_call, gather_call)
     e2e = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel)
-    e2e["copy_all_inputs"] = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel,
-                                     gather_from_host=False)
-    e2e["eager"] = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel, graph=False)
-
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, desc, el, runs = time_oracle(w, args.cpu_seconds)
-        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc}
+    if full:
+        e2e["copy_all_inputs"] = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel,
+                                         gather_from_host=False)
+        e2e["eager"] = run_e2e(args, w, xd, calls, dev, stream, kept, off_d, total_kept, sel, graph=False)
 
     stage_us = {n: float(np.median(st[:, i]) * 1e3) for i, n in enumerate(("score", "topk", "compact"))}
     stage_us["timing"] = ("a second pass with CUDA events between the separate calls (score with its own "
                           "head-group fold, top-k, gather); the timed steps use the one-call score + top-k, "
                           "whose top-k kernel adds the head-group partials, with events at step boundaries only")
-    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps, "warmup": warm,
-            "ms_per_step": total_ms / steps, "p50_us": float(np.median(per_step_ms) * 1e3),
-            "p10_us": float(np.percentile(per_step_ms, 10) * 1e3), "p90_us": float(np.percentile(per_step_ms, 90) * 1e3),
-            "warm": warm,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "bf16" if w.dtype == "bf16" else "e4m3", "data": "synthetic",
-            "config": {"workload": f"{w.name}: {w.description}", "batch": w.batch, "visual_tokens": w.total_vis,
-                       "text_tokens": w.total_txt, "q_heads": w.hq, "kv_heads": w.hkv, "head_dim": w.head_dim,
-                       "keep": (f"ratio {w.keep_ratio}" if w.keep_k is None else "keep_k per request"),
-                       "kept_tokens": total_kept, "gather": list(w.gather),
-                       "l2": ("flushed between timed steps (write of %d MB)" % (flush.numel() * 4 >> 20))
-                       if flush is not None else "inputs larger than L2, no flush",
-                       "parallelism": f"replicas x{world}, one batch per GPU, no collective",
-                       "score_launch": {"kernel": select.KERNELS.get(plan[0]), "cluster": plan[1],
-                                        "tiles_per_cta": plan[2], "head_groups": plan[3]}},
-            "stages_p50_us": stage_us,
-            "stages_roofline": stage_rooflines(alg, stage_us, float(np.median(per_step_ms) * 1e3), pk, w.dtype),
-            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "next": nxt,
-            "gpu_launches": launches_per_step * steps, "clocks": clocks,
-            "wall_s": wall}
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+    rec = {"value": value, "unit": UNIT, "steps": steps, "warmup": warm_steps, "ms_per_step": total_ms / steps,
+           "p50_us": float(np.median(per_step_ms) * 1e3), "p10_us": float(np.percentile(per_step_ms, 10) * 1e3),
+           "p90_us": float(np.percentile(per_step_ms, 90) * 1e3), "warm": warm_stats,
+           "dtype": "bf16" if w.dtype == "bf16" else "e4m3", "config": config_of(w),
+           "kept_tokens": total_kept,
+           "l2": ("flushed between timed steps (write of %d MB)" % (flush.numel() * 4 >> 20))
+           if flush is not None else "inputs larger than L2, no flush",
+           "score_launch": {"kernel": select.KERNELS.get(plan[0]), "cluster": plan[1], "tiles_per_cta": plan[2],
+                            "head_groups": plan[3]},
+           "stages_p50_us": stage_us,
+           "stages_roofline": stage_rooflines(alg, stage_us, float(np.median(per_step_ms) * 1e3), pk, w.dtype),
+           "roofline": roof, "e2e": e2e, "next": nxt, "gpu_launches": launches_per_step * steps,
+           "clocks": clocks, "wall_s": wall}
     sel.close()
-    return 0
+    del xd, dsts, scores, kept, flush
+    torch.cuda.empty_cache()
+    return rec
 
 
 def run_splice(w, xd, sel, kept, off_d, off_h, dev, stream, steps, flush, pk):

@@ -281,6 +281,26 @@ litevlm_status_t litevlm_select_topk(litevlm_select_t handle, int32_t batch, con
                                      litevlm_stream_t stream);
 
 /*
+ * Kept-token counts of a batch, on the host, before any device work (Results
+ * section, "Visual Token Compression": the ratio r of visual tokens kept;
+ * Table 1's token counts follow from rounding r * N_b down). The same numbers
+ * litevlm_select_topk writes to out_offsets_h, so a caller can size kept_idx
+ * and the gather outputs before it calls topk.
+ *   batch          >= 0 (not limited by any handle)
+ *   seq_offsets_h  host int32 [batch+1] prefix of N_b
+ *   keep_k_h       host int32 [batch] or NULL; NULL selects keep_ratio,
+ *                  k_b = floor((double)keep_ratio * N_b)
+ *   keep_ratio     0 <= r <= 1, used only when keep_k_h is NULL
+ *   out_offsets_h  host int32 [batch+1]: out_offsets_h[b+1] = out_offsets_h[b] + k_b
+ * No handle, no CUDA call, nothing enqueued; out_offsets_h is written only when
+ * the call succeeds. Errors (message from litevlm_select_last_error(NULL)):
+ * INVALID_ARG for a NULL pointer, bad offsets, k_b outside [0, N_b] or r
+ * outside [0, 1].
+ */
+litevlm_status_t litevlm_select_keep_offsets(int32_t batch, const int32_t* seq_offsets_h, const int32_t* keep_k_h,
+                                             float keep_ratio, int32_t* out_offsets_h);
+
+/*
  * Gather of the kept rows into the compacted sequence (the LLM prefill input;
  * Design section: the module shortens the LLM input sequence; Speculative
  * Decoding Head: K/V rows feed the KV cache).
@@ -399,6 +419,19 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t handle, int32_t batc
 litevlm_status_t litevlm_select_check_device(litevlm_select_t handle, litevlm_stream_t stream);
 
 /*
+ * Budget of every device-side wait of the kernels this handle launches, in SM
+ * clock cycles (default 4e9, about 2 s at 2 GHz; 0 restores it). A wait that
+ * runs past it sets LITEVLM_ERR_TIMEOUT in the handle's error word, its kernel
+ * drains the copies and contractions it issued, frees its tensor memory and
+ * returns; litevlm_select_check_device then reports TIMEOUT, clears the word
+ * and re-arms the fold tickets, and the handle stays usable. No counterpart in
+ * the paper: a failure-detection control, used by the tests to make a wait run
+ * out on purpose. The results of a call that timed out are not valid.
+ * Errors: INVALID_ARG for a NULL handle or cycles < 0.
+ */
+litevlm_status_t litevlm_select_set_wait_budget(litevlm_select_t handle, int64_t cycles);
+
+/*
  * litevlm_select_score without a handle and without allocating anything.
  * The paper has no counterpart: this is an integration entry point.
  *
@@ -421,7 +454,9 @@ litevlm_status_t litevlm_select_check_device(litevlm_select_t handle, litevlm_st
  *     groups, G * total_visual <= 1048576.
  *   - A call beyond either limit returns LITEVLM_ERR_WORKSPACE and enqueues
  *     nothing. Limit 1 is checked before any CUDA call.
- *   - Each call clears the tickets it uses with cudaMemsetAsync on `stream`.
+ *   - A call that splits the heads clears the tickets it uses with
+ *     cudaMemsetAsync on `stream`, after every host-side check (a rejected
+ *     call enqueues nothing).
  * Calls that overlap on one device (other streams, other host threads) share
  * this scratch and race. Serialise them.
  *

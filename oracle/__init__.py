@@ -20,6 +20,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "litevlm_oracle.c")
+_SRC_THREADS = os.path.join(_HERE, "litevlm_oracle_threads.c")  # all-cores score for the CPU baseline
 _BUILD = os.path.join(_HERE, "_build")
 _LIB = os.path.join(_BUILD, "liblitevlm_oracle.so")
 _lock = threading.Lock()
@@ -29,11 +30,13 @@ DTYPE_CODES = {"f32": 0, "bf16": 1, "e4m3": 2}
 
 
 def build(src: str = _SRC, out: str = _LIB, extra_flags=()) -> str:
-    """Compile the oracle with gcc (no fused multiply-add contraction)."""
+    """Compile the oracle with gcc (no fused multiply-add contraction). The
+    default build also links the all-cores score (litevlm_oracle_threads.c)."""
     os.makedirs(os.path.dirname(out), exist_ok=True)
     tmp = out + f".tmp{os.getpid()}"
-    cmd = ["gcc", "-std=c99", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
-           *extra_flags, "-o", tmp, src, "-lm"]
+    srcs = [src] + ([_SRC_THREADS] if src == _SRC else [])
+    cmd = ["gcc", "-std=c99", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared", "-pthread",
+           *extra_flags, "-o", tmp, *srcs, "-lm"]
     subprocess.run(cmd, check=True)
     os.replace(tmp, out)
     return out
@@ -46,7 +49,8 @@ def load(path: Optional[str] = None):
         return _bind(ctypes.CDLL(path))
     with _lock:
         if _lib is None:
-            if (not os.path.exists(_LIB)) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+            if (not os.path.exists(_LIB)) or os.path.getmtime(_LIB) < max(os.path.getmtime(_SRC),
+                                                                          os.path.getmtime(_SRC_THREADS)):
                 build()
             _lib = _bind(ctypes.CDLL(_LIB))
     return _lib
@@ -74,6 +78,9 @@ def _bind(lib):
     lib.litevlm_oracle_select_views.restype = ctypes.c_int
     lib.litevlm_oracle_project.argtypes = [i64, i32, i32, P, P, f64, P, P, i32, P, f64, P]
     lib.litevlm_oracle_project.restype = ctypes.c_int
+    if hasattr(lib, "litevlm_oracle_score_threads"):
+        lib.litevlm_oracle_score_threads.argtypes = [i32, P, P, i32, i32, i32, i32, P, P, f64, f64, P, i32]
+        lib.litevlm_oracle_score_threads.restype = ctypes.c_int
     return lib
 
 
@@ -117,6 +124,23 @@ def score(q: np.ndarray, k: np.ndarray, seq_offsets, text_offsets, hq: int, hkv:
         raise OracleError(f"litevlm_oracle_score returned {rc}")
     if details:
         return out, s64, rows, lse
+    return out
+
+
+def score_threads(q: np.ndarray, k: np.ndarray, seq_offsets, text_offsets, hq: int, hkv: int, head_dim: int,
+                  dtype: str = "bf16", q_scale: float = 1.0, k_scale: float = 1.0, threads: int = 1, lib=None):
+    """The scores of ``score`` computed on `threads` POSIX threads, bit for bit
+    the same (the serial summation order is kept)."""
+    lib = lib or load()
+    so = np.ascontiguousarray(seq_offsets, dtype=np.int32)
+    to = np.ascontiguousarray(text_offsets, dtype=np.int32)
+    q = np.ascontiguousarray(q)
+    k = np.ascontiguousarray(k)
+    out = np.zeros(int(so[-1]), dtype=np.float32)
+    rc = lib.litevlm_oracle_score_threads(so.size - 1, _ptr(so), _ptr(to), hq, hkv, head_dim, DTYPE_CODES[dtype],
+                                          _ptr(q), _ptr(k), float(q_scale), float(k_scale), _ptr(out), int(threads))
+    if rc != 0:
+        raise OracleError(f"litevlm_oracle_score_threads returned {rc}")
     return out
 
 
@@ -247,10 +271,12 @@ def project(x_bf16: np.ndarray, gamma, eps: float, w_bf16: np.ndarray, bias=None
 
 
 def select(w_inputs: dict, hq: int, hkv: int, head_dim: int, dtype: str, keep_k=None, keep_ratio=0.0,
-           gather=("hidden",), lib=None):
-    """The whole path on one batch: scores, kept indices, offsets and gathered rows."""
-    s = score(w_inputs["q"], w_inputs["k"], w_inputs["seq_offsets"], w_inputs["text_offsets"], hq, hkv,
-              head_dim, dtype, w_inputs.get("q_scale", 1.0), w_inputs.get("k_scale", 1.0), lib=lib)
+           gather=("hidden",), lib=None, threads: int = 1):
+    """The whole path on one batch: scores, kept indices, offsets and gathered
+    rows. threads > 1 computes the scores on that many threads (same bits)."""
+    args = (w_inputs["q"], w_inputs["k"], w_inputs["seq_offsets"], w_inputs["text_offsets"], hq, hkv, head_dim,
+            dtype, w_inputs.get("q_scale", 1.0), w_inputs.get("k_scale", 1.0))
+    s = score(*args, lib=lib) if threads <= 1 else score_threads(*args, threads=threads, lib=lib)
     kept, off = topk(w_inputs["seq_offsets"], s, keep_k=keep_k, keep_ratio=keep_ratio, lib=lib)
     rows = {name: compact(kept, w_inputs[name], lib=lib) for name in gather}
     return s, kept, off, rows

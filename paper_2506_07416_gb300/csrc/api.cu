@@ -40,6 +40,7 @@ struct litevlm_select {
     lvs::TopkShape topk_shape;    // per-request sizes passed to the top-k kernel by value
     std::string last_error;
     int32_t last_launches = 0;  // kernels the last call on this handle enqueued
+    long long wait_budget = lvs::kWaitBudgetCycles;  // clock cycles each device-side wait may take
 };
 
 namespace {
@@ -396,7 +397,7 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
                             const int32_t* text_offsets_h, const void* k_vis, const int32_t* seq_offsets_d,
                             const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
                             const CtxKeys* ctx, litevlm_stream_t stream, bool allow_defer = false,
-                            int* deferred_groups = nullptr)
+                            int* deferred_groups = nullptr, size_t clear_tickets = 0)
 {
     if (deferred_groups) *deferred_groups = 0;
     const litevlm_select_config_t& c = h->cfg;
@@ -453,7 +454,7 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
     p.hq = c.num_q_heads;
     p.hkv = c.num_kv_heads;
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
-    p.wait_budget = lvs::kWaitBudgetCycles;
+    p.wait_budget = h->wait_budget;
     p.slot_cols = (max_t + 15) & ~15;
     p.query_last = (c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
     p.extra = nullptr;
@@ -477,7 +478,7 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
         ca.hkv = c.num_kv_heads;
         ca.query_last = p.query_last;
         ca.c_log2 = p.c_log2;
-        ca.wait_budget = lvs::kWaitBudgetCycles;
+        ca.wait_budget = h->wait_budget;
         const cudaError_t ce = lvs::launch_ctx_stats(ca, row_bytes, fp8, (cudaStream_t)stream);
         if (ce != cudaSuccess) return cuda_fail(h, ce, "context-key statistics launch");
         p.extra = h->ctx_stats;
@@ -506,6 +507,12 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
             });
             p.order_n = batch;
         }
+    }
+    // a caller whose tickets may not be at rest (the no-alloc entry point's
+    // shared static scratch) has them cleared here, after every host-side check
+    if (clear_tickets > 0 && plan.groups > 1) {
+        const cudaError_t ce = cudaMemsetAsync(h->counters, 0, sizeof(int32_t) * clear_tickets, (cudaStream_t)stream);
+        if (ce != cudaSuccess) return cuda_fail(h, ce, "clearing the fold tickets");
     }
     const cudaError_t e =
         choice.resident
@@ -908,7 +915,7 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
     p.y8 = out_scale > 0.f ? static_cast<uint8_t*>(y) : nullptr;
     p.out_inv_scale = out_scale > 0.f ? 1.f / out_scale : 0.f;
     p.err = h->err_d;
-    p.wait_budget = lvs::kWaitBudgetCycles;
+    p.wait_budget = h->wait_budget;
     const cudaError_t e = lvs::launch_proj(tm_x, tm_w, p, bm, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "project launch");
     h->last_launches = 1;
@@ -943,6 +950,48 @@ litevlm_status_t litevlm_select_host_view(litevlm_select_t h, const void* host, 
         return fail(h, LITEVLM_ERR_INVALID_ARG, "the runtime gives this host memory no device address");
     }
     *device_view = d;
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_keep_offsets(int32_t batch, const int32_t* seq_offsets_h, const int32_t* keep_k_h,
+                                             float keep_ratio, int32_t* out_offsets_h)
+{
+    g_create_error.clear();
+    if (batch < 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
+    if (!out_offsets_h) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "out_offsets_h is NULL");
+    if (!keep_k_h && !(keep_ratio >= 0.f && keep_ratio <= 1.f))
+        return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "keep_ratio must be in [0, 1]");
+    if (batch == 0) {
+        out_offsets_h[0] = 0;
+        return LITEVLM_OK;
+    }
+    int64_t tot_n = 0;
+    litevlm_status_t s = check_offsets(nullptr, seq_offsets_h, batch, INT32_MAX, "seq_offsets", &tot_n);
+    if (s != LITEVLM_OK) return s;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int32_t n = seq_offsets_h[b + 1] - seq_offsets_h[b];
+        const int64_t k = keep_k_h ? (int64_t)keep_k_h[b] : keep_count_host(n, keep_ratio);
+        if (k < 0 || k > n)
+            return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "keep_k[" + std::to_string(b) + "] = " + std::to_string(k) +
+                                                              " outside [0, " + std::to_string(n) + "]");
+    }
+    // written only once every request is known to be valid
+    out_offsets_h[0] = 0;
+    int64_t run = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int32_t n = seq_offsets_h[b + 1] - seq_offsets_h[b];
+        run += keep_k_h ? (int64_t)keep_k_h[b] : keep_count_host(n, keep_ratio);
+        out_offsets_h[b + 1] = (int32_t)run;
+    }
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_set_wait_budget(litevlm_select_t h, int64_t cycles)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (cycles < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "cycles must be >= 0 (0 restores the default)");
+    h->wait_budget = cycles == 0 ? lvs::kWaitBudgetCycles : (long long)cycles;
     return LITEVLM_OK;
 }
 
@@ -1104,14 +1153,12 @@ extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, in
     if (s == LITEVLM_OK && plan[3] > 1 && (int64_t)plan[3] * tot_n > kNoAllocPartialFloats)
         s = fail(&h, LITEVLM_ERR_WORKSPACE,
                  "head groups x total_visual exceeds the static partial-score scratch (1048576 floats)");
-    // tickets start at zero (a launch that gave up may have left some taken)
-    if (s == LITEVLM_OK && plan[3] > 1) {
-        e = cudaMemsetAsync(h.counters, 0, sizeof(int32_t) * (size_t)n_tickets, (cudaStream_t)stream);
-        if (e != cudaSuccess) s = cuda_fail(&h, e, "score_noalloc: clearing the fold tickets");
-    }
+    // the tickets start at zero (a launch that gave up may have left some
+    // taken): score_impl clears them after all of its host-side checks, right
+    // before the launch, so a rejected call enqueues nothing
     if (s == LITEVLM_OK)
-        s = litevlm_select_score(&h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d,
-                                 seq_offsets_h, q_scale, k_scale, scores, stream);
+        s = score_impl(&h, batch, q_text, text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h,
+                       q_scale, k_scale, scores, nullptr, stream, false, nullptr, (size_t)n_tickets);
     {
         std::lock_guard<std::mutex> lock(g_noalloc_mutex);
         NoAllocDevice& d = g_noalloc[dev];

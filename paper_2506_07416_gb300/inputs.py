@@ -69,17 +69,6 @@ class Workload:
     def text_offsets(self) -> np.ndarray:
         return _offsets(self.n_txt)
 
-    def keep_counts(self, ratio: Optional[float] = None) -> List[int]:
-        """Number of rows kept per request: keep_k if given, else floor(r * N_b).
-
-        The ratio is a float32 number widened to double before the product,
-        which is how the C-ABI and the oracle read it.
-        """
-        if self.keep_k is not None and ratio is None:
-            return [int(x) for x in self.keep_k]
-        r = float(np.float32(self.keep_ratio if ratio is None else ratio))
-        return [max(0, min(n, int(math.floor(r * n)))) for n in self.n_vis]
-
     def row_bytes(self) -> Dict[str, int]:
         return {"hidden": self.hidden * 2, "k": self.hkv * self.head_dim * (2 if self.dtype == "bf16" else 1),
                 "v": self.hkv * self.head_dim * 2}

@@ -65,8 +65,11 @@ def _load():
     lib.litevlm_select_score_plan.argtypes = [P, i32, P, P, P]
     lib.litevlm_select_splice.argtypes = [P, i32, P, P, P, P, P, P, P, P, P, P, P, P, i64, P, P, P, P, P]
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
+    lib.litevlm_select_keep_offsets.argtypes = [i32, P, P, f32, P]
+    lib.litevlm_select_set_wait_budget.argtypes = [P, i64]
     for fn in ("create", "destroy", "score", "score_full_keys", "topk", "compact", "check_device", "score_plan",
-               "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project", "score_topk", "host_view"):
+               "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project", "score_topk", "host_view",
+               "keep_offsets", "set_wait_budget"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -79,7 +82,8 @@ EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_la
            "litevlm_select_check_device", "litevlm_select_score_plan", "litevlm_select_score_noalloc",
            "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views",
            "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project",
-           "litevlm_select_last_launches", "litevlm_select_score_topk", "litevlm_select_host_view"]
+           "litevlm_select_last_launches", "litevlm_select_score_topk", "litevlm_select_host_view",
+           "litevlm_select_keep_offsets", "litevlm_select_set_wait_budget"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -239,6 +243,20 @@ def check_device(handle: int, stream=None) -> None:
     _check(LIB.litevlm_select_check_device(handle, _stream_ptr(stream)), handle)
 
 
+def keep_offsets(seq_offsets_h, keep_k_h=None, keep_ratio: float = 0.0) -> np.ndarray:
+    """litevlm_select_keep_offsets: prefix of the kept-token counts k_b (host only)."""
+    so = _host_i32(seq_offsets_h)
+    kk = _host_i32(keep_k_h)
+    out = np.zeros(len(so), np.int32)
+    _check(LIB.litevlm_select_keep_offsets(len(so) - 1, _ptr(so), _ptr(kk), keep_ratio, _ptr(out)), None)
+    return out
+
+
+def set_wait_budget(handle: int, cycles: int) -> None:
+    """litevlm_select_set_wait_budget: clock cycles each device-side wait may take (0: default)."""
+    _check(LIB.litevlm_select_set_wait_budget(handle, int(cycles)), handle)
+
+
 def score_noalloc(num_q_heads: int, num_kv_heads: int, head_dim: int, qk_dtype: str, batch: int, q_text,
                   text_offsets_d, text_offsets_h, k_vis, seq_offsets_d, seq_offsets_h, q_scale: float,
                   k_scale: float, scores, err_d, stream=None) -> None:
@@ -338,10 +356,7 @@ class Selector:
         if kk_h is not None:
             kk_d = keep_k if isinstance(keep_k, torch.Tensor) and keep_k.is_cuda else \
                 torch.from_numpy(kk_h).to(k.device)
-            total = int(kk_h.sum())
-        else:
-            r = float(np.float32(keep_ratio))
-            total = int(sum(min(n, max(0, int(np.floor(r * n)))) for n in np.diff(so_h)))
+        total = int(keep_offsets(so_h, kk_h, keep_ratio)[-1])
         scores = torch.empty(max(1, int(so_h[-1])), dtype=torch.float32, device=k.device)
         kept = torch.empty(max(total, 1), dtype=torch.int32, device=k.device)
         off_d = torch.empty(batch + 1, dtype=torch.int32, device=k.device)
@@ -390,11 +405,7 @@ class Selector:
             kk_d = keep_k if isinstance(keep_k, torch.Tensor) and keep_k.is_cuda else \
                 torch.from_numpy(kk_h).to(scores.device)
         off_h = np.zeros(batch + 1, dtype=np.int32)
-        if kk_h is not None:
-            total = int(kk_h.sum())
-        else:
-            r = float(np.float32(keep_ratio))
-            total = int(sum(min(n, max(0, int(np.floor(r * n)))) for n in np.diff(so_h)))
+        total = int(keep_offsets(so_h, kk_h, keep_ratio)[-1])
         if kept_idx is None:
             kept_idx = torch.empty(max(total, 1), dtype=torch.int32, device=scores.device)
         if out_offsets is None:
@@ -444,6 +455,9 @@ class Selector:
 
     def check_device(self, stream=None) -> None:
         check_device(self.handle, stream)
+
+    def set_wait_budget(self, cycles: int) -> None:
+        set_wait_budget(self.handle, cycles)
 
     def score_plan(self, text_offsets_h, seq_offsets_h):
         so = _host_i32(seq_offsets_h)

@@ -103,3 +103,45 @@ def test_create_without_gpu_reports_cuda_error(sel):
     rc = sel.LIB.litevlm_select_create(ctypes.byref(_cfg(sel)), ctypes.byref(h))
     assert rc == 4 and h.value is None
     assert b"create" in sel.LIB.litevlm_select_last_error(None)
+
+
+def test_keep_offsets_match_the_oracle_keep_count(sel):
+    # litevlm_select_keep_offsets is the library's own k_b = floor((double)r * N_b)
+    # (Results, "Visual Token Compression"); it must agree with the oracle's
+    # litevlm_oracle_keep_count request by request, on the bench sizes, the
+    # paper's Table 1 sizes and random ones, for ratios that are not exact in fp32
+    import numpy as np
+    import oracle
+    rng = np.random.Generator(np.random.PCG64(11))
+    sizes = [0, 1, 7, 128, 576, 896, 1536, 3072, 3456, 6144, 65536] + list(rng.integers(0, 10000, size=40))
+    so = np.zeros(len(sizes) + 1, np.int32)
+    so[1:] = np.cumsum(sizes)
+    for r in (0.0, 0.1, 0.2, 0.25, 0.3, 1.0 / 3.0, 0.5, 0.7, 0.8, 0.9, 0.999, 1.0):
+        off = sel.keep_offsets(so, None, r)
+        want = np.concatenate([[0], np.cumsum([oracle.keep_count(int(n), r) for n in sizes])])
+        assert np.array_equal(off, want), r
+    kk = np.array([min(n, 3) for n in sizes], np.int32)
+    off = sel.keep_offsets(so, kk, 0.0)
+    assert np.array_equal(off, np.concatenate([[0], np.cumsum(kk)]))
+    assert sel.keep_offsets(np.zeros(1, np.int32), None, 0.5).tolist() == [0]
+
+
+def test_keep_offsets_rejects_bad_arguments_and_leaves_the_output(sel):
+    import numpy as np
+    so = np.array([0, 10, 30], np.int32)
+    out = np.full(3, -7, np.int32)
+    L = sel.LIB
+    assert L.litevlm_select_keep_offsets(2, so.ctypes.data, None, 1.5, out.ctypes.data) == 1
+    assert L.litevlm_select_keep_offsets(2, so.ctypes.data, None, float("nan"), out.ctypes.data) == 1
+    bad_k = np.array([3, 21], np.int32)  # 21 > N_1 = 20
+    assert L.litevlm_select_keep_offsets(2, so.ctypes.data, bad_k.ctypes.data, 0.0, out.ctypes.data) == 1
+    assert b"keep_k[1]" in L.litevlm_select_last_error(None)
+    neg = np.array([0, 10, 5], np.int32)
+    assert L.litevlm_select_keep_offsets(2, neg.ctypes.data, None, 0.5, out.ctypes.data) == 1
+    assert L.litevlm_select_keep_offsets(2, so.ctypes.data, None, 0.5, None) == 1
+    assert L.litevlm_select_keep_offsets(-1, so.ctypes.data, None, 0.5, out.ctypes.data) == 1
+    assert out.tolist() == [-7, -7, -7]
+
+
+def test_wait_budget_setter_needs_a_handle(sel):
+    assert sel.LIB.litevlm_select_set_wait_budget(None, 100) == 1

@@ -316,6 +316,13 @@ def test_tiny_whole_path(sel):
 
 # ----------------------------------------------------------------------------- full size
 
+def _rows_u8(t):
+    """Rows of a device tensor as host bytes, [rows, row_bytes] uint8."""
+    t = t.contiguous()
+    u = t if t.dtype == torch.uint8 else t.view(torch.uint8)
+    return u.reshape(t.shape[0], -1).cpu().numpy()
+
+
 FULL = [("single", [0]), ("highres", [0]), ("fp8_ragged", None), ("sweep", [0, 77, 127])]
 
 
@@ -373,6 +380,12 @@ def test_full_size_workload(sel, name, sample):
             assert torch.equal(dst.view(torch.uint8) if dst.dtype != torch.uint8 else dst,
                                src.index_select(0, idx).view(torch.uint8) if src.dtype != torch.uint8
                                else src.index_select(0, idx))
+        # and on the sampled requests, byte for byte against the oracle's gather
+        for b in sample:
+            kb = ok[ooff[b]:ooff[b + 1]] - so[b]
+            for src, dst in zip(srcs, outs):
+                want = oracle.compact(kb, _rows_u8(src[so[b]:so[b + 1]]))
+                np.testing.assert_array_equal(_rows_u8(dst[off_h[b]:off_h[b + 1]]), want)
     del xd
     torch.cuda.empty_cache()
 

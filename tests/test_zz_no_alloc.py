@@ -4,9 +4,11 @@ library's static device arrays, no handle and no allocation.
 The GPU test compares two consecutive calls with the handle-based
 litevlm_select_score on the same inputs. Both take the same launch plan and
 the kernels reduce in a fixed order, so the scores must be bit-identical; the
-second call also checks that the first left the static fold tickets ready.
-Named to be collected after the other test files, so it also runs after them
-in one process (and the library's static scratch has already been used)."""
+second call runs on scratch the first one has used (each call clears the fold
+tickets it needs before its launch). One case is also compared directly with
+the oracle at the bf16 tolerance. Named to be collected after the other test
+files, so it also runs after them in one process (and the library's static
+scratch has already been used)."""
 import os
 
 import numpy as np
@@ -75,3 +77,20 @@ def test_noalloc_matches_handle_path_on_two_consecutive_calls(sel, w):
     for out in outs:
         assert torch.equal(out, ref)
     s.close()
+
+
+@pytest.mark.gpu
+def test_noalloc_matches_the_oracle(sel):
+    import oracle
+    from gpu_util import assert_scores_close, to_device
+    w = CASES[1]
+    x = inputs.make_numpy(w)
+    xd = to_device(x, w)
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = torch.full((w.total_vis,), float("nan"), dtype=torch.float32, device="cuda")
+    sel.score_noalloc(w.hq, w.hkv, w.head_dim, w.dtype, w.batch, xd["q"], xd["text_offsets"], x["text_offsets"],
+                      xd["k"], xd["seq_offsets"], x["seq_offsets"], 1.0, 1.0, out, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    o = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, w.dtype)
+    assert_scores_close(out.cpu().numpy(), o, w.dtype)
