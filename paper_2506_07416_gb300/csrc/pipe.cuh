@@ -16,12 +16,17 @@ struct Ctl {
     long long budget;
 };
 
+// Suspend-time hint of the retries (ns): a waiting thread sleeps until its
+// phase completes or this much time passes, then checks the abort flag and
+// the budget.
+constexpr uint32_t kWaitSleepNs = 20000;
+
 __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, const Ctl& c)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait_sleep(bar, parity, kWaitSleepNs)) return true;
         if (*c.abort) return false;
         if (clock64() - t0 > c.budget) {
             *c.abort = 1;
@@ -36,7 +41,7 @@ __device__ __forceinline__ bool wait_phase_cluster(uint32_t bar, uint32_t parity
     if (mbar_try_wait_cluster(bar, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
-        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (mbar_try_wait_cluster_sleep(bar, parity, kWaitSleepNs)) return true;
         if (*c.abort) return false;
         if (clock64() - t0 > c.budget) {
             *c.abort = 1;

@@ -23,15 +23,18 @@
 //   C  each visual token adds sum_i e_ij * w_i (= sum_i 2^(s_ij * c - b_i)) to
 //      its running score, and the slot goes back to the MMA warp.
 // While the statistics travel, the producer keeps the next head's K tiles
-// streaming into the ring. The two epilogue warpgroups split each slot's text
-// columns (no cross-warpgroup merge of statistics); each keeps its own partial
-// score rows, added in a fixed order at the end. With several head groups the
-// CTAs write partial rows and a per-tile ticket lets the last writer of each
-// tile add them (fixed group order).
+// streaming into the ring. The four epilogue warpgroups split each slot's text
+// columns (a quarter each, read 16 columns at a time; no cross-warpgroup merge
+// of statistics), so every SM sub-partition runs four epilogue warps that hide
+// one another's TMEM-load and exponential latencies; each warpgroup keeps its
+// own partial score rows, added in a fixed order at the end. With several head
+// groups the CTAs write partial rows and a per-tile ticket lets the last writer
+// of each tile add them (fixed group order).
 //
-// Warp roles (320 threads): warp 0 = TMA producer, warp 1 = TMEM allocator and
-// MMA issuer, warps 2..5 / 6..9 = epilogue warpgroups 0 / 1. Waits are bounded
-// (clock budget) as in score_tc.cu.
+// Warp roles (608 threads): warp 0 = TMA producer, warp 1 = TMEM allocator
+// and MMA issuer of the even tiles, warp 2 = MMA issuer of the odd tiles,
+// warps 3..18 = epilogue warpgroups 0..3 (TMEM lane quadrant = warp % 4).
+// Waits are bounded (clock budget) as in score_tc.cu.
 
 #include <math.h>
 
@@ -43,7 +46,9 @@ namespace lvs {
 
 namespace {
 
-constexpr int kResThreads = 320;
+constexpr int kResWG = 4;                       // epilogue warpgroups
+constexpr int kResThreads = 96 + 128 * kResWG;  // producer warp, two MMA warps, epilogue
+constexpr int kResChunk = 16;                   // text columns per epilogue TMEM load
 constexpr int kResTmemCols = 512;
 constexpr int kResMaxSlots = 16;
 constexpr int kBufSlots = kResMaxSlots / 2;  // slots per buffer with two TMEM buffers
@@ -55,14 +60,16 @@ struct ResLayout {
     static constexpr int KB = ROW_BYTES / 128;
     static constexpr int TILE_BYTES = kTileRows * ROW_BYTES;
     static constexpr int Q_BYTES = MROWS * ROW_BYTES;
+    static constexpr int WGC = MROWS / kResWG;  // most text columns one warpgroup owns (16 or 32)
     // statistics receive buffer: [kStatSlots heads][cluster rank][column] (m, l);
     // cluster size times slot columns must fit RECV_COLS
     static constexpr int RECV_COLS = ROW_BYTES == 256 ? 640 : 1024;
-    static constexpr int ACC_BYTES = 2 * kResMaxSlots * kTileRows * 4;  // per warpgroup partial rows
-    static constexpr int SCR_BYTES = 3 * 2 * 4 * 64 * 4;  // [max of head s & 1 (2) | sum][wg][warp][64 cols]
+    static constexpr int ACC_BYTES = kResWG * kResMaxSlots * kTileRows * 4;  // per warpgroup partial rows
+    // [max of head s & 1 (2) | sum][wg][quadrant warp][WGC columns]
+    static constexpr int SCR_BYTES = 3 * kResWG * 4 * WGC * 4;
     static constexpr int NBAR_FIXED = 2 * 2 + 2 * kResMaxSlots + kStatSlots + 1;
-    static constexpr int FIXED = 2 * Q_BYTES + ACC_BYTES + SCR_BYTES + kStatSlots * RECV_COLS * 8 + 4 * 64 * 4 +
-                                 kResMaxSlots * 4 + (NBAR_FIXED + 2 * 10) * 8 + 64 + 1024;
+    static constexpr int FIXED = 2 * Q_BYTES + ACC_BYTES + SCR_BYTES + kStatSlots * RECV_COLS * 8 +
+                                 2 * kResWG * WGC * 4 + kResMaxSlots * 4 + (NBAR_FIXED + 2 * 10) * 8 + 64 + 1024;
     static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
     static constexpr int kStages = STAGES_FIT > 10 ? 10 : STAGES_FIT;
     static constexpr int OFF_K = 0;
@@ -71,8 +78,8 @@ struct ResLayout {
     static constexpr int OFF_SCR = OFF_ACC + ACC_BYTES;
     static constexpr int OFF_RECV = OFF_SCR + SCR_BYTES;
     static constexpr int OFF_B2 = OFF_RECV + kStatSlots * RECV_COLS * 8;
-    static constexpr int OFF_MC = OFF_B2 + 2 * 64 * 4;     // column weights per warpgroup column
-    static constexpr int OFF_FLAGS = OFF_MC + 2 * 64 * 4;  // CTA column max * c per warpgroup column
+    static constexpr int OFF_MC = OFF_B2 + kResWG * WGC * 4;     // column weights per warpgroup column
+    static constexpr int OFF_FLAGS = OFF_MC + kResWG * WGC * 4;  // -(CTA column max * c) per warpgroup column
     static constexpr int OFF_BAR = OFF_FLAGS + kResMaxSlots * 4;
     static constexpr int NBAR = 2 * kStages + NBAR_FIXED;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
@@ -80,13 +87,26 @@ struct ResLayout {
     static constexpr int ALLOC = BYTES + 1024;
 };
 
-// x[c] (c < 32, one value per lane per column) -> sum over the warp's lanes of
-// column `lane`, returned in lane `lane`.
-__device__ __forceinline__ float transpose_sum32(float (&x)[32], int lane)
+// Columns one epilogue warpgroup owns for n2 slot columns (n2 % 16 == 0), and
+// the widest TMEM column a slot's epilogue reads relative to the slot start
+// (the last warpgroup's last 16-column chunk may reach past the slot; the
+// extra columns are read, never used or written).
+__host__ __device__ __forceinline__ int res_wg_cols(int n2) { return n2 / kResWG; }
+__host__ __device__ __forceinline__ int res_read_span(int n2)
+{
+    const int cpw = res_wg_cols(n2);
+    return (kResWG - 1) * cpw + kResChunk * ((cpw + kResChunk - 1) / kResChunk);
+}
+
+// x[c] (c < 16, one value per lane per column) -> sum over the warp's 32 lanes
+// of column (lane & 15), returned in every lane: four halving exchanges leave
+// lane l with column l & 15 summed over the 16 lanes that share bit 4 of l,
+// and one more exchange adds the two halves.
+__device__ __forceinline__ float transpose_sum16(float (&x)[16], int lane)
 {
 #pragma unroll
-    for (int step = 0; step < 5; ++step) {
-        const int o = 16 >> step;
+    for (int step = 0; step < 4; ++step) {
+        const int o = 8 >> step;
         const bool up = (lane & o) != 0;
 #pragma unroll
         for (int k = 0; k < o; ++k) {
@@ -95,7 +115,7 @@ __device__ __forceinline__ float transpose_sum32(float (&x)[32], int lane)
             x[k] = keep + __shfl_xor_sync(0xffffffffu, send, o);
         }
     }
-    return x[0];
+    return x[0] + __shfl_xor_sync(0xffffffffu, x[0], 16);
 }
 
 // What a CTA serves of its request: the text rows, the tile range, and whether
@@ -117,7 +137,7 @@ __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int 
     r.n_tiles = (r.N + kTileRows - 1) / kTileRows;
     const int tpc = r.N > 0 ? (r.n_tiles + (int)csize - 1) / (int)csize : 0;
     // Shape errors are caught on the host; this only keeps the kernel within its buffers.
-    const int span = p.slot_cols / 2 + 32 * ((p.slot_cols / 2 + 31) / 32);  // columns the epilogue reads per slot
+    const int span = res_read_span(p.slot_cols);  // columns the epilogue reads per slot
     r.nb = p.res_nb == 2 ? 2 : 1;
     const int buf_cols = r.nb == 2 ? kBufCols : kResTmemCols;
     r.bad = r.T > mrows || r.n2 > p.slot_cols || (r.N > 0 && r.T <= 0) ||
@@ -184,8 +204,9 @@ __global__ void __launch_bounds__(kResThreads, 1)
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
     float* acc_s = reinterpret_cast<float*>(smem + L::OFF_ACC);
-    float* scr_max = reinterpret_cast<float*>(smem + L::OFF_SCR);        // [head & 1][wg][warp][64]
-    float* scr_sum = scr_max + 2 * 2 * 4 * 64;                            // [wg][warp][64]
+    constexpr int WGC = L::WGC;
+    float* scr_max = reinterpret_cast<float*>(smem + L::OFF_SCR);        // [head & 1][wg][warp][WGC]
+    float* scr_sum = scr_max + 2 * kResWG * 4 * WGC;                      // [wg][warp][WGC]
     const float2* recv = reinterpret_cast<const float2*>(smem + L::OFF_RECV);
     float* b2_s = reinterpret_cast<float*>(smem + L::OFF_B2);
     float* mc_s = reinterpret_cast<float*>(smem + L::OFF_MC);
@@ -198,14 +219,14 @@ __global__ void __launch_bounds__(kResThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(BAR(Q_FULL + i), 1);
-            mbar_init(BAR(Q_EMPTY + i), 1);
+            mbar_init(BAR(Q_EMPTY + i), 2);  // one commit per MMA-issuing thread
         }
         for (int i = 0; i < kStatSlots; ++i) mbar_init(BAR(STATS + i), 1);  // the local arm; peers complete bytes
         for (int i = 0; i < kResMaxSlots; ++i) {
             mbar_init(BAR(S_FULL + i), 1);
-            mbar_init(BAR(S_EMPTY + i), 8);  // one arrival per epilogue warp
+            mbar_init(BAR(S_EMPTY + i), 4 * kResWG);  // one arrival per epilogue warp
         }
-        mbar_init(BAR(DRAIN), 1);
+        mbar_init(BAR(DRAIN), 2);
         *abort_flag = 0;
         fence_mbar_init_cluster();
     }
@@ -289,12 +310,21 @@ __global__ void __launch_bounds__(kResThreads, 1)
         }
         __syncwarp();
         cluster_wait();
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+    } else if (warp <= 2) {
+        // ------------------------------------------------------------ MMA issuers
+        // Two issuing threads (lane 0 of warps 1 and 2) take alternate tiles:
+        // issuing a tile (two barrier waits, the contractions, two commits)
+        // costs more time than the tensor core needs to run it, so one thread's
+        // waits and commits overlap the other thread's contractions. Each
+        // thread follows the global tile sequence for the ring's stage and
+        // phase and commits its own contractions. The operand descriptors are
+        // made once (per head for Q, per tile for K) and each K step adds a
+        // constant to the start-address field (shared-memory offsets stay below
+        // 256 KB, so the 14-bit field never carries).
         if (lane == 0) {
+            const int who = warp - 1;  // 0: even tiles, 1: odd tiles
             if (mt > 0) {
                 const uint32_t idesc = idesc_make(128, (uint32_t)n2, FMT);
-                uint32_t ks = 0, kph = 0;
                 bool ok = true;
                 for (int s = 0; s < hpg && ok; ++s) {
                     const int qb = s & 1;
@@ -302,25 +332,29 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     const uint32_t use = nb == 2 ? (uint32_t)(s >> 1) : (uint32_t)s;  // earlier heads in this buffer
                     if (!wait_phase(BAR(Q_FULL + qb), (s >> 1) & 1, ctl)) break;
                     tc_fence_after();
-                    const uint32_t qaddr = base + L::OFF_Q + qb * L::Q_BYTES;
-                    for (int tl = 0; tl < mt; ++tl) {
+                    const uint64_t qdesc = sdesc_k_sw128(base + L::OFF_Q + qb * L::Q_BYTES);
+                    for (int tl = who; tl < mt; tl += 2) {
                         const int sl = buf * kBufSlots + tl;
+                        const int gt = s * mt + tl;  // the ring runs over the tiles of all heads in order
+                        const uint32_t ks = (uint32_t)(gt % kStages), kph = (uint32_t)(gt / kStages) & 1u;
                         if (!wait_phase(BAR(K_FULL + ks), kph, ctl)) { ok = false; break; }
                         if (!wait_phase(BAR(S_EMPTY + sl), (use & 1u) ^ 1u, ctl)) { ok = false; break; }
                         tc_fence_after();
-                        const uint32_t kaddr = base + L::OFF_K + ks * L::TILE_BYTES;
+                        const uint64_t kdesc = sdesc_k_sw128(base + L::OFF_K + ks * L::TILE_BYTES);
                         const uint32_t d = tmem + (uint32_t)(buf * kBufCols + tl * scols);
 #pragma unroll
                         for (int st = 0; st < KSTEPS; ++st) {
-                            const uint32_t qoff = (st >> 2) * (MROWS * 128) + (st & 3) * 32;
-                            const uint32_t koff = (st >> 2) * (kTileRows * 128) + (st & 3) * 32;
-                            if (FP8) mma_f8(d, sdesc_k_sw128(kaddr + koff), sdesc_k_sw128(qaddr + qoff), idesc, st > 0);
-                            else mma_f16(d, sdesc_k_sw128(kaddr + koff), sdesc_k_sw128(qaddr + qoff), idesc, st > 0);
+                            constexpr uint64_t kQ16 = MROWS * 128 / 16, kK16 = kTileRows * 128 / 16;
+                            const uint64_t qoff = (uint64_t)(st >> 2) * kQ16 + (uint64_t)(st & 3) * 2;
+                            const uint64_t koff = (uint64_t)(st >> 2) * kK16 + (uint64_t)(st & 3) * 2;
+                            if (FP8) mma_f8(d, kdesc + koff, qdesc + qoff, idesc, st > 0);
+                            else mma_f16(d, kdesc + koff, qdesc + qoff, idesc, st > 0);
                         }
                         mma_commit(BAR(S_FULL + sl));
                         mma_commit(BAR(K_EMPTY + ks));
-                        if (++ks == kStages) { ks = 0; kph ^= 1; }
                     }
+                    // Q(s) is free once both threads' contractions of head s are done
+                    // (one arrival each; a thread without tiles in this head arrives at once)
                     if (ok) mma_commit(BAR(Q_EMPTY + qb));
                 }
             }
@@ -332,31 +366,31 @@ __global__ void __launch_bounds__(kResThreads, 1)
         __syncwarp();
         cluster_wait();
     } else {
-        // ------------------------------------------------------------ epilogue (2 warpgroups)
+        // ------------------------------------------------------------ epilogue (kResWG warpgroups)
         cluster_wait();  // the peers' barriers and buffers exist before any statistics go out
         // Control flow is identical for every thread of a warpgroup (named
         // barriers); after an abort every wait returns at once. Warp-synchronous
         // instructions (tcgen05.ld, redux.sync, shuffles) run under branches
-        // that are uniform in the CTA only: always 32 columns per chunk, columns
+        // that are uniform in the CTA only: always 16 columns per chunk, columns
         // past the warpgroup's range masked arithmetically.
         // Iteration i runs A and B of head i and sends its statistics, then C of
         // head i - 1 with two TMEM buffers (the statistics of head i - 1 had a
         // whole A + B to travel, and the MMAs of head i + 1 fill the other buffer
         // while C reads it, slot by slot), or C of head i with one buffer.
-        const int wg = (warp - 2) >> 2;
+        const int wg = (warp - 3) >> 2;
         const int quad = warp & 3;
-        const int et = threadIdx.x - 64;               // 0..255
+        const int et = threadIdx.x - 96;               // 0 .. 128 * kResWG - 1
         const int wt = et - 128 * wg;                  // 0..127 within the warpgroup
         const int vrow = quad * 32 + lane;             // visual token of this lane within a tile
         const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
         const uint32_t wg_bar = 2u + (uint32_t)wg;
-        const int h2 = n2 >> 1;                        // this warpgroup's columns: [c_begin, c_begin + h2)
-        const int c_begin = wg * h2;
-        const int nch = (h2 + 31) >> 5;
+        const int cpw = res_wg_cols(n2);               // this warpgroup's columns: [c_begin, c_begin + cpw)
+        const int c_begin = wg * cpw;
+        const int nch = (cpw + kResChunk - 1) / kResChunk;
         float* accw = acc_s + wg * kResMaxSlots * kTileRows;
-        float* ssum = scr_sum + wg * 4 * 64;
-        float* b2w = b2_s + wg * 64;                   // weight of column c_begin + c, 0 for c >= h2 or >= T
-        float* mcw = mc_s + wg * 64;                   // -(CTA column max * c) of column c_begin + c
+        float* ssum = scr_sum + wg * 4 * WGC;
+        float* b2w = b2_s + wg * WGC;                  // weight of column c_begin + c, 0 for c >= cpw or >= T
+        float* mcw = mc_s + wg * WGC;                  // -(CTA column max * c) of column c_begin + c
         const uint32_t recv_base = base + L::OFF_RECV;
         const uint32_t tcol = tmem + lane_off;
         for (int tl = 0; tl < mt; ++tl) accw[tl * kTileRows + vrow] = 0.f;
@@ -375,22 +409,21 @@ __global__ void __launch_bounds__(kResThreads, 1)
             const uint32_t use = nb == 2 ? (uint32_t)(s >> 1) : (uint32_t)s;
             const int slot = s & (kStatSlots - 1);
             const uint32_t tbuf = tcol + (uint32_t)(buf * kBufCols);
-            float* smax = scr_max + ((s & 1) * 2 + wg) * 4 * 64;
+            float* smax = scr_max + ((s & 1) * kResWG + wg) * 4 * WGC;
             if (et == 0) mbar_arrive_expect_tx(BAR(STATS + slot), (uint32_t)(csize * n2 * 8));
             for (int ch = 0; ch < nch; ++ch) {
-                const int cw = min(32, h2 - 32 * ch);
-                const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
+                const uint32_t col0 = (uint32_t)(c_begin + kResChunk * ch);
                 // ---- A: column maxima, per thread over its slots, then over the lanes
-                float cm[32];
+                float cm[16];
 #pragma unroll
-                for (int c = 0; c < 32; ++c) cm[c] = -INFINITY;
+                for (int c = 0; c < 16; ++c) cm[c] = -INFINITY;
                 {
-                    float va[32], vb[32];
+                    float va[16], vb[16];
                     if (ch == 0 && mt > 0) {  // a rank without tiles gets no MMA
                         wait_phase(BAR(S_FULL + buf * kBufSlots), use & 1u, ctl);
                         tc_fence_after();
                     }
-                    tmem_ld32(tbuf + col0, va);
+                    tmem_ld16(tbuf + col0, va);
                     for (int tl = 0; tl < mt; tl += 2) {
                         const int t1 = min(tl + 1, mt - 1), t2 = min(tl + 2, mt - 1);
                         tmem_wait_ld();
@@ -398,40 +431,43 @@ __global__ void __launch_bounds__(kResThreads, 1)
                             wait_phase(BAR(S_FULL + buf * kBufSlots + t1), use & 1u, ctl);
                             tc_fence_after();
                         }
-                        tmem_ld32(tbuf + (uint32_t)(t1 * scols) + col0, vb);
+                        tmem_ld16(tbuf + (uint32_t)(t1 * scols) + col0, vb);
                         if (lane_valid(tl)) {
 #pragma unroll
-                            for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], va[c]);
+                            for (int c = 0; c < 16; c += 2) {
+                                cm[c] = fmaxf(cm[c], va[c]);
+                                cm[c + 1] = fmaxf(cm[c + 1], va[c + 1]);
+                            }
                         }
                         tmem_wait_ld();
                         if (ch == 0 && tl + 2 < mt) {
                             wait_phase(BAR(S_FULL + buf * kBufSlots + t2), use & 1u, ctl);
                             tc_fence_after();
                         }
-                        tmem_ld32(tbuf + (uint32_t)(t2 * scols) + col0, va);
+                        tmem_ld16(tbuf + (uint32_t)(t2 * scols) + col0, va);
                         if (lane_valid(tl + 1)) {
 #pragma unroll
-                            for (int c = 0; c < 32; ++c) cm[c] = fmaxf(cm[c], vb[c]);
+                            for (int c = 0; c < 16; ++c) cm[c] = fmaxf(cm[c], vb[c]);
                         }
                     }
                     tmem_wait_ld();
                 }
 #pragma unroll
-                for (int c = 0; c < 32; ++c) cm[c] = warp_max_f32(cm[c]);
+                for (int c = 0; c < 16; ++c) cm[c] = warp_max_f32(cm[c]);
                 if (lane == 0) {
 #pragma unroll
-                    for (int c = 0; c < 32; c += 4)
-                        *reinterpret_cast<float4*>(smax + quad * 64 + 32 * ch + c) =
+                    for (int c = 0; c < 16; c += 4)
+                        *reinterpret_cast<float4*>(smax + quad * WGC + kResChunk * ch + c) =
                             make_float4(cm[c], cm[c + 1], cm[c + 2], cm[c + 3]);
                 }
                 named_bar_sync(wg_bar, 128);
                 // CTA-local column max * c, once per column, read back by B from shared
-                // memory (keeps 32 registers per thread free in B)
-                if (wt < 32) {
-                    float m = smax[32 * ch + wt];
+                // memory (keeps registers free in B)
+                if (wt < kResChunk) {
+                    float m = smax[kResChunk * ch + wt];
 #pragma unroll
-                    for (int q = 1; q < 4; ++q) m = fmaxf(m, smax[q * 64 + 32 * ch + wt]);
-                    mcw[32 * ch + wt] = -(m * cl);  // columns past cw: garbage, never used
+                    for (int q = 1; q < 4; ++q) m = fmaxf(m, smax[q * WGC + kResChunk * ch + wt]);
+                    mcw[kResChunk * ch + wt] = -(m * cl);  // columns past cpw: garbage, never used
                 }
                 named_bar_sync(wg_bar, 128);
             }
@@ -441,25 +477,25 @@ __global__ void __launch_bounds__(kResThreads, 1)
             const int buf = nb == 2 ? (s & 1) : 0;
             const int slot = s & (kStatSlots - 1);
             const uint32_t tbuf = tcol + (uint32_t)(buf * kBufCols);
-            float* smax = scr_max + ((s & 1) * 2 + wg) * 4 * 64;
+            float* smax = scr_max + ((s & 1) * kResWG + wg) * 4 * WGC;
             for (int ch = 0; ch < nch; ++ch) {
-                const int cw = min(32, h2 - 32 * ch);
-                const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
+                const int cw = min(kResChunk, cpw - kResChunk * ch);  // 4, 8, 12 or 16
+                const uint32_t col0 = (uint32_t)(c_begin + kResChunk * ch);
                 // ---- B: e = 2^(s*c - m*c) written back over the logits (this warpgroup's
                 // columns only); per-thread column sums of e, then over the warp's lanes
-                float sm[32];
+                float sm[16];
 #pragma unroll
-                for (int c = 0; c < 32; ++c) sm[c] = 0.f;
+                for (int c = 0; c < 16; ++c) sm[c] = 0.f;
                 for (int tl = 0; tl < mt; ++tl) {
-                    float v[32];
+                    float v[16];
                     const uint32_t ta = tbuf + (uint32_t)(tl * scols) + col0;
-                    tmem_ld32(ta, v);
+                    tmem_ld16(ta, v);
                     tmem_wait_ld();
                     const bool ok = lane_valid(tl);
                     const float2 cl2 = make_float2(cl, cl);
 #pragma unroll
-                    for (int c = 0; c < 32; c += 4) {
-                        const float4 m4 = *reinterpret_cast<const float4*>(mcw + 32 * ch + c);
+                    for (int c = 0; c < 16; c += 4) {
+                        const float4 m4 = *reinterpret_cast<const float4*>(mcw + kResChunk * ch + c);
                         const float2 x01 = ffma2(make_float2(v[c], v[c + 1]), cl2, make_float2(m4.x, m4.y));
                         const float2 x23 = ffma2(make_float2(v[c + 2], v[c + 3]), cl2, make_float2(m4.z, m4.w));
                         const float e0 = ok ? ex2(x01.x) : 0.f;
@@ -477,19 +513,19 @@ __global__ void __launch_bounds__(kResThreads, 1)
                         sm[c + 2] = s23.x;
                         sm[c + 3] = s23.y;
                     }
-                    tmem_st_cols(ta, v, cw);
+                    tmem_st_cols16(ta, v, cw);
                 }
-                const float colsum = transpose_sum32(sm, lane);
-                if (lane < cw) ssum[quad * 64 + 32 * ch + lane] = colsum;
+                const float colsum = transpose_sum16(sm, lane);
+                if (lane < cw) ssum[quad * WGC + kResChunk * ch + lane] = colsum;
                 named_bar_sync(wg_bar, 128);
                 // ---- publish (m, l) of columns col0 .. col0+cw-1 to every CTA of the cluster
-                if (quad == 2 && lane < cw) {  // the warpgroup's first warp
-                    const int c = 32 * ch + lane;
+                if (quad == 2 && lane < cw) {  // one warp of the warpgroup
+                    const int c = kResChunk * ch + lane;
                     float m = smax[c], l = ssum[c];
 #pragma unroll
                     for (int q = 1; q < 4; ++q) {
-                        m = fmaxf(m, smax[q * 64 + c]);
-                        l += ssum[q * 64 + c];
+                        m = fmaxf(m, smax[q * WGC + c]);
+                        l += ssum[q * WGC + c];
                     }
                     const int col = c_begin + c;
                     const uint32_t dst = recv_base + (uint32_t)(((slot * (int)csize + (int)rank) * scols + col) * 8);
@@ -505,14 +541,14 @@ __global__ void __launch_bounds__(kResThreads, 1)
             const int buf = nb == 2 ? (s & 1) : 0;
             const int slot = s & (kStatSlots - 1);
             const uint32_t tbuf = tcol + (uint32_t)(buf * kBufCols);
-            const float* smax = scr_max + ((s & 1) * 2 + wg) * 4 * 64;
+            const float* smax = scr_max + ((s & 1) * kResWG + wg) * 4 * WGC;
             // merge the cluster's statistics of this head (rank order) into the
             // column weights w = 2^(m_local*c - b), b = M*c + log2(L); 0 for unused columns
             wait_phase_cluster(BAR(STATS + slot), (uint32_t)(s / kStatSlots) & 1u, ctl);
-            if (wt < 64) {
+            if (wt < WGC) {
                 const int col = c_begin + wt;
                 float wval = 0.f;
-                if (wt < h2 && col < T) {
+                if (wt < cpw && col < T) {
                     const float2* rs = recv + (slot * (int)csize) * scols + col;  // rank r at rs[r * scols]
                     float M = -INFINITY;
                     for (int r = 0; r < (int)csize; ++r) M = fmaxf(M, rs[r * scols].x);
@@ -528,7 +564,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     }
                     float mloc = smax[wt];  // this CTA's column max: the e values' reference
 #pragma unroll
-                    for (int q = 1; q < 4; ++q) mloc = fmaxf(mloc, smax[q * 64 + wt]);
+                    for (int q = 1; q < 4; ++q) mloc = fmaxf(mloc, smax[q * WGC + wt]);
                     wval = mloc == -INFINITY ? 0.f : ex2(fmaf(mloc, cl, -b));
                 }
                 b2w[wt] = wval;
@@ -537,36 +573,36 @@ __global__ void __launch_bounds__(kResThreads, 1)
             // ---- C: per-visual-token sums of e * w over this warpgroup's columns;
             // each slot goes back to the MMA warp after its last chunk is read
             for (int ch = 0; ch < nch; ++ch) {
-                const int cw = min(32, h2 - 32 * ch);
-                const uint32_t col0 = (uint32_t)(c_begin + 32 * ch);
+                const int cw = min(kResChunk, cpw - kResChunk * ch);
+                const uint32_t col0 = (uint32_t)(c_begin + kResChunk * ch);
                 const bool last = ch == nch - 1;
-                float wv[32];
+                float wv[16];
 #pragma unroll
-                for (int c = 0; c < 32; c += 4) {
-                    const float4 w4 = *reinterpret_cast<const float4*>(b2w + 32 * ch + c);
+                for (int c = 0; c < 16; c += 4) {
+                    const float4 w4 = *reinterpret_cast<const float4*>(b2w + kResChunk * ch + c);
                     wv[c] = w4.x;
                     wv[c + 1] = w4.y;
                     wv[c + 2] = w4.z;
                     wv[c + 3] = w4.w;
                 }
-                float va[32], vb[32];
-                if (mt > 0) tmem_ld32(tbuf + col0, va);
+                float va[16], vb[16];
+                if (mt > 0) tmem_ld16(tbuf + col0, va);
                 for (int tl = 0; tl < mt; tl += 2) {
                     tmem_wait_ld();  // va: slot tl
                     if (last) release(buf, tl);
-                    if (tl + 1 < mt) tmem_ld32(tbuf + (uint32_t)((tl + 1) * scols) + col0, vb);
+                    if (tl + 1 < mt) tmem_ld16(tbuf + (uint32_t)((tl + 1) * scols) + col0, vb);
                     float2 a01 = make_float2(0.f, 0.f);
 #pragma unroll
-                    for (int c = 0; c < 32; c += 2)
+                    for (int c = 0; c < 16; c += 2)
                         if (c < cw) a01 = ffma2(make_float2(va[c], va[c + 1]), make_float2(wv[c], wv[c + 1]), a01);
                     accw[tl * kTileRows + vrow] += a01.x + a01.y;
                     if (tl + 1 < mt) {
                         tmem_wait_ld();  // vb: slot tl + 1
                         if (last) release(buf, tl + 1);
-                        if (tl + 2 < mt) tmem_ld32(tbuf + (uint32_t)((tl + 2) * scols) + col0, va);
+                        if (tl + 2 < mt) tmem_ld16(tbuf + (uint32_t)((tl + 2) * scols) + col0, va);
                         a01 = make_float2(0.f, 0.f);
 #pragma unroll
-                        for (int c = 0; c < 32; c += 2)
+                        for (int c = 0; c < 16; c += 2)
                             if (c < cw) a01 = ffma2(make_float2(vb[c], vb[c + 1]), make_float2(wv[c], wv[c + 1]), a01);
                         accw[(tl + 1) * kTileRows + vrow] += a01.x + a01.y;
                     }
@@ -591,18 +627,20 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 back(s);
             }
         }
-        // ---- results: the two warpgroups' partial rows, added in a fixed order
-        named_bar_sync(1, 256);
+        // ---- results: the warpgroups' partial rows, added in a fixed order
+        named_bar_sync(1, 128 * kResWG);
         const float denom = (float)p.hq * (float)T;
-        for (int tl = wg; tl < mt; tl += 2) {
+        for (int tl = wg; tl < mt; tl += kResWG) {
             const int j = (tile_begin + tl) * kTileRows + vrow;
             if (j < N) {
-                const float a = acc_s[tl * kTileRows + vrow] + acc_s[kResMaxSlots * kTileRows + tl * kTileRows + vrow];
+                float a = acc_s[tl * kTileRows + vrow];
+#pragma unroll
+                for (int g = 1; g < kResWG; ++g) a += acc_s[g * kResMaxSlots * kTileRows + tl * kTileRows + vrow];
                 if (!multi) p.out[n0 + j] = a / denom;
                 else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
             }
         }
-        if (multi && !p.defer_fold) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 256, 1, fold_flags);
+        if (multi && !p.defer_fold) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 128 * kResWG, 1, fold_flags);
         tc_fence_before();
     }
 
@@ -673,13 +711,13 @@ int res_capacity(int cluster)
 
 }  // namespace
 
-// Tiles per CTA: the epilogue reads 32 columns per chunk, so the last slot's
-// padded read, (r - 1) * slot_cols + slot_cols / 2 + 32 * chunks, must stay
-// within the 512 TMEM columns (256 per buffer with two head buffers).
+// Tiles per CTA: the epilogue reads 16 columns per chunk, so the last slot's
+// padded read, (r - 1) * slot_cols + res_read_span(slot_cols), must stay within
+// the 512 TMEM columns (256 per buffer with two head buffers).
 int res_max_tiles(int slot_cols, int nb)
 {
     if (slot_cols <= 0) return 0;
-    const int h2 = slot_cols / 2, span = h2 + 32 * ((h2 + 31) / 32);
+    const int span = res_read_span(slot_cols);
     const int cols = nb == 2 ? kBufCols : kResTmemCols;
     int r = nb == 2 ? kBufSlots : kResMaxSlots;
     while (r > 0 && (r - 1) * slot_cols + span > cols) --r;
