@@ -432,6 +432,21 @@ litevlm_status_t litevlm_select_check_device(litevlm_select_t handle, litevlm_st
 litevlm_status_t litevlm_select_set_wait_budget(litevlm_select_t handle, int64_t cycles);
 
 /*
+ * Debug switches of a handle, for tests of the failure path (no counterpart in
+ * the paper). LITEVLM_DEBUG_STALL_SCORE: in the score launches that use the
+ * TMEM-resident kernel (litevlm_select_score_plan reports plan[0] of 2 or 3),
+ * the TMA producer first waits on an mbarrier that nothing completes, so that
+ * wait runs out of the wait budget before any copy or contraction is issued;
+ * every other wait of the launch then gives up as well. The launch writes
+ * invalid scores, and litevlm_select_check_device reports LITEVLM_ERR_TIMEOUT.
+ * Nothing faults, traps or hangs: each wait is bounded by the budget. flags = 0
+ * restores normal operation. Errors: INVALID_ARG for a NULL handle or an
+ * unknown flag.
+ */
+#define LITEVLM_DEBUG_STALL_SCORE 1
+litevlm_status_t litevlm_select_set_debug_flags(litevlm_select_t handle, int32_t flags);
+
+/*
  * litevlm_select_score without a handle and without allocating anything.
  * The paper has no counterpart: this is an integration entry point.
  *

@@ -41,6 +41,7 @@ struct litevlm_select {
     std::string last_error;
     int32_t last_launches = 0;  // kernels the last call on this handle enqueued
     long long wait_budget = lvs::kWaitBudgetCycles;  // clock cycles each device-side wait may take
+    int32_t debug_flags = 0;                         // LITEVLM_DEBUG_* (tests of the failure path)
 };
 
 namespace {
@@ -455,6 +456,7 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
     p.hkv = c.num_kv_heads;
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
     p.wait_budget = h->wait_budget;
+    p.stall = (h->debug_flags & LITEVLM_DEBUG_STALL_SCORE) != 0 && choice.resident;
     p.slot_cols = (max_t + 15) & ~15;
     p.query_last = (c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
     p.extra = nullptr;
@@ -983,6 +985,15 @@ litevlm_status_t litevlm_select_keep_offsets(int32_t batch, const int32_t* seq_o
         run += keep_k_h ? (int64_t)keep_k_h[b] : keep_count_host(n, keep_ratio);
         out_offsets_h[b + 1] = (int32_t)run;
     }
+    return LITEVLM_OK;
+}
+
+litevlm_status_t litevlm_select_set_debug_flags(litevlm_select_t h, int32_t flags)
+{
+    if (!h) return LITEVLM_ERR_INVALID_ARG;
+    h->last_error.clear();
+    if (flags & ~LITEVLM_DEBUG_STALL_SCORE) return fail(h, LITEVLM_ERR_INVALID_ARG, "unknown debug flag");
+    h->debug_flags = flags;
     return LITEVLM_OK;
 }
 

@@ -26,8 +26,8 @@ __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, const 
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
+        if (*c.abort) return false;  // checked before sleeping, so waits after an abort end at once
         if (mbar_try_wait_sleep(bar, parity, kWaitSleepNs)) return true;
-        if (*c.abort) return false;
         if (clock64() - t0 > c.budget) {
             *c.abort = 1;
             atomicOr(c.err, kErrTimeout);
@@ -41,8 +41,8 @@ __device__ __forceinline__ bool wait_phase_cluster(uint32_t bar, uint32_t parity
     if (mbar_try_wait_cluster(bar, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
+        if (*c.abort) return false;  // checked before sleeping, so waits after an abort end at once
         if (mbar_try_wait_cluster_sleep(bar, parity, kWaitSleepNs)) return true;
-        if (*c.abort) return false;
         if (clock64() - t0 > c.budget) {
             *c.abort = 1;
             atomicOr(c.err, kErrTimeout);

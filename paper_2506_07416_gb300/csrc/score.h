@@ -34,6 +34,7 @@ struct ScoreLaunch {
     int32_t defer_fold;       // 1 (with groups > 1): leave the group partials; the top-k kernel adds them
     float c_log2;             // q_scale * k_scale / sqrt(d) * log2(e)
     long long wait_budget;
+    int32_t stall;            // resident kernel: the producer first waits on a barrier nothing completes (tests)
     // [sum T][Hq] normaliser terms of the system and causal text keys (unit of
     // the merged statistic b, from ctx_stats.cu), or null: visual keys only
     const float* extra;

@@ -67,7 +67,7 @@ struct ResLayout {
     static constexpr int ACC_BYTES = kResWG * kResMaxSlots * kTileRows * 4;  // per warpgroup partial rows
     // [max of head s & 1 (2) | sum][wg][quadrant warp][WGC columns]
     static constexpr int SCR_BYTES = 3 * kResWG * 4 * WGC * 4;
-    static constexpr int NBAR_FIXED = 2 * 2 + 2 * kResMaxSlots + kStatSlots + 1;
+    static constexpr int NBAR_FIXED = 2 * 2 + 2 * kResMaxSlots + kStatSlots + 2;
     static constexpr int FIXED = 2 * Q_BYTES + ACC_BYTES + SCR_BYTES + kStatSlots * RECV_COLS * 8 +
                                  2 * kResWG * WGC * 4 + kResMaxSlots * 4 + (NBAR_FIXED + 2 * 10) * 8 + 64 + 1024;
     static constexpr int STAGES_FIT = (227 * 1024 - FIXED) / TILE_BYTES;
@@ -200,7 +200,8 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const uint32_t bar0 = base + L::OFF_BAR;
     auto BAR = [&](int i) -> uint32_t { return bar0 + 8u * (uint32_t)i; };
     const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + 2, S_FULL = Q_EMPTY + 2,
-              S_EMPTY = S_FULL + kResMaxSlots, STATS = S_EMPTY + kResMaxSlots, DRAIN = STATS + kStatSlots;
+              S_EMPTY = S_FULL + kResMaxSlots, STATS = S_EMPTY + kResMaxSlots, DRAIN = STATS + kStatSlots,
+              STALL = DRAIN + 1;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
     float* acc_s = reinterpret_cast<float*>(smem + L::OFF_ACC);
@@ -227,6 +228,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
             mbar_init(BAR(S_EMPTY + i), 4 * kResWG);  // one arrival per epilogue warp
         }
         mbar_init(BAR(DRAIN), 2);
+        mbar_init(BAR(STALL), 1);  // nothing ever arrives (the debug stall below)
         *abort_flag = 0;
         fence_mbar_init_cluster();
     }
@@ -273,11 +275,16 @@ __global__ void __launch_bounds__(kResThreads, 1)
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0 && mt > 0) {
+            // Debug stall (p.stall, a test of the failure path): wait on a barrier
+            // that nothing completes before issuing any copy, so this wait runs out
+            // of budget, and every other wait of the launch runs out or sees the
+            // abort flag, with no copy or contraction in flight.
+            // Nothing is issued after the stall ran out.
+            bool ok = !p.stall || wait_phase(BAR(STALL), 0, ctl);
             uint32_t ks = 0, kph = 0;
             int k_issued[kStages];
             int q_issued[2] = {0, 0};
             for (int s = 0; s < kStages; ++s) k_issued[s] = 0;
-            bool ok = true;
             for (int s = 0; s < hpg && ok; ++s) {
                 const int h = hg * hpg + s;
                 const int g = h / G;
@@ -410,7 +417,9 @@ __global__ void __launch_bounds__(kResThreads, 1)
             const int slot = s & (kStatSlots - 1);
             const uint32_t tbuf = tcol + (uint32_t)(buf * kBufCols);
             float* smax = scr_max + ((s & 1) * kResWG + wg) * 4 * WGC;
-            if (et == 0) mbar_arrive_expect_tx(BAR(STATS + slot), (uint32_t)(csize * n2 * 8));
+            // (not after an abort: that phase would never complete, and arming it
+            // again four heads later would arrive twice on it)
+            if (et == 0 && !*abort_flag) mbar_arrive_expect_tx(BAR(STATS + slot), (uint32_t)(csize * n2 * 8));
             for (int ch = 0; ch < nch; ++ch) {
                 const uint32_t col0 = (uint32_t)(c_begin + kResChunk * ch);
                 // ---- A: column maxima, per thread over its slots, then over the lanes
@@ -519,7 +528,9 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 if (lane < cw) ssum[quad * WGC + kResChunk * ch + lane] = colsum;
                 named_bar_sync(wg_bar, 128);
                 // ---- publish (m, l) of columns col0 .. col0+cw-1 to every CTA of the cluster
-                if (quad == 2 && lane < cw) {  // one warp of the warpgroup
+                // (not after an abort: the peers may not be waiting for it, and no
+                // statistic is left in flight when the CTA exits)
+                if (quad == 2 && lane < cw && !*abort_flag) {  // one warp of the warpgroup
                     const int c = kResChunk * ch + lane;
                     float m = smax[c], l = ssum[c];
 #pragma unroll

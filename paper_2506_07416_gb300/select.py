@@ -67,9 +67,10 @@ def _load():
     lib.litevlm_select_score_noalloc.argtypes = [i32, i32, i32, i32, i32, P, P, P, P, P, P, f32, f32, P, P, P]
     lib.litevlm_select_keep_offsets.argtypes = [i32, P, P, f32, P]
     lib.litevlm_select_set_wait_budget.argtypes = [P, i64]
+    lib.litevlm_select_set_debug_flags.argtypes = [P, i32]
     for fn in ("create", "destroy", "score", "score_full_keys", "topk", "compact", "check_device", "score_plan",
                "score_noalloc", "splice", "views", "fold_norm", "rope_table", "project", "score_topk", "host_view",
-               "keep_offsets", "set_wait_budget"):
+               "keep_offsets", "set_wait_budget", "set_debug_flags"):
         getattr(lib, "litevlm_select_" + fn).restype = ctypes.c_int
     return lib
 
@@ -83,7 +84,7 @@ EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_la
            "litevlm_select_splice", "litevlm_select_score_full_keys", "litevlm_select_views",
            "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project",
            "litevlm_select_last_launches", "litevlm_select_score_topk", "litevlm_select_host_view",
-           "litevlm_select_keep_offsets", "litevlm_select_set_wait_budget"]
+           "litevlm_select_keep_offsets", "litevlm_select_set_wait_budget", "litevlm_select_set_debug_flags"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)"}
@@ -255,6 +256,14 @@ def keep_offsets(seq_offsets_h, keep_k_h=None, keep_ratio: float = 0.0) -> np.nd
 def set_wait_budget(handle: int, cycles: int) -> None:
     """litevlm_select_set_wait_budget: clock cycles each device-side wait may take (0: default)."""
     _check(LIB.litevlm_select_set_wait_budget(handle, int(cycles)), handle)
+
+
+DEBUG_STALL_SCORE = 1
+
+
+def set_debug_flags(handle: int, flags: int) -> None:
+    """litevlm_select_set_debug_flags: switches for tests of the failure path (0: off)."""
+    _check(LIB.litevlm_select_set_debug_flags(handle, int(flags)), handle)
 
 
 def score_noalloc(num_q_heads: int, num_kv_heads: int, head_dim: int, qk_dtype: str, batch: int, q_text,
@@ -458,6 +467,9 @@ class Selector:
 
     def set_wait_budget(self, cycles: int) -> None:
         set_wait_budget(self.handle, cycles)
+
+    def set_debug_flags(self, flags: int) -> None:
+        set_debug_flags(self.handle, flags)
 
     def score_plan(self, text_offsets_h, seq_offsets_h):
         so = _host_i32(seq_offsets_h)

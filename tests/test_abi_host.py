@@ -145,3 +145,7 @@ def test_keep_offsets_rejects_bad_arguments_and_leaves_the_output(sel):
 
 def test_wait_budget_setter_needs_a_handle(sel):
     assert sel.LIB.litevlm_select_set_wait_budget(None, 100) == 1
+
+
+def test_debug_flags_setter_needs_a_handle(sel):
+    assert sel.LIB.litevlm_select_set_debug_flags(None, 0) == 1
