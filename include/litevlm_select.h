@@ -74,6 +74,8 @@ typedef enum {
 #define LITEVLM_FLAG_SCORE_RESIDENT 2 /* use the TMEM-resident kernel whenever the shapes allow it */
 #define LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER 8 /* the same, with one TMEM head buffer only (no head overlap) */
 #define LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS 16 /* the same, two TMEM head buffers where the shapes allow it */
+#define LITEVLM_FLAG_SCORE_RESIDENT_FLAT 64 /* the same, one buffer, with the flattened (request, head) schedule
+                                               whenever every request has the same token counts */
 /* OR-ed with at most one of the above: only the last text token of each request
  * is a query, T_b counts as 1 in the mean (the last-token variant of attention-
  * score pruning, Related Work / FastV). Requests may then have more than 128
@@ -402,9 +404,14 @@ litevlm_status_t litevlm_select_splice(litevlm_select_t handle, int32_t batch, c
  * device work; the occupancy of a kernel variant is queried once per handle).
  * plan[0] = kernel (1: K re-read per pass; 2: logits resident in tensor
  * memory, one head at a time; 3: the same with two heads in tensor memory, so
- * one head's epilogue overlaps the next head's MMAs and statistics exchange),
+ * one head's epilogue overlaps the next head's MMAs and statistics exchange;
+ * 4: as 2, with a flattened schedule, for batches whose requests all have the
+ * same visual and text token counts: the batch's (request, head) pairs are
+ * split evenly over every cluster that fits on the GPU at once, each cluster
+ * running its share back to back across request boundaries),
  * plan[1] = CTAs per thread-block cluster, plan[2] = 128-token tiles per CTA,
- * plan[3] = query-head groups (grid y). plan holds 4 int32.
+ * plan[3] = query-head groups (grid y), or the number of clusters for plan[0]
+ * = 4. plan holds 4 int32.
  * Errors as for litevlm_select_score's host-side checks.
  */
 litevlm_status_t litevlm_select_score_plan(litevlm_select_t handle, int32_t batch, const int32_t* text_offsets_h,
@@ -434,7 +441,7 @@ litevlm_status_t litevlm_select_set_wait_budget(litevlm_select_t handle, int64_t
 /*
  * Debug switches of a handle, for tests of the failure path (no counterpart in
  * the paper). LITEVLM_DEBUG_STALL_SCORE: in the score launches that use the
- * TMEM-resident kernel (litevlm_select_score_plan reports plan[0] of 2 or 3),
+ * TMEM-resident kernel (litevlm_select_score_plan reports plan[0] of 2, 3 or 4),
  * the TMA producer first waits on an mbarrier that nothing completes, so that
  * wait runs out of the wait budget before any copy or contraction is issued;
  * every other wait of the launch then gives up as well. The launch writes
@@ -460,7 +467,9 @@ litevlm_status_t litevlm_select_set_debug_flags(litevlm_select_t handle, int32_t
  * Same computation, arguments and host-side checks as litevlm_select_score.
  * A handle's config is replaced by num_q_heads, num_kv_heads, head_dim and
  * qk_dtype, with the same rules as in litevlm_select_create. The kernel and
- * launch shape are chosen as litevlm_select_score would choose them.
+ * launch shape are chosen as litevlm_select_score would choose them, except
+ * that the flattened schedule (plan[0] = 4) is never used here: its partial
+ * rows could exceed the static scratch.
  *
  * Scratch: two static device arrays in this library, one per device:
  * 4 MiB of partial scores and 64 KiB of fold tickets.

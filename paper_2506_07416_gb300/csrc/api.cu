@@ -42,6 +42,7 @@ struct litevlm_select {
     int32_t last_launches = 0;  // kernels the last call on this handle enqueued
     long long wait_budget = lvs::kWaitBudgetCycles;  // clock cycles each device-side wait may take
     int32_t debug_flags = 0;                         // LITEVLM_DEBUG_* (tests of the failure path)
+    bool allow_flat = true;  // the resident kernel's flattened schedule may be chosen (not in the no-alloc path)
 };
 
 namespace {
@@ -120,8 +121,20 @@ struct ScoreChoice {
 // its K tiles need at the CTA's share of HBM bandwidth. Waves of CTAs come from the measured
 // cluster occupancy of the kernel. The re-read kernel streams every K tile
 // twice (weight 1.6).
+// True when every request has the same, non-zero, visual and text token
+// counts (the resident kernel's flattened schedule needs it).
+bool uniform_batch(int batch, const int32_t* seq_offsets_h, const int32_t* text_offsets_h)
+{
+    if (batch < 2) return false;
+    const int32_t n = seq_offsets_h[1] - seq_offsets_h[0], t = text_offsets_h[1] - text_offsets_h[0];
+    if (n <= 0 || t <= 0) return false;
+    for (int32_t b = 1; b < batch; ++b)
+        if (seq_offsets_h[b + 1] - seq_offsets_h[b] != n || text_offsets_h[b + 1] - text_offsets_h[b] != t) return false;
+    return true;
+}
+
 ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* seq_offsets_h, int max_t, int row_bytes,
-                                bool fp8)
+                                bool fp8, bool uniform = false)
 {
     const litevlm_select_config_t& c = h->cfg;
     const int hq = c.num_q_heads;
@@ -144,6 +157,7 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* se
     mix((uint64_t)c.num_kv_heads);
     mix((uint64_t)row_bytes);
     mix((uint64_t)c.flags);
+    mix((uint64_t)(uniform && h->allow_flat));
     for (int b = 0; b < batch; ++b) mix((uint64_t)td[b]);
     for (const auto& m : h->plan_memo)
         if (m.used && m.key == key) return ScoreChoice{m.resident, m.plan};
@@ -162,10 +176,11 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* se
     const int kflags = c.flags & ~LITEVLM_FLAG_QUERY_LAST_TOKEN;
     if (kflags != LITEVLM_FLAG_SCORE_REREAD) {
         if (kflags == LITEVLM_FLAG_SCORE_RESIDENT || kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
-            kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS)
+            kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS || kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT)
             best_cost = 1e300;
         for (int nb = 1; nb <= 2; ++nb) {
-            if (nb == 2 && kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER) continue;
+            if (nb == 2 && (kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER || kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT))
+                continue;
             if (nb == 1 && kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) continue;
             const int R = lvs::res_max_tiles(slot_cols, nb);
             for (int cl = 1; cl <= cmax; ++cl) {
@@ -202,6 +217,40 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* se
                         best = ScoreChoice{true, pl};
                     }
                 }
+            }
+        }
+    }
+    // Flattened schedule (every request the same size, one TMEM head buffer):
+    // the batch's (request, head) pairs split evenly over every cluster that
+    // fits on the GPU at once, so there is no partial last wave; the clusters
+    // run their pairs back to back and each request boundary costs a write of
+    // the request's rows (a fold where a request spans two clusters).
+    if (uniform && h->allow_flat && kflags != LITEVLM_FLAG_SCORE_REREAD &&
+        kflags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) {
+        const int R = lvs::res_max_tiles(slot_cols, 1);
+        const long long pairs = (long long)batch * hq;
+        for (int cl = 1; cl <= cmax; ++cl) {
+            const int tpc = (max_tiles + cl - 1) / cl;
+            if (tpc > R) continue;
+            if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;
+            int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
+            if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
+            if (cap <= 0) continue;
+            long long nclu = cap / cl;
+            if (nclu > pairs) nclu = pairs;
+            if (nclu > lvs::kFlatMax) nclu = lvs::kFlatMax;
+            if (nclu < 1) continue;
+            const double per_head = (double)tpc + (cl > 1 ? 1.0 : 0.25);
+            const long long per_cluster = (pairs + nclu - 1) / nclu;
+            const double boundaries = (double)per_cluster / hq + 1.0;
+            double cost = 6.0 + (double)per_cluster * per_head + 2.0 * boundaries;
+            if (kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT) cost -= 1e200;  // forced: any flat plan beats the others
+            if (cost < best_cost - 1e-9) {
+                best_cost = cost;
+                lvs::ScorePlan pl{cl, tpc, 1};
+                pl.res_nb = 1;
+                pl.flat = (int)nclu;
+                best = ScoreChoice{true, pl};
             }
         }
     }
@@ -256,7 +305,7 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
     const int kflags = c->flags & ~LITEVLM_FLAG_QUERY_LAST_TOKEN;
     if (c->flags < 0 || (kflags != 0 && kflags != LITEVLM_FLAG_SCORE_REREAD && kflags != LITEVLM_FLAG_SCORE_RESIDENT &&
                          kflags != LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER &&
-                         kflags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS))
+                         kflags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS && kflags != LITEVLM_FLAG_SCORE_RESIDENT_FLAT))
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "flags must be 0 or one LITEVLM_FLAG_SCORE_* value");
     if (c->head_dim <= 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "head_dim must be > 0");
     if (!lvs::score_shape_supported(c->head_dim, c->qk_dtype == LITEVLM_FP8_E4M3))
@@ -377,11 +426,12 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, co
     plan[0] = plan[1] = plan[2] = plan[3] = 0;
     if (batch == 0 || sh.tot_n == 0) return LITEVLM_OK;
     const bool fp8 = h->cfg.qk_dtype == LITEVLM_FP8_E4M3;
-    const ScoreChoice ch = choose_score_kernel(h, batch, seq_offsets_h, sh.max_t, h->cfg.head_dim * (fp8 ? 1 : 2), fp8);
-    plan[0] = ch.resident ? 1 + ch.plan.res_nb : 1;
+    const ScoreChoice ch = choose_score_kernel(h, batch, seq_offsets_h, sh.max_t, h->cfg.head_dim * (fp8 ? 1 : 2), fp8,
+                                               uniform_batch(batch, seq_offsets_h, text_offsets_h));
+    plan[0] = !ch.resident ? 1 : ch.plan.flat > 0 ? 4 : 1 + ch.plan.res_nb;
     plan[1] = ch.plan.cluster;
     plan[2] = ch.plan.tiles_per_cta;
-    plan[3] = ch.plan.groups;
+    plan[3] = ch.plan.flat > 0 ? ch.plan.flat : ch.plan.groups;
     return LITEVLM_OK;
 }
 
@@ -432,7 +482,8 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
         if (!aligned16(ctx->k_text) || (ctx->k_sys && !aligned16(ctx->k_sys)))
             return fail(h, LITEVLM_ERR_INVALID_ARG, "k_sys and k_text must be 16-byte aligned");
     }
-    const ScoreChoice choice = choose_score_kernel(h, batch, seq_offsets_h, max_t, row_bytes, fp8);
+    const ScoreChoice choice = choose_score_kernel(h, batch, seq_offsets_h, max_t, row_bytes, fp8,
+                                                   uniform_batch(batch, seq_offsets_h, text_offsets_h));
     const lvs::ScorePlan& plan = choice.plan;
     if (plan.tiles_per_cta > lvs::kMaxTilesPerCta)
         return fail(h, LITEVLM_ERR_UNSUPPORTED, "request too long for one cluster");
@@ -1149,6 +1200,7 @@ extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, in
         h.plan_memo_next = d.plan_memo_next[fam];
     }
     h.err_d = err_d;
+    h.allow_flat = false;  // its partial rows could exceed the static scratch
     h.cfg.max_batch = batch;
     h.cfg.max_total_visual = tot_n;
     h.cfg.max_total_text = text_offsets_h[batch] > 0 ? text_offsets_h[batch] : 0;

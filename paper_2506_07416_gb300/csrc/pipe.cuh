@@ -138,19 +138,21 @@ __device__ __forceinline__ float merge_cluster_row(uint32_t my_addr, uint32_t cs
 __device__ __forceinline__ int fold_ticket_index(int b, int n0, int t) { return n0 / kTileRows + t + b; }
 
 // After a CTA wrote its partial rows (head group hg) for tiles [tile_begin,
-// tile_begin + mt): take one ticket per tile; the last of the `groups` CTAs
-// that own a tile adds the group partials of that tile in index order and
-// writes the scores. `nthreads` threads (ids 0..nthreads-1, synchronised by
+// tile_begin + mt): take one ticket per tile; the last of the `parts` CTAs
+// (default: the head groups) that own a tile adds the partials of that tile
+// in index order and writes the scores. `nthreads` threads (ids 0..nthreads-1, synchronised by
 // named barrier `bar_id`) take part; `flags` is shared memory for mt ints.
 __device__ __forceinline__ void fold_tiles(const ScoreLaunch& p, int b, int n0, int N, int T, int tile_begin,
-                                           int mt, int tid, int nthreads, uint32_t bar_id, volatile int* flags)
+                                           int mt, int tid, int nthreads, uint32_t bar_id, volatile int* flags,
+                                           int parts = 0)
 {
+    if (parts <= 0) parts = p.groups;  // partial rows of this request (head groups, or clusters of a flat launch)
     __threadfence();
     named_bar_sync(bar_id, nthreads);
     for (int tl = tid; tl < mt; tl += nthreads) {
         int* c = p.counters + fold_ticket_index(b, n0, tile_begin + tl);
         const int ticket = atomicAdd(c, 1);
-        const int last = ticket == p.groups - 1;
+        const int last = ticket == parts - 1;
         if (last) *c = 0;  // ready for the next launch
         flags[tl] = last;
     }
@@ -166,13 +168,13 @@ __device__ __forceinline__ void fold_tiles(const ScoreLaunch& p, int b, int n0, 
         if (j >= N) continue;
         const float* src = p.partials + n0 + j;
         float sum = 0.f;
-        for (int g = 0; g < p.groups; g += 16) {
+        for (int g = 0; g < parts; g += 16) {
             float v[16];
 #pragma unroll
-            for (int q = 0; q < 16; ++q) v[q] = g + q < p.groups ? __ldcg(src + (int64_t)(g + q) * p.total_vis) : 0.f;
+            for (int q = 0; q < 16; ++q) v[q] = g + q < parts ? __ldcg(src + (int64_t)(g + q) * p.total_vis) : 0.f;
 #pragma unroll
             for (int q = 0; q < 16; ++q)
-                if (g + q < p.groups) sum += v[q];
+                if (g + q < parts) sum += v[q];
         }
         p.out[n0 + j] = sum / denom;
     }

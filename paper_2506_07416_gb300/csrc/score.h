@@ -15,6 +15,7 @@ constexpr int kMaxTilesPerCta = 32;      // score tiles one CTA may own
 constexpr int kMaxCluster = 16;
 constexpr int kOrderMax = 2048;          // batches up to this size are launched largest request first
 constexpr int kOffsetsByValue = 64;      // batches up to this size carry their offsets in the launch parameters
+constexpr int kFlatMax = 160;            // clusters of a flattened resident launch (at least one per SM pair)
 
 struct ScoreLaunch {
     const int32_t* seq_off;   // device [batch+1]
@@ -51,6 +52,13 @@ struct ScoreLaunch {
     // k % groups. order_n == 0: requests in index order.
     int32_t order_n;
     uint16_t order[kOrderMax];
+    // Flattened schedule of the resident kernel (flat_n > 0; every request has
+    // the same visual and text token counts): the batch's (request, head) pairs
+    // in request-major order, cluster k taking pairs [flat_r[k], flat_r[k+1]);
+    // a request whose heads span several clusters is folded from their partial
+    // rows (part = cluster - first cluster of the request).
+    int32_t flat_n;
+    int32_t flat_r[kFlatMax + 1];
 };
 
 struct ScorePlan {
@@ -58,6 +66,7 @@ struct ScorePlan {
     int tiles_per_cta;
     int groups;               // head groups (grid.y); partial rows when > 1
     int res_nb = 1;           // resident kernel: TMEM head buffers
+    int flat = 0;             // resident kernel: clusters of the flattened (request, head) schedule, 0: none
 };
 
 // Host helpers (score_tc.cu)

@@ -170,10 +170,17 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = cluster_ctarank();
     const uint32_t csize = cluster_nctarank();
-    const int item = (int)(blockIdx.x / csize);  // this cluster's (request, head group)
-    const int req_i = item / p.groups;
-    const int b = p.order_n > 0 ? (int)p.order[req_i] : req_i;
-    const int hg = item - req_i * p.groups;
+    // This cluster's work: one (request, head group), or with a flattened
+    // schedule the pairs [fr0, fr0 + nheads) of the request-major list of
+    // (request, head) pairs, which may cross request boundaries (all requests
+    // then have the same token counts); b is the first request.
+    const int item = (int)(blockIdx.x / csize);
+    const bool flat = p.flat_n > 0;
+    const int fr0 = flat ? p.flat_r[item] : 0;
+    const int nheads = flat ? p.flat_r[item + 1] - fr0 : p.heads_per_group;
+    const int req_i = flat ? 0 : item / p.groups;
+    const int b = flat ? fr0 / p.hq : (p.order_n > 0 ? (int)p.order[req_i] : req_i);
+    const int hg = flat ? 0 : item - req_i * p.groups;
 
     // With the full-key-set terms (p.extra, written by the kernel launched just
     // before this one) only the threads that read them wait for that kernel,
@@ -254,7 +261,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
 
     const ResShape shp = res_shape<L::RECV_COLS>(p, n0, n1, tq, t1, rank, csize, MROWS);
     const int N = shp.N, t0 = shp.t0, T = shp.T, n2 = shp.n2, nb = shp.nb;
-    const bool bad_shape = shp.bad;  // uniform for the whole cluster (same request)
+    const bool bad_shape = shp.bad || (flat && nb != 1);  // uniform for the whole cluster
     if (bad_shape || N <= 0) {
         if (p.extra) griddep_wait();
         if (bad_shape && threadIdx.x == 0 && rank == 0 && hg == 0) atomicOr(p.err, kErrShape);
@@ -271,6 +278,18 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const int tile_begin = shp.tile_begin;
     const int tile_end = tile_begin + shp.mt;
     const int mt = shp.mt;
+    // request, query head, first visual row and first query row of head s of
+    // this CTA's sequence (with a flattened schedule the requests' rows follow
+    // one another at equal strides)
+    struct HeadRef {
+        int b, h, n0, t0;
+    };
+    const int t_stride = t1 - tq;
+    auto head_of = [&](int s_) -> HeadRef {
+        if (!flat) return HeadRef{b, hg * hpg + s_, n0, t0};
+        const int rh = fr0 + s_, bb = rh / p.hq;
+        return HeadRef{bb, rh - bb * p.hq, n0 + (bb - b) * N, t0 + (bb - b) * t_stride};
+    };
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
@@ -285,8 +304,9 @@ __global__ void __launch_bounds__(kResThreads, 1)
             int k_issued[kStages];
             int q_issued[2] = {0, 0};
             for (int s = 0; s < kStages; ++s) k_issued[s] = 0;
-            for (int s = 0; s < hpg && ok; ++s) {
-                const int h = hg * hpg + s;
+            for (int s = 0; s < nheads && ok; ++s) {
+                const HeadRef hr = head_of(s);
+                const int h = hr.h;
                 const int g = h / G;
                 const int qb = s & 1;
                 if (!wait_phase(BAR(Q_EMPTY + qb), ((s >> 1) & 1) ^ 1, ctl)) break;
@@ -294,7 +314,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 const uint32_t qdst = base + L::OFF_Q + qb * L::Q_BYTES;
 #pragma unroll
                 for (int kb = 0; kb < L::KB; ++kb)
-                    tma_load_3d(qdst + kb * MROWS * 128, &tm_q, BAR(Q_FULL + qb), kb * ELEMS_PER_KB, h, t0);
+                    tma_load_3d(qdst + kb * MROWS * 128, &tm_q, BAR(Q_FULL + qb), kb * ELEMS_PER_KB, h, hr.t0);
                 ++q_issued[qb];
                 for (int t = tile_begin; t < tile_end; ++t) {
                     if (!wait_phase(BAR(K_EMPTY + ks), kph ^ 1, ctl)) { ok = false; break; }
@@ -303,7 +323,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
 #pragma unroll
                     for (int kb = 0; kb < L::KB; ++kb)
                         tma_load_3d(kdst + kb * kTileRows * 128, &tm_k, BAR(K_FULL + ks), kb * ELEMS_PER_KB, g,
-                                    n0 + t * kTileRows);
+                                    hr.n0 + t * kTileRows);
                     ++k_issued[ks];
                     if (++ks == kStages) { ks = 0; kph ^= 1; }
                 }
@@ -333,7 +353,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
             if (mt > 0) {
                 const uint32_t idesc = idesc_make(128, (uint32_t)n2, FMT);
                 bool ok = true;
-                for (int s = 0; s < hpg && ok; ++s) {
+                for (int s = 0; s < nheads && ok; ++s) {
                     const int qb = s & 1;
                     const int buf = nb == 2 ? (s & 1) : 0;
                     const uint32_t use = nb == 2 ? (uint32_t)(s >> 1) : (uint32_t)s;  // earlier heads in this buffer
@@ -571,7 +591,8 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     float b = fmaf(M, cl, __log2f(Ls));
                     if (p.extra) {
                         griddep_wait();
-                        b = log2_add(b, p.extra[(int64_t)(t0 + col) * p.hq + hg * hpg + s]);
+                        const HeadRef hr = head_of(s);
+                        b = log2_add(b, p.extra[(int64_t)(hr.t0 + col) * p.hq + hr.h]);
                     }
                     float mloc = smax[wt];  // this CTA's column max: the e values' reference
 #pragma unroll
@@ -625,33 +646,72 @@ __global__ void __launch_bounds__(kResThreads, 1)
         // A of head i, then C of head i - 1 (its statistics travelled during A),
         // which frees the other buffer so the MMAs of head i + 1 run under B of
         // head i.
+        const float denom = (float)p.hq * (float)T;
+        // Flattened schedule: the scores of request hr.b, whose last head in this
+        // cluster's range has been through C. All of its heads in the range:
+        // final scores; otherwise this cluster's partial rows, folded by the last
+        // of the request's clusters to finish each tile (fixed part order).
+        auto flush = [&](const HeadRef& hr) {
+            const int first = hr.b * p.hq, last = first + p.hq - 1;
+            const bool whole = first >= fr0 && last < fr0 + nheads;
+            auto cluster_of = [&](int pair) {  // the cluster whose range holds the pair
+                int lo = 0, hi = p.flat_n - 1;
+                while (lo < hi) {
+                    const int mid = (lo + hi + 1) >> 1;
+                    if (p.flat_r[mid] <= pair) lo = mid;
+                    else hi = mid - 1;
+                }
+                return lo;
+            };
+            const int cf = whole ? item : cluster_of(first);
+            const int parts = whole ? 1 : cluster_of(last) - cf + 1;
+            named_bar_sync(1, 128 * kResWG);  // every warpgroup's C contributions are in place
+            for (int tl = wg; tl < mt; tl += kResWG) {
+                const int j = (tile_begin + tl) * kTileRows + vrow;
+                if (j < N) {
+                    float a = acc_s[tl * kTileRows + vrow];
+#pragma unroll
+                    for (int g = 1; g < kResWG; ++g) a += acc_s[g * kResMaxSlots * kTileRows + tl * kTileRows + vrow];
+                    if (whole) p.out[hr.n0 + j] = a / denom;
+                    else p.partials[(int64_t)(item - cf) * p.total_vis + hr.n0 + j] = a;
+                }
+            }
+            named_bar_sync(1, 128 * kResWG);  // every row is read before it is cleared
+            for (int tl = 0; tl < mt; ++tl) accw[tl * kTileRows + vrow] = 0.f;
+            if (!whole) fold_tiles(p, hr.b, hr.n0, N, T, tile_begin, mt, et, 128 * kResWG, 1, fold_flags, parts);
+        };
         if (nb == 2) {
-            for (int it = 0; it <= hpg; ++it) {
-                if (it < hpg) front_a(it);
+            for (int it = 0; it <= nheads; ++it) {
+                if (it < nheads) front_a(it);
                 if (it >= 1) back(it - 1);
-                if (it < hpg) front_b(it);
+                if (it < nheads) front_b(it);
             }
         } else {
-            for (int s = 0; s < hpg; ++s) {
+            for (int s = 0; s < nheads; ++s) {
                 front_a(s);
                 front_b(s);
                 back(s);
+                if (flat) {
+                    const HeadRef hr = head_of(s);
+                    if (s == nheads - 1 || hr.h == p.hq - 1) flush(hr);
+                }
             }
         }
         // ---- results: the warpgroups' partial rows, added in a fixed order
-        named_bar_sync(1, 128 * kResWG);
-        const float denom = (float)p.hq * (float)T;
-        for (int tl = wg; tl < mt; tl += kResWG) {
-            const int j = (tile_begin + tl) * kTileRows + vrow;
-            if (j < N) {
-                float a = acc_s[tl * kTileRows + vrow];
+        if (!flat) {
+            named_bar_sync(1, 128 * kResWG);
+            for (int tl = wg; tl < mt; tl += kResWG) {
+                const int j = (tile_begin + tl) * kTileRows + vrow;
+                if (j < N) {
+                    float a = acc_s[tl * kTileRows + vrow];
 #pragma unroll
-                for (int g = 1; g < kResWG; ++g) a += acc_s[g * kResMaxSlots * kTileRows + tl * kTileRows + vrow];
-                if (!multi) p.out[n0 + j] = a / denom;
-                else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
+                    for (int g = 1; g < kResWG; ++g) a += acc_s[g * kResMaxSlots * kTileRows + tl * kTileRows + vrow];
+                    if (!multi) p.out[n0 + j] = a / denom;
+                    else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
+                }
             }
+            if (multi && !p.defer_fold) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 128 * kResWG, 1, fold_flags);
         }
-        if (multi && !p.defer_fold) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, 128 * kResWG, 1, fold_flags);
         tc_fence_before();
     }
 
@@ -682,7 +742,8 @@ cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const S
     cudaError_t e = res_prepare<ROW_BYTES, FP8, MROWS>(plan.cluster);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(plan.cluster * plan.groups * batch), 1, 1);
+    const int items = plan.flat > 0 ? plan.flat : plan.groups * batch;
+    cfg.gridDim = dim3((unsigned)(plan.cluster * items), 1, 1);
     cfg.blockDim = dim3(kResThreads, 1, 1);
     cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS>::ALLOC;
     cfg.stream = stream;
@@ -760,6 +821,14 @@ cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm
     q.groups = plan.groups;
     q.heads_per_group = p.hq / plan.groups;
     q.ctas_per_request = plan.cluster * plan.groups;
+    q.flat_n = 0;
+    if (plan.flat > 0) {  // equal shares of the batch's (request, head) pairs, in request-major order
+        if (plan.flat > kFlatMax || plan.res_nb != 1) return cudaErrorInvalidValue;
+        const long long pairs = (long long)batch * p.hq;
+        q.flat_n = plan.flat;
+        for (int k = 0; k <= plan.flat; ++k) q.flat_r[k] = (int32_t)(pairs * k / plan.flat);
+        q.order_n = 0;
+    }
     if (fp8)
         return mrows == 64 ? res_launch<128, true, 64>(tm_q, tm_k, q, plan, batch, stream)
                            : res_launch<128, true, 128>(tm_q, tm_k, q, plan, batch, stream);

@@ -85,9 +85,11 @@ EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_la
            "litevlm_select_fold_norm", "litevlm_select_rope_table", "litevlm_select_project",
            "litevlm_select_last_launches", "litevlm_select_score_topk", "litevlm_select_host_view",
            "litevlm_select_keep_offsets", "litevlm_select_set_wait_budget", "litevlm_select_set_debug_flags"]
-FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16}
+FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16, "resident_flat": 64}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
-           3: "score_res (logits resident in TMEM, two heads overlapped)"}
+           3: "score_res (logits resident in TMEM, two heads overlapped)",
+           4: "score_res (logits resident in TMEM, one head at a time, flattened (request, head) schedule over "
+              "every cluster that fits at once)"}
 
 
 def _check(rc: int, handle) -> None:
