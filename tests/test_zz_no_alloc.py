@@ -94,3 +94,34 @@ def test_noalloc_matches_the_oracle(sel):
     assert int(err.item()) == 0
     o = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, w.dtype)
     assert_scores_close(out.cpu().numpy(), o, w.dtype)
+
+
+@pytest.mark.gpu
+def test_noalloc_rejects_head_groups_beyond_the_partial_scratch(sel):
+    """Limit 2: a launch that splits the query heads over G > 1 groups needs G x
+    total_visual partial scores; beyond the static 1048576 floats the call
+    returns WORKSPACE, enqueues nothing and leaves the output as it was."""
+    if not torch.cuda.is_available():
+        pytest.fail("the GPU tests need a CUDA device")
+    found = None
+    for n, t, hq, hkv in ((65536, 64, 32, 32), (60000, 128, 28, 4), (50000, 16, 16, 16), (65536, 128, 32, 8)):
+        so = np.array([0, n], np.int32)
+        to = np.array([0, t], np.int32)
+        s = sel.Selector(1, n, t, hq, hkv, 128, "bf16")
+        plan = s.score_plan(to, so)
+        s.close()
+        if plan[0] != 4 and plan[3] > 1 and plan[3] * n > (1 << 20):
+            found = (n, t, hq, hkv, so, to)
+            break
+    assert found is not None, "no shape among the candidates splits its heads beyond the scratch"
+    n, t, hq, hkv, so, to = found
+    q = torch.zeros((t, hq, 128), dtype=torch.bfloat16, device="cuda")
+    k = torch.zeros((n, hkv, 128), dtype=torch.bfloat16, device="cuda")
+    so_d, to_d = torch.from_numpy(so).cuda(), torch.from_numpy(to).cuda()
+    out = torch.full((n,), float("nan"), dtype=torch.float32, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    with pytest.raises(sel.LitevlmError) as ei:
+        sel.score_noalloc(hq, hkv, 128, "bf16", 1, q, to_d, to, k, so_d, so, 1.0, 1.0, out, err)
+    assert ei.value.name == "WORKSPACE"
+    torch.cuda.synchronize()
+    assert bool(torch.isnan(out).all()) and int(err.item()) == 0
