@@ -54,8 +54,13 @@ constexpr int kResMaxSlots = 16;
 constexpr int kBufSlots = kResMaxSlots / 2;  // slots per buffer with two TMEM buffers
 constexpr int kBufCols = kResTmemCols / 2;   // columns per buffer with two TMEM buffers
 constexpr int kStatSlots = 4;                // heads whose statistics may be in flight
+// Compact layout (256-byte rows, up to 64 text rows): score rows for at most 8
+// tiles per CTA and a 320-column statistics buffer leave room for a fifth K
+// stage. A launch whose tiles per CTA and cluster x slot columns fit takes it.
+constexpr int kResCompactTiles = 8;
+constexpr int kResCompactRecv = 320;
 
-template <int ROW_BYTES, int MROWS>
+template <int ROW_BYTES, int MROWS, bool COMPACT>
 struct ResLayout {
     static constexpr int KB = ROW_BYTES / 128;
     static constexpr int TILE_BYTES = kTileRows * ROW_BYTES;
@@ -63,8 +68,9 @@ struct ResLayout {
     static constexpr int WGC = MROWS / kResWG;  // most text columns one warpgroup owns (16 or 32)
     // statistics receive buffer: [kStatSlots heads][cluster rank][column] (m, l);
     // cluster size times slot columns must fit RECV_COLS
-    static constexpr int RECV_COLS = ROW_BYTES == 256 ? 640 : 1024;
-    static constexpr int ACC_BYTES = kResWG * kResMaxSlots * kTileRows * 4;  // per warpgroup partial rows
+    static constexpr int RECV_COLS = COMPACT ? kResCompactRecv : ROW_BYTES == 256 ? 640 : 1024;
+    static constexpr int ACC_TILES = COMPACT ? kResCompactTiles : kResMaxSlots;  // score rows kept per warpgroup
+    static constexpr int ACC_BYTES = kResWG * ACC_TILES * kTileRows * 4;
     // [max of head s & 1 (2) | sum][wg][quadrant warp][WGC columns]
     static constexpr int SCR_BYTES = 3 * kResWG * 4 * WGC * 4;
     static constexpr int NBAR_FIXED = 2 * 2 + 2 * kResMaxSlots + kStatSlots + 2;
@@ -125,7 +131,7 @@ struct ResShape {
     bool bad;
 };
 
-template <int RECV_COLS>
+template <int RECV_COLS, int ACC_TILES>
 __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int n1, int tq, int t1, uint32_t rank,
                                               uint32_t csize, int mrows)
 {
@@ -142,18 +148,18 @@ __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int 
     const int buf_cols = r.nb == 2 ? kBufCols : kResTmemCols;
     r.bad = r.T > mrows || r.n2 > p.slot_cols || (r.N > 0 && r.T <= 0) ||
             (tpc > 0 && (tpc - 1) * p.slot_cols + span > buf_cols) ||
-            tpc > (r.nb == 2 ? kBufSlots : kResMaxSlots) || (int)csize * p.slot_cols > RECV_COLS;
+            tpc > (r.nb == 2 ? kBufSlots : kResMaxSlots) || tpc > ACC_TILES || (int)csize * p.slot_cols > RECV_COLS;
     r.tile_begin = min(r.n_tiles, (int)rank * tpc);
     r.mt = min(r.n_tiles, r.tile_begin + tpc) - r.tile_begin;
     return r;
 }
 
-template <int ROW_BYTES, bool FP8, int MROWS>
+template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT>
 __global__ void __launch_bounds__(kResThreads, 1)
     score_res_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ ScoreLaunch p)
 {
-    using L = ResLayout<ROW_BYTES, MROWS>;
+    using L = ResLayout<ROW_BYTES, MROWS, COMPACT>;
     constexpr int KSTEPS = ROW_BYTES / 32;
     constexpr int ELEMS_PER_KB = FP8 ? 128 : 64;
     constexpr uint32_t FMT = FP8 ? 0u : 1u;
@@ -161,6 +167,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
     static_assert(kStages >= 3, "ring depth");
     static_assert(L::ALLOC > 116 * 1024, "one CTA per SM");
     static_assert(L::ALLOC <= 227 * 1024, "shared memory per CTA");
+    static_assert(!COMPACT || kStages == 5, "the compact layout exists for its fifth K stage");
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -259,7 +266,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const uint32_t tmem = *tmem_slot;
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
-    const ResShape shp = res_shape<L::RECV_COLS>(p, n0, n1, tq, t1, rank, csize, MROWS);
+    const ResShape shp = res_shape<L::RECV_COLS, L::ACC_TILES>(p, n0, n1, tq, t1, rank, csize, MROWS);
     const int N = shp.N, t0 = shp.t0, T = shp.T, n2 = shp.n2, nb = shp.nb;
     const bool bad_shape = shp.bad || (flat && nb != 1);  // uniform for the whole cluster
     if (bad_shape || N <= 0) {
@@ -352,6 +359,18 @@ __global__ void __launch_bounds__(kResThreads, 1)
             const int who = warp - 1;  // 0: even tiles, 1: odd tiles
             if (mt > 0) {
                 const uint32_t idesc = idesc_make(128, (uint32_t)n2, FMT);
+                // A stage's consecutive loads can belong to different threads
+                // (tiles gt and gt - kStages of opposite parity within their
+                // heads). The K_FULL parity test is only sound once the stage's
+                // previous load has landed, which a thread knows of its own tiles
+                // but not of the other thread's: for those tiles it first waits
+                // for the release of the previous load (its contraction done, so
+                // its data had landed). `cross` marks them by tile.
+                uint32_t cross = 0;
+                for (int tl = who; tl < mt; tl += 2) {
+                    const int ptl = ((tl - kStages) % mt + mt) % mt;
+                    if ((ptl ^ tl) & 1) cross |= 1u << tl;
+                }
                 bool ok = true;
                 for (int s = 0; s < nheads && ok; ++s) {
                     const int qb = s & 1;
@@ -364,6 +383,10 @@ __global__ void __launch_bounds__(kResThreads, 1)
                         const int sl = buf * kBufSlots + tl;
                         const int gt = s * mt + tl;  // the ring runs over the tiles of all heads in order
                         const uint32_t ks = (uint32_t)(gt % kStages), kph = (uint32_t)(gt / kStages) & 1u;
+                        if (((cross >> tl) & 1u) && gt >= kStages && !wait_phase(BAR(K_EMPTY + ks), kph ^ 1u, ctl)) {
+                            ok = false;
+                            break;
+                        }
                         if (!wait_phase(BAR(K_FULL + ks), kph, ctl)) { ok = false; break; }
                         if (!wait_phase(BAR(S_EMPTY + sl), (use & 1u) ^ 1u, ctl)) { ok = false; break; }
                         tc_fence_after();
@@ -414,7 +437,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         const int cpw = res_wg_cols(n2);               // this warpgroup's columns: [c_begin, c_begin + cpw)
         const int c_begin = wg * cpw;
         const int nch = (cpw + kResChunk - 1) / kResChunk;
-        float* accw = acc_s + wg * kResMaxSlots * kTileRows;
+        float* accw = acc_s + wg * L::ACC_TILES * kTileRows;
         float* ssum = scr_sum + wg * 4 * WGC;
         float* b2w = b2_s + wg * WGC;                  // weight of column c_begin + c, 0 for c >= cpw or >= T
         float* mcw = mc_s + wg * WGC;                  // -(CTA column max * c) of column c_begin + c
@@ -671,7 +694,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 if (j < N) {
                     float a = acc_s[tl * kTileRows + vrow];
 #pragma unroll
-                    for (int g = 1; g < kResWG; ++g) a += acc_s[g * kResMaxSlots * kTileRows + tl * kTileRows + vrow];
+                    for (int g = 1; g < kResWG; ++g) a += acc_s[g * L::ACC_TILES * kTileRows + tl * kTileRows + vrow];
                     if (whole) p.out[hr.n0 + j] = a / denom;
                     else p.partials[(int64_t)(item - cf) * p.total_vis + hr.n0 + j] = a;
                 }
@@ -705,7 +728,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 if (j < N) {
                     float a = acc_s[tl * kTileRows + vrow];
 #pragma unroll
-                    for (int g = 1; g < kResWG; ++g) a += acc_s[g * kResMaxSlots * kTileRows + tl * kTileRows + vrow];
+                    for (int g = 1; g < kResWG; ++g) a += acc_s[g * L::ACC_TILES * kTileRows + tl * kTileRows + vrow];
                     if (!multi) p.out[n0 + j] = a / denom;
                     else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
                 }
@@ -724,28 +747,28 @@ __global__ void __launch_bounds__(kResThreads, 1)
     cluster_sync_all();
 }
 
-template <int ROW_BYTES, bool FP8, int MROWS>
+template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT>
 cudaError_t res_prepare(int cluster)
 {
-    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS>;
+    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS, COMPACT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         ResLayout<ROW_BYTES, MROWS>::ALLOC);
+                                         ResLayout<ROW_BYTES, MROWS, COMPACT>::ALLOC);
     if (e == cudaSuccess && cluster > 8) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     return e;
 }
 
-template <int ROW_BYTES, bool FP8, int MROWS>
+template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT = false>
 cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p, const ScorePlan& plan,
                        int batch, cudaStream_t stream)
 {
-    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS>;
-    cudaError_t e = res_prepare<ROW_BYTES, FP8, MROWS>(plan.cluster);
+    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS, COMPACT>;
+    cudaError_t e = res_prepare<ROW_BYTES, FP8, MROWS, COMPACT>(plan.cluster);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     const int items = plan.flat > 0 ? plan.flat : plan.groups * batch;
     cfg.gridDim = dim3((unsigned)(plan.cluster * items), 1, 1);
     cfg.blockDim = dim3(kResThreads, 1, 1);
-    cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS>::ALLOC;
+    cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS, COMPACT>::ALLOC;
     cfg.stream = stream;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -758,14 +781,17 @@ cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const S
     return cudaLaunchKernelEx(&cfg, kern, tm_q, tm_k, p);
 }
 
+// Clusters of the given size that fit on the GPU at once. Both layouts take
+// more than half of an SM's shared memory (one CTA per SM), so the full
+// layout's answer holds for the compact one too.
 template <int ROW_BYTES, bool FP8, int MROWS>
 int res_capacity(int cluster)
 {
-    if (res_prepare<ROW_BYTES, FP8, MROWS>(cluster) != cudaSuccess) return 0;
+    if (res_prepare<ROW_BYTES, FP8, MROWS, false>(cluster) != cudaSuccess) return 0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(cluster, 64, 1);
     cfg.blockDim = dim3(kResThreads, 1, 1);
-    cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS>::ALLOC;
+    cfg.dynamicSmemBytes = ResLayout<ROW_BYTES, MROWS, false>::ALLOC;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = cluster;
@@ -774,7 +800,7 @@ int res_capacity(int cluster)
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, score_res_kernel<ROW_BYTES, FP8, MROWS>, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, score_res_kernel<ROW_BYTES, FP8, MROWS, false>, &cfg) != cudaSuccess) {
         cudaGetLastError();
         return 0;
     }
@@ -799,7 +825,7 @@ int res_max_tiles(int slot_cols, int nb)
 int res_max_cluster(int row_bytes, int slot_cols)
 {
     if (slot_cols <= 0) return 0;
-    const int recv = row_bytes == 256 ? ResLayout<256, 64>::RECV_COLS : ResLayout<128, 64>::RECV_COLS;
+    const int recv = row_bytes == 256 ? ResLayout<256, 64, false>::RECV_COLS : ResLayout<128, 64, false>::RECV_COLS;
     const int c = recv / slot_cols;
     return c < kMaxCluster ? c : kMaxCluster;
 }
@@ -832,9 +858,12 @@ cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm
     if (fp8)
         return mrows == 64 ? res_launch<128, true, 64>(tm_q, tm_k, q, plan, batch, stream)
                            : res_launch<128, true, 128>(tm_q, tm_k, q, plan, batch, stream);
-    if (row_bytes == 256)
-        return mrows == 64 ? res_launch<256, false, 64>(tm_q, tm_k, q, plan, batch, stream)
-                           : res_launch<256, false, 128>(tm_q, tm_k, q, plan, batch, stream);
+    if (row_bytes == 256 && mrows == 64) {
+        if (plan.tiles_per_cta <= kResCompactTiles && plan.cluster * p.slot_cols <= kResCompactRecv)
+            return res_launch<256, false, 64, true>(tm_q, tm_k, q, plan, batch, stream);
+        return res_launch<256, false, 64>(tm_q, tm_k, q, plan, batch, stream);
+    }
+    if (row_bytes == 256) return res_launch<256, false, 128>(tm_q, tm_k, q, plan, batch, stream);
     return mrows == 64 ? res_launch<128, false, 64>(tm_q, tm_k, q, plan, batch, stream)
                        : res_launch<128, false, 128>(tm_q, tm_k, q, plan, batch, stream);
 }
