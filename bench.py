@@ -58,7 +58,9 @@ def parse_args(argv=None):
                     help="other workloads measured after the headline one, comma-separated, or 'none'; "
                          "auto: the three others when the headline is the default sweep on one GPU")
     ap.add_argument("--score-kernel", default="auto", choices=["auto", "reread", "resident", "resident_1buf",
-                                                                     "resident_2buf"])
+                                                                     "resident_2buf", "resident_flat"])
+    ap.add_argument("--query-split", default="whole", choices=["whole", "split"],
+                    help="resident plans for T > 64: each head's text rows whole, or as two pseudo-heads")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next", action="store_true", help="skip the next-row measurements (splice, ...)")
@@ -421,7 +423,7 @@ def measure(args, w, steps, warm_steps, dev, rank, world, full):
     ratio = float(w.keep_ratio or 0.0)
     total_kept = int(sum(alg["kept"]))
     sel = select.Selector(w.batch, w.total_vis, w.total_txt, w.hq, w.hkv, w.head_dim, w.dtype,
-                          score_kernel=args.score_kernel)
+                          score_kernel=args.score_kernel, query_split=args.query_split)
     h = sel.handle
     scores = torch.empty(w.total_vis, dtype=torch.float32, device=dev)
     kept = torch.empty(max(1, total_kept), dtype=torch.int32, device=dev)

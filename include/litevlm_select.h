@@ -76,6 +76,15 @@ typedef enum {
 #define LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS 16 /* the same, two TMEM head buffers where the shapes allow it */
 #define LITEVLM_FLAG_SCORE_RESIDENT_FLAT 64 /* the same, one buffer, with the flattened (request, head) schedule
                                                whenever every request has the same token counts */
+/* OR-ed with the above: resident plans for requests of more than 64 text
+ * tokens run each query head's text rows as two pseudo-heads (the first
+ * ceil(T/2) rows, then the rest) on the 64-row kernel, which reads the head's
+ * K tiles once per half (the second time from L2). The sums over heads and
+ * text rows are unchanged by the split (each text row's softmax is its own).
+ * Off by default: on GB300 it measured slower than the re-read kernel on the
+ * shapes tried (a 6144-token request with 128 text rows and 28 / 4 heads; a
+ * ragged e4m3 batch of 32 requests). Not with LITEVLM_FLAG_QUERY_LAST_TOKEN. */
+#define LITEVLM_FLAG_SCORE_SPLIT_QUERIES 128
 /* OR-ed with at most one of the above: only the last text token of each request
  * is a query, T_b counts as 1 in the mean (the last-token variant of attention-
  * score pruning, Related Work / FastV). Requests may then have more than 128
@@ -90,7 +99,8 @@ typedef struct {
     int32_t num_kv_heads;      /* Hkv, Hq % Hkv == 0 */
     int32_t head_dim;          /* d: 64 or 128 for bf16, 128 for e4m3 */
     litevlm_dtype_t qk_dtype;
-    int32_t flags;             /* 0 or one LITEVLM_FLAG_SCORE_* value, optionally | LITEVLM_FLAG_QUERY_LAST_TOKEN */
+    int32_t flags;             /* 0 or one LITEVLM_FLAG_SCORE_* kernel value, optionally
+                                  | LITEVLM_FLAG_SCORE_SPLIT_QUERIES | LITEVLM_FLAG_QUERY_LAST_TOKEN */
 } litevlm_select_config_t;
 
 typedef struct litevlm_select* litevlm_select_t;
@@ -408,10 +418,11 @@ litevlm_status_t litevlm_select_splice(litevlm_select_t handle, int32_t batch, c
  * 4: as 2, with a flattened schedule, for batches whose requests all have the
  * same visual and text token counts: the batch's (request, head) pairs are
  * split evenly over every cluster that fits on the GPU at once, each cluster
- * running its share back to back across request boundaries),
+ * running its share back to back across request boundaries; 5, 6, 7: as 2,
+ * 3, 4 with the query split, so heads count pseudo-heads below),
  * plan[1] = CTAs per thread-block cluster, plan[2] = 128-token tiles per CTA,
  * plan[3] = query-head groups (grid y), or the number of clusters for plan[0]
- * = 4. plan holds 4 int32.
+ * = 4 or 7. plan holds 4 int32.
  * Errors as for litevlm_select_score's host-side checks.
  */
 litevlm_status_t litevlm_select_score_plan(litevlm_select_t handle, int32_t batch, const int32_t* text_offsets_h,

@@ -125,7 +125,7 @@ struct ScoreChoice {
 // counts (the resident kernel's flattened schedule needs it).
 bool uniform_batch(int batch, const int32_t* seq_offsets_h, const int32_t* text_offsets_h)
 {
-    if (batch < 2) return false;
+    if (batch < 1) return false;
     const int32_t n = seq_offsets_h[1] - seq_offsets_h[0], t = text_offsets_h[1] - text_offsets_h[0];
     if (n <= 0 || t <= 0) return false;
     for (int32_t b = 1; b < batch; ++b)
@@ -173,26 +173,38 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* se
     ScoreChoice best{false, lvs::plan_score(bt, hq, c.num_kv_heads, lvs::kTileRows * row_bytes, tcap, &tc_cost)};
     double best_cost = 1.6 * tc_cost;
     const int max_tiles = batch > 0 ? td[0] : 0;
-    const int kflags = c.flags & ~LITEVLM_FLAG_QUERY_LAST_TOKEN;
-    if (kflags != LITEVLM_FLAG_SCORE_REREAD) {
-        if (kflags == LITEVLM_FLAG_SCORE_RESIDENT || kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
-            kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS || kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT)
-            best_cost = 1e300;
+    const bool split_queries = (c.flags & LITEVLM_FLAG_SCORE_SPLIT_QUERIES) != 0;
+    const int kflags = c.flags & ~(LITEVLM_FLAG_QUERY_LAST_TOKEN | LITEVLM_FLAG_SCORE_SPLIT_QUERIES);
+    if (kflags == LITEVLM_FLAG_SCORE_RESIDENT || kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER ||
+        kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS || kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT)
+        best_cost = 1e300;
+    // Query split (LITEVLM_FLAG_SCORE_SPLIT_QUERIES, T > 64): the resident plans
+    // run each head's text rows as two pseudo-heads of at most 64 rows on the
+    // 64-row kernel (the second half re-reads the head's K tiles, from L2). The
+    // partial-row workspace holds Hq rows, so a request's rows come in at most
+    // Hq parts.
+    const bool split = split_queries && max_t > 64 && !(c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN);
+    for (int qs = split ? 2 : 1; qs <= (split ? 2 : 1) && kflags != LITEVLM_FLAG_SCORE_REREAD; ++qs) {
+        const int mrows_r = qs == 2 ? 64 : mrows;
+        const int slot_r = qs == 2 ? (((max_t + 1) / 2 + 15) & ~15) : slot_cols;
+        const int hq_r = hq * qs;
+        const int cmax = lvs::res_max_cluster(row_bytes, slot_r);
+        int* rcap = h->res_capacity[mrows_r == 64 ? 0 : 1];
         for (int nb = 1; nb <= 2; ++nb) {
             if (nb == 2 && (kflags == LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER || kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT))
                 continue;
             if (nb == 1 && kflags == LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) continue;
-            const int R = lvs::res_max_tiles(slot_cols, nb);
+            const int R = lvs::res_max_tiles(slot_r, nb);
             for (int cl = 1; cl <= cmax; ++cl) {
                 const int tpc = (max_tiles + cl - 1) / cl;
                 if (tpc > R) continue;
                 if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;  // an idle rank on the largest request
-                int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
-                if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
+                int& cap = rcap[cl];
+                if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows_r, cl);
                 if (cap <= 0) continue;
                 for (int g = 1; g <= hq; ++g) {
-                    if (hq % g) continue;
-                    const int hpg = hq / g;
+                    if (hq_r % g) continue;
+                    const int hpg = hq_r / g;
                     if (nb == 2 && hpg < 2) continue;  // nothing to overlap
                     const long long ctas = (long long)batch * cl * g;
                     const double active = (double)(ctas < cap ? ctas : cap);
@@ -214,43 +226,54 @@ ScoreChoice choose_score_kernel(litevlm_select_t h, int batch, const int32_t* se
                         best_cost = cost;
                         lvs::ScorePlan pl{cl, tpc, g};
                         pl.res_nb = nb;
+                        pl.qsplit = qs;
                         best = ScoreChoice{true, pl};
                     }
                 }
             }
         }
-    }
-    // Flattened schedule (every request the same size, one TMEM head buffer):
-    // the batch's (request, head) pairs split evenly over every cluster that
-    // fits on the GPU at once, so there is no partial last wave; the clusters
-    // run their pairs back to back and each request boundary costs a write of
-    // the request's rows (a fold where a request spans two clusters).
-    if (uniform && h->allow_flat && kflags != LITEVLM_FLAG_SCORE_REREAD &&
-        kflags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) {
-        const int R = lvs::res_max_tiles(slot_cols, 1);
-        const long long pairs = (long long)batch * hq;
-        for (int cl = 1; cl <= cmax; ++cl) {
-            const int tpc = (max_tiles + cl - 1) / cl;
-            if (tpc > R) continue;
-            if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;
-            int& cap = h->res_capacity[mrows == 64 ? 0 : 1][cl];
-            if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows, cl);
-            if (cap <= 0) continue;
-            long long nclu = cap / cl;
-            if (nclu > pairs) nclu = pairs;
-            if (nclu > lvs::kFlatMax) nclu = lvs::kFlatMax;
-            if (nclu < 1) continue;
-            const double per_head = (double)tpc + (cl > 1 ? 1.0 : 0.25);
-            const long long per_cluster = (pairs + nclu - 1) / nclu;
-            const double boundaries = (double)per_cluster / hq + 1.0;
-            double cost = 6.0 + (double)per_cluster * per_head + 2.0 * boundaries;
-            if (kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT) cost -= 1e200;  // forced: any flat plan beats the others
-            if (cost < best_cost - 1e-9) {
-                best_cost = cost;
-                lvs::ScorePlan pl{cl, tpc, 1};
-                pl.res_nb = 1;
-                pl.flat = (int)nclu;
-                best = ScoreChoice{true, pl};
+        // Flattened schedule (every request the same size, one TMEM head buffer):
+        // the batch's (request, head) pairs split evenly over every cluster that
+        // fits on the GPU at once, so there is no partial last wave; the clusters
+        // run their pairs back to back and each request boundary costs a write of
+        // the request's rows (a fold where a request spans two clusters).
+        if (uniform && h->allow_flat && kflags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS) {
+            const int R = lvs::res_max_tiles(slot_r, 1);
+            const long long pairs = (long long)batch * hq_r;
+            for (int cl = 1; cl <= cmax; ++cl) {
+                const int tpc = (max_tiles + cl - 1) / cl;
+                if (tpc > R) continue;
+                if (cl > 1 && (cl - 1) * tpc >= max_tiles) continue;
+                int& cap = rcap[cl];
+                if (cap < 0) cap = lvs::res_cluster_capacity(row_bytes, fp8, mrows_r, cl);
+                if (cap <= 0) continue;
+                long long nclu = cap / cl;
+                if (nclu > pairs) nclu = pairs;
+                if (nclu > lvs::kFlatMax) nclu = lvs::kFlatMax;
+                if (nclu < 1) continue;
+                // clusters a request's pairs reach (its partial rows), at most Hq
+                int parts = 1;
+                for (int b = 0, k0 = 0; b < batch; ++b) {
+                    const long long first = (long long)b * hq_r, last = first + hq_r - 1;
+                    while (k0 + 1 < nclu && pairs * (k0 + 1) / nclu <= first) ++k0;
+                    int k1 = k0;
+                    while (k1 + 1 < nclu && pairs * (k1 + 1) / nclu <= last) ++k1;
+                    if (k1 - k0 + 1 > parts) parts = k1 - k0 + 1;
+                }
+                if (parts > hq) continue;
+                const double per_head = (double)tpc + (cl > 1 ? 1.0 : 0.25);
+                const long long per_cluster = (pairs + nclu - 1) / nclu;
+                const double boundaries = (double)per_cluster / hq_r + 1.0;
+                double cost = 6.0 + (double)per_cluster * per_head + 2.0 * boundaries;
+                if (kflags == LITEVLM_FLAG_SCORE_RESIDENT_FLAT) cost -= 1e200;  // forced: any flat plan beats the others
+                if (cost < best_cost - 1e-9) {
+                    best_cost = cost;
+                    lvs::ScorePlan pl{cl, tpc, 1};
+                    pl.res_nb = 1;
+                    pl.flat = (int)nclu;
+                    pl.qsplit = qs;
+                    best = ScoreChoice{true, pl};
+                }
             }
         }
     }
@@ -302,7 +325,7 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "num_q_heads must be a positive multiple of num_kv_heads");
     if (c->qk_dtype != LITEVLM_BF16 && c->qk_dtype != LITEVLM_FP8_E4M3)
         return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "qk_dtype must be LITEVLM_BF16 or LITEVLM_FP8_E4M3");
-    const int kflags = c->flags & ~LITEVLM_FLAG_QUERY_LAST_TOKEN;
+    const int kflags = c->flags & ~(LITEVLM_FLAG_QUERY_LAST_TOKEN | LITEVLM_FLAG_SCORE_SPLIT_QUERIES);
     if (c->flags < 0 || (kflags != 0 && kflags != LITEVLM_FLAG_SCORE_REREAD && kflags != LITEVLM_FLAG_SCORE_RESIDENT &&
                          kflags != LITEVLM_FLAG_SCORE_RESIDENT_ONE_BUFFER &&
                          kflags != LITEVLM_FLAG_SCORE_RESIDENT_TWO_BUFFERS && kflags != LITEVLM_FLAG_SCORE_RESIDENT_FLAT))
@@ -428,7 +451,7 @@ litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, co
     const bool fp8 = h->cfg.qk_dtype == LITEVLM_FP8_E4M3;
     const ScoreChoice ch = choose_score_kernel(h, batch, seq_offsets_h, sh.max_t, h->cfg.head_dim * (fp8 ? 1 : 2), fp8,
                                                uniform_batch(batch, seq_offsets_h, text_offsets_h));
-    plan[0] = !ch.resident ? 1 : ch.plan.flat > 0 ? 4 : 1 + ch.plan.res_nb;
+    plan[0] = !ch.resident ? 1 : (ch.plan.flat > 0 ? 4 : 1 + ch.plan.res_nb) + (ch.plan.qsplit == 2 ? 3 : 0);
     plan[1] = ch.plan.cluster;
     plan[2] = ch.plan.tiles_per_cta;
     plan[3] = ch.plan.flat > 0 ? ch.plan.flat : ch.plan.groups;
@@ -487,7 +510,8 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
     const lvs::ScorePlan& plan = choice.plan;
     if (plan.tiles_per_cta > lvs::kMaxTilesPerCta)
         return fail(h, LITEVLM_ERR_UNSUPPORTED, "request too long for one cluster");
-    const int mrows = max_t <= 64 ? 64 : 128;  // text rows of the pass-1 MMA
+    const bool qsplit = choice.resident && plan.qsplit == 2;
+    const int mrows = max_t <= 64 || qsplit ? 64 : 128;  // text rows of a head's (pseudo-head's) MMA
 
     CUtensorMap tm_q, tm_k;
     s = encode_rows_map(h, &tm_q, q_text, c.head_dim, c.num_q_heads, tot_t, mrows, fp8, "q_text");
@@ -508,7 +532,8 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
     p.wait_budget = h->wait_budget;
     p.stall = (h->debug_flags & LITEVLM_DEBUG_STALL_SCORE) != 0 && choice.resident;
-    p.slot_cols = (max_t + 15) & ~15;
+    p.slot_cols = ((qsplit ? (max_t + 1) / 2 : max_t) + 15) & ~15;
+    p.qsplit = qsplit ? 2 : 1;
     p.query_last = (c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;
     p.extra = nullptr;
     // the top-k CTA of a request reads groups x N_b partial values: worth it

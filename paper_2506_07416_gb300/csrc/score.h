@@ -29,7 +29,11 @@ struct ScoreLaunch {
     int32_t heads_per_group;
     int32_t groups;
     int32_t ctas_per_request; // cluster size * groups
-    int32_t slot_cols;        // resident kernel: TMEM columns per slot (T rounded up to 16, max over batch)
+    int32_t slot_cols;        // resident kernel: TMEM columns per slot (query rows per head, rounded up to 16)
+    // resident kernel: 1, or 2 when each query head's text rows run as two
+    // pseudo-heads (the first ceil(T/2) rows, then the rest): heads_per_group,
+    // groups and the flattened pairs count pseudo-heads, hq stays the model's
+    int32_t qsplit;
     int32_t res_nb;           // resident kernel: TMEM head buffers, 1 or 2 (2: heads overlap)
     int32_t query_last;       // 1: only the last text token of each request is a query
     int32_t defer_fold;       // 1 (with groups > 1): leave the group partials; the top-k kernel adds them
@@ -67,6 +71,7 @@ struct ScorePlan {
     int groups;               // head groups (grid.y); partial rows when > 1
     int res_nb = 1;           // resident kernel: TMEM head buffers
     int flat = 0;             // resident kernel: clusters of the flattened (request, head) schedule, 0: none
+    int qsplit = 1;           // resident kernel: 2 = each head's text rows as two pseudo-heads (64-row kernel)
 };
 
 // Host helpers (score_tc.cu)

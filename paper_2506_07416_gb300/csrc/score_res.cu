@@ -127,7 +127,7 @@ __device__ __forceinline__ float transpose_sum16(float (&x)[16], int lane)
 // What a CTA serves of its request: the text rows, the tile range, and whether
 // the shape fits the kernel's buffers (uniform over the cluster).
 struct ResShape {
-    int N, t0, T, n2, n_tiles, tile_begin, mt, nb;
+    int N, t0, T, Th, n2, n_tiles, tile_begin, mt, nb;
     bool bad;
 };
 
@@ -139,14 +139,15 @@ __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int 
     r.N = n1 - n0;
     r.t0 = p.query_last && t1 > tq ? t1 - 1 : tq;  // last-token queries: one row
     r.T = t1 - r.t0;
-    r.n2 = (r.T + 15) & ~15;
+    r.Th = p.qsplit == 2 ? (r.T + 1) >> 1 : r.T;  // rows of the first (largest) pseudo-head
+    r.n2 = (r.Th + 15) & ~15;
     r.n_tiles = (r.N + kTileRows - 1) / kTileRows;
     const int tpc = r.N > 0 ? (r.n_tiles + (int)csize - 1) / (int)csize : 0;
     // Shape errors are caught on the host; this only keeps the kernel within its buffers.
     const int span = res_read_span(p.slot_cols);  // columns the epilogue reads per slot
     r.nb = p.res_nb == 2 ? 2 : 1;
     const int buf_cols = r.nb == 2 ? kBufCols : kResTmemCols;
-    r.bad = r.T > mrows || r.n2 > p.slot_cols || (r.N > 0 && r.T <= 0) ||
+    r.bad = r.Th > mrows || r.n2 > p.slot_cols || (r.N > 0 && r.T <= 0) || (p.qsplit == 2 && p.query_last) ||
             (tpc > 0 && (tpc - 1) * p.slot_cols + span > buf_cols) ||
             tpc > (r.nb == 2 ? kBufSlots : kResMaxSlots) || tpc > ACC_TILES || (int)csize * p.slot_cols > RECV_COLS;
     r.tile_begin = min(r.n_tiles, (int)rank * tpc);
@@ -186,7 +187,8 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const int fr0 = flat ? p.flat_r[item] : 0;
     const int nheads = flat ? p.flat_r[item + 1] - fr0 : p.heads_per_group;
     const int req_i = flat ? 0 : item / p.groups;
-    const int b = flat ? fr0 / p.hq : (p.order_n > 0 ? (int)p.order[req_i] : req_i);
+    const int hqe = p.hq * p.qsplit;  // heads of a request as scheduled (pseudo-heads with the query split)
+    const int b = flat ? fr0 / hqe : (p.order_n > 0 ? (int)p.order[req_i] : req_i);
     const int hg = flat ? 0 : item - req_i * p.groups;
 
     // With the full-key-set terms (p.extra, written by the kernel launched just
@@ -267,7 +269,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
     const ResShape shp = res_shape<L::RECV_COLS, L::ACC_TILES>(p, n0, n1, tq, t1, rank, csize, MROWS);
-    const int N = shp.N, t0 = shp.t0, T = shp.T, n2 = shp.n2, nb = shp.nb;
+    const int N = shp.N, t0 = shp.t0, T = shp.T, Th = shp.Th, n2 = shp.n2, nb = shp.nb;
     const bool bad_shape = shp.bad || (flat && nb != 1);  // uniform for the whole cluster
     if (bad_shape || N <= 0) {
         if (p.extra) griddep_wait();
@@ -285,17 +287,27 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const int tile_begin = shp.tile_begin;
     const int tile_end = tile_begin + shp.mt;
     const int mt = shp.mt;
-    // request, query head, first visual row and first query row of head s of
-    // this CTA's sequence (with a flattened schedule the requests' rows follow
-    // one another at equal strides)
+    // request, scheduled head (pseudo-head with the query split), query head,
+    // first visual row, first query row and query rows of head s of this CTA's
+    // sequence (with a flattened schedule the requests' rows follow one another
+    // at equal strides). With the query split, pseudo-head 2h + u of a request
+    // holds the query rows [u * Th, min((u + 1) * Th, T)) of head h.
     struct HeadRef {
-        int b, h, n0, t0;
+        int b, ph, h, n0, t0, T;
     };
     const int t_stride = t1 - tq;
     auto head_of = [&](int s_) -> HeadRef {
-        if (!flat) return HeadRef{b, hg * hpg + s_, n0, t0};
-        const int rh = fr0 + s_, bb = rh / p.hq;
-        return HeadRef{bb, rh - bb * p.hq, n0 + (bb - b) * N, t0 + (bb - b) * t_stride};
+        int bb = b, ph = hg * hpg + s_, nn0 = n0, tt0 = t0;
+        if (flat) {
+            const int rh = fr0 + s_;
+            bb = rh / hqe;
+            ph = rh - bb * hqe;
+            nn0 = n0 + (bb - b) * N;
+            tt0 = t0 + (bb - b) * t_stride;
+        }
+        if (p.qsplit != 2) return HeadRef{bb, ph, ph, nn0, tt0, T};
+        const int u = ph & 1;
+        return HeadRef{bb, ph, ph >> 1, nn0, tt0 + u * Th, u ? T - Th : Th};
     };
 
     if (warp == 0) {
@@ -599,10 +611,11 @@ __global__ void __launch_bounds__(kResThreads, 1)
             // merge the cluster's statistics of this head (rank order) into the
             // column weights w = 2^(m_local*c - b), b = M*c + log2(L); 0 for unused columns
             wait_phase_cluster(BAR(STATS + slot), (uint32_t)(s / kStatSlots) & 1u, ctl);
+            const HeadRef hs = head_of(s);
             if (wt < WGC) {
                 const int col = c_begin + wt;
                 float wval = 0.f;
-                if (wt < cpw && col < T) {
+                if (wt < cpw && col < hs.T) {
                     const float2* rs = recv + (slot * (int)csize) * scols + col;  // rank r at rs[r * scols]
                     float M = -INFINITY;
                     for (int r = 0; r < (int)csize; ++r) M = fmaxf(M, rs[r * scols].x);
@@ -614,8 +627,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     float b = fmaf(M, cl, __log2f(Ls));
                     if (p.extra) {
                         griddep_wait();
-                        const HeadRef hr = head_of(s);
-                        b = log2_add(b, p.extra[(int64_t)(hr.t0 + col) * p.hq + hr.h]);
+                        b = log2_add(b, p.extra[(int64_t)(hs.t0 + col) * p.hq + hs.h]);
                     }
                     float mloc = smax[wt];  // this CTA's column max: the e values' reference
 #pragma unroll
@@ -675,7 +687,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         // final scores; otherwise this cluster's partial rows, folded by the last
         // of the request's clusters to finish each tile (fixed part order).
         auto flush = [&](const HeadRef& hr) {
-            const int first = hr.b * p.hq, last = first + p.hq - 1;
+            const int first = hr.b * hqe, last = first + hqe - 1;
             const bool whole = first >= fr0 && last < fr0 + nheads;
             auto cluster_of = [&](int pair) {  // the cluster whose range holds the pair
                 int lo = 0, hi = p.flat_n - 1;
@@ -716,7 +728,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 back(s);
                 if (flat) {
                     const HeadRef hr = head_of(s);
-                    if (s == nheads - 1 || hr.h == p.hq - 1) flush(hr);
+                    if (s == nheads - 1 || hr.ph == hqe - 1) flush(hr);
                 }
             }
         }
@@ -845,12 +857,13 @@ cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm
     ScoreLaunch q = p;
     q.res_nb = plan.res_nb;
     q.groups = plan.groups;
-    q.heads_per_group = p.hq / plan.groups;
+    q.qsplit = plan.qsplit;
+    q.heads_per_group = p.hq * plan.qsplit / plan.groups;
     q.ctas_per_request = plan.cluster * plan.groups;
     q.flat_n = 0;
     if (plan.flat > 0) {  // equal shares of the batch's (request, head) pairs, in request-major order
         if (plan.flat > kFlatMax || plan.res_nb != 1) return cudaErrorInvalidValue;
-        const long long pairs = (long long)batch * p.hq;
+        const long long pairs = (long long)batch * p.hq * plan.qsplit;
         q.flat_n = plan.flat;
         for (int k = 0; k <= plan.flat; ++k) q.flat_r[k] = (int32_t)(pairs * k / plan.flat);
         q.order_n = 0;

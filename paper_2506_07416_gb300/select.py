@@ -86,10 +86,13 @@ EXPORTS = ["litevlm_select_create", "litevlm_select_destroy", "litevlm_select_la
            "litevlm_select_last_launches", "litevlm_select_score_topk", "litevlm_select_host_view",
            "litevlm_select_keep_offsets", "litevlm_select_set_wait_budget", "litevlm_select_set_debug_flags"]
 FLAGS = {"auto": 0, "reread": 1, "resident": 2, "resident_1buf": 8, "resident_2buf": 16, "resident_flat": 64}
+# LITEVLM_FLAG_SCORE_SPLIT_QUERIES: resident plans for T > 64 run each head's text rows as two pseudo-heads
+QUERY_SPLIT = {"whole": 0, "split": 128}
 KERNELS = {1: "score_tc (K re-read per pass)", 2: "score_res (logits resident in TMEM, one head at a time)",
            3: "score_res (logits resident in TMEM, two heads overlapped)",
            4: "score_res (logits resident in TMEM, one head at a time, flattened (request, head) schedule over "
               "every cluster that fits at once)"}
+KERNELS.update({k + 3: v + ", each head's text rows as two pseudo-heads" for k, v in list(KERNELS.items())[1:]})
 
 
 def _check(rc: int, handle) -> None:
@@ -139,10 +142,14 @@ QUERY_LAST_TOKEN = 32
 
 
 def create(max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int, num_kv_heads: int,
-           head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto", query: str = "all") -> int:
-    """query: "all" (every text token is a query) or "last" (only the last one)."""
+           head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto", query: str = "all",
+           query_split: str = "whole") -> int:
+    """query: "all" (every text token is a query) or "last" (only the last one).
+    query_split: "whole", or "split" (resident plans for T > 64 run each head's
+    text rows as two pseudo-heads)."""
     cfg = Config(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
-                 DTYPES[qk_dtype], FLAGS[score_kernel] | (QUERY_LAST_TOKEN if query == "last" else 0))
+                 DTYPES[qk_dtype], FLAGS[score_kernel] | QUERY_SPLIT[query_split] |
+                 (QUERY_LAST_TOKEN if query == "last" else 0))
     h = ctypes.c_void_p()
     _check(LIB.litevlm_select_create(ctypes.byref(cfg), ctypes.byref(h)), None)
     return h.value
@@ -296,9 +303,9 @@ class Selector:
 
     def __init__(self, max_batch: int, max_total_visual: int, max_total_text: int, num_q_heads: int,
                  num_kv_heads: int, head_dim: int, qk_dtype: str = "bf16", score_kernel: str = "auto",
-                 query: str = "all"):
+                 query: str = "all", query_split: str = "whole"):
         self.handle = create(max_batch, max_total_visual, max_total_text, num_q_heads, num_kv_heads, head_dim,
-                             qk_dtype, score_kernel, query)
+                             qk_dtype, score_kernel, query, query_split)
         self.qk_dtype = qk_dtype
 
     def close(self) -> None:

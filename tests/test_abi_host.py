@@ -72,6 +72,8 @@ def _cfg(sel, **kw):
     (dict(max_total_visual=-5), 1),
     (dict(flags=3), 1),
     (dict(flags=-1), 1),
+    (dict(flags=2 | 128 | 512), 1),  # an unknown bit beside valid ones
+    (dict(flags=256), 1),
     (dict(qk_dtype=7), 1),
     (dict(head_dim=96), 2),
     (dict(head_dim=64, qk_dtype=1), 2),

@@ -110,7 +110,7 @@ def test_noalloc_rejects_head_groups_beyond_the_partial_scratch(sel):
         s = sel.Selector(1, n, t, hq, hkv, 128, "bf16")
         plan = s.score_plan(to, so)
         s.close()
-        if plan[0] != 4 and plan[3] > 1 and plan[3] * n > (1 << 20):
+        if plan[0] not in (4, 7) and plan[3] > 1 and plan[3] * n > (1 << 20):
             found = (n, t, hq, hkv, so, to)
             break
     assert found is not None, "no shape among the candidates splits its heads beyond the scratch"
