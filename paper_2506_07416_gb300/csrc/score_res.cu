@@ -131,7 +131,7 @@ struct ResShape {
     bool bad;
 };
 
-template <int RECV_COLS, int ACC_TILES>
+template <int RECV_COLS, int ACC_TILES, bool QS>
 __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int n1, int tq, int t1, uint32_t rank,
                                               uint32_t csize, int mrows)
 {
@@ -139,7 +139,7 @@ __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int 
     r.N = n1 - n0;
     r.t0 = p.query_last && t1 > tq ? t1 - 1 : tq;  // last-token queries: one row
     r.T = t1 - r.t0;
-    r.Th = p.qsplit == 2 ? (r.T + 1) >> 1 : r.T;  // rows of the first (largest) pseudo-head
+    r.Th = QS ? (r.T + 1) >> 1 : r.T;  // rows of the first (largest) pseudo-head
     r.n2 = (r.Th + 15) & ~15;
     r.n_tiles = (r.N + kTileRows - 1) / kTileRows;
     const int tpc = r.N > 0 ? (r.n_tiles + (int)csize - 1) / (int)csize : 0;
@@ -147,7 +147,7 @@ __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int 
     const int span = res_read_span(p.slot_cols);  // columns the epilogue reads per slot
     r.nb = p.res_nb == 2 ? 2 : 1;
     const int buf_cols = r.nb == 2 ? kBufCols : kResTmemCols;
-    r.bad = r.Th > mrows || r.n2 > p.slot_cols || (r.N > 0 && r.T <= 0) || (p.qsplit == 2 && p.query_last) ||
+    r.bad = r.Th > mrows || r.n2 > p.slot_cols || (r.N > 0 && r.T <= 0) || (QS && (p.query_last || p.qsplit != 2)) ||
             (tpc > 0 && (tpc - 1) * p.slot_cols + span > buf_cols) ||
             tpc > (r.nb == 2 ? kBufSlots : kResMaxSlots) || tpc > ACC_TILES || (int)csize * p.slot_cols > RECV_COLS;
     r.tile_begin = min(r.n_tiles, (int)rank * tpc);
@@ -155,7 +155,9 @@ __device__ __forceinline__ ResShape res_shape(const ScoreLaunch& p, int n0, int 
     return r;
 }
 
-template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT>
+// QS: the query split (each head's text rows as two pseudo-heads), a template
+// parameter so that the kernels without it carry none of its bookkeeping.
+template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT, bool QS>
 __global__ void __launch_bounds__(kResThreads, 1)
     score_res_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ ScoreLaunch p)
@@ -187,8 +189,10 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const int fr0 = flat ? p.flat_r[item] : 0;
     const int nheads = flat ? p.flat_r[item + 1] - fr0 : p.heads_per_group;
     const int req_i = flat ? 0 : item / p.groups;
-    const int hqe = p.hq * p.qsplit;  // heads of a request as scheduled (pseudo-heads with the query split)
-    const int b = flat ? fr0 / hqe : (p.order_n > 0 ? (int)p.order[req_i] : req_i);
+    // heads of a request as scheduled (pseudo-heads with the query split); read
+    // from the parameters where it is used rather than held in a register
+#define LVS_HQE (QS ? 2 * p.hq : p.hq)
+    const int b = flat ? fr0 / LVS_HQE : (p.order_n > 0 ? (int)p.order[req_i] : req_i);
     const int hg = flat ? 0 : item - req_i * p.groups;
 
     // With the full-key-set terms (p.extra, written by the kernel launched just
@@ -268,7 +272,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
     const uint32_t tmem = *tmem_slot;
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
-    const ResShape shp = res_shape<L::RECV_COLS, L::ACC_TILES>(p, n0, n1, tq, t1, rank, csize, MROWS);
+    const ResShape shp = res_shape<L::RECV_COLS, L::ACC_TILES, QS>(p, n0, n1, tq, t1, rank, csize, MROWS);
     const int N = shp.N, t0 = shp.t0, T = shp.T, Th = shp.Th, n2 = shp.n2, nb = shp.nb;
     const bool bad_shape = shp.bad || (flat && nb != 1);  // uniform for the whole cluster
     if (bad_shape || N <= 0) {
@@ -297,17 +301,22 @@ __global__ void __launch_bounds__(kResThreads, 1)
     };
     const int t_stride = t1 - tq;
     auto head_of = [&](int s_) -> HeadRef {
-        int bb = b, ph = hg * hpg + s_, nn0 = n0, tt0 = t0;
-        if (flat) {
-            const int rh = fr0 + s_;
-            bb = rh / hqe;
-            ph = rh - bb * hqe;
-            nn0 = n0 + (bb - b) * N;
-            tt0 = t0 + (bb - b) * t_stride;
+        if constexpr (!QS) {
+            if (!flat) return HeadRef{b, hg * hpg + s_, hg * hpg + s_, n0, t0, T};
+            const int rh = fr0 + s_, bb = rh / p.hq;
+            return HeadRef{bb, rh - bb * p.hq, rh - bb * p.hq, n0 + (bb - b) * N, t0 + (bb - b) * t_stride, T};
+        } else {
+            int bb = b, ph = hg * hpg + s_, nn0 = n0, tt0 = t0;
+            if (flat) {
+                const int rh = fr0 + s_;
+                bb = rh / LVS_HQE;
+                ph = rh - bb * LVS_HQE;
+                nn0 = n0 + (bb - b) * N;
+                tt0 = t0 + (bb - b) * t_stride;
+            }
+            const int u = ph & 1;
+            return HeadRef{bb, ph, ph >> 1, nn0, tt0 + u * Th, u ? T - Th : Th};
         }
-        if (p.qsplit != 2) return HeadRef{bb, ph, ph, nn0, tt0, T};
-        const int u = ph & 1;
-        return HeadRef{bb, ph, ph >> 1, nn0, tt0 + u * Th, u ? T - Th : Th};
     };
 
     if (warp == 0) {
@@ -611,11 +620,14 @@ __global__ void __launch_bounds__(kResThreads, 1)
             // merge the cluster's statistics of this head (rank order) into the
             // column weights w = 2^(m_local*c - b), b = M*c + log2(L); 0 for unused columns
             wait_phase_cluster(BAR(STATS + slot), (uint32_t)(s / kStatSlots) & 1u, ctl);
-            const HeadRef hs = head_of(s);
+            // query rows of head s (with the query split, pseudo-heads alternate
+            // halves: the parity of the request's pseudo-head index, which is the
+            // parity of its index in the schedule since a request has an even count)
+            const int Ts = !QS ? T : ((((flat ? fr0 : hg * hpg) + s) & 1) ? T - Th : Th);
             if (wt < WGC) {
                 const int col = c_begin + wt;
                 float wval = 0.f;
-                if (wt < cpw && col < hs.T) {
+                if (wt < cpw && col < Ts) {
                     const float2* rs = recv + (slot * (int)csize) * scols + col;  // rank r at rs[r * scols]
                     float M = -INFINITY;
                     for (int r = 0; r < (int)csize; ++r) M = fmaxf(M, rs[r * scols].x);
@@ -627,6 +639,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     float b = fmaf(M, cl, __log2f(Ls));
                     if (p.extra) {
                         griddep_wait();
+                        const HeadRef hs = head_of(s);
                         b = log2_add(b, p.extra[(int64_t)(hs.t0 + col) * p.hq + hs.h]);
                     }
                     float mloc = smax[wt];  // this CTA's column max: the e values' reference
@@ -687,7 +700,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         // final scores; otherwise this cluster's partial rows, folded by the last
         // of the request's clusters to finish each tile (fixed part order).
         auto flush = [&](const HeadRef& hr) {
-            const int first = hr.b * hqe, last = first + hqe - 1;
+            const int first = hr.b * LVS_HQE, last = first + LVS_HQE - 1;
             const bool whole = first >= fr0 && last < fr0 + nheads;
             auto cluster_of = [&](int pair) {  // the cluster whose range holds the pair
                 int lo = 0, hi = p.flat_n - 1;
@@ -728,7 +741,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 back(s);
                 if (flat) {
                     const HeadRef hr = head_of(s);
-                    if (s == nheads - 1 || hr.ph == hqe - 1) flush(hr);
+                    if (s == nheads - 1 || hr.ph == LVS_HQE - 1) flush(hr);
                 }
             }
         }
@@ -757,24 +770,25 @@ __global__ void __launch_bounds__(kResThreads, 1)
     }
     if (p.extra) griddep_wait();  // returns at once for threads that already waited
     cluster_sync_all();
+#undef LVS_HQE
 }
 
-template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT>
+template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT, bool QS>
 cudaError_t res_prepare(int cluster)
 {
-    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS, COMPACT>;
+    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS, COMPACT, QS>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          ResLayout<ROW_BYTES, MROWS, COMPACT>::ALLOC);
     if (e == cudaSuccess && cluster > 8) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     return e;
 }
 
-template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT = false>
+template <int ROW_BYTES, bool FP8, int MROWS, bool COMPACT = false, bool QS = false>
 cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const ScoreLaunch& p, const ScorePlan& plan,
                        int batch, cudaStream_t stream)
 {
-    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS, COMPACT>;
-    cudaError_t e = res_prepare<ROW_BYTES, FP8, MROWS, COMPACT>(plan.cluster);
+    auto kern = score_res_kernel<ROW_BYTES, FP8, MROWS, COMPACT, QS>;
+    cudaError_t e = res_prepare<ROW_BYTES, FP8, MROWS, COMPACT, QS>(plan.cluster);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     const int items = plan.flat > 0 ? plan.flat : plan.groups * batch;
@@ -799,7 +813,7 @@ cudaError_t res_launch(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const S
 template <int ROW_BYTES, bool FP8, int MROWS>
 int res_capacity(int cluster)
 {
-    if (res_prepare<ROW_BYTES, FP8, MROWS, false>(cluster) != cudaSuccess) return 0;
+    if (res_prepare<ROW_BYTES, FP8, MROWS, false, false>(cluster) != cudaSuccess) return 0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(cluster, 64, 1);
     cfg.blockDim = dim3(kResThreads, 1, 1);
@@ -812,7 +826,7 @@ int res_capacity(int cluster)
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, score_res_kernel<ROW_BYTES, FP8, MROWS, false>, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, score_res_kernel<ROW_BYTES, FP8, MROWS, false, false>, &cfg) != cudaSuccess) {
         cudaGetLastError();
         return 0;
     }
@@ -868,12 +882,20 @@ cudaError_t launch_score_resident(const CUtensorMap& tm_q, const CUtensorMap& tm
         for (int k = 0; k <= plan.flat; ++k) q.flat_r[k] = (int32_t)(pairs * k / plan.flat);
         q.order_n = 0;
     }
+    const bool compact = plan.tiles_per_cta <= kResCompactTiles && plan.cluster * p.slot_cols <= kResCompactRecv;
+    if (plan.qsplit == 2) {  // the 64-row kernels only
+        if (mrows != 64) return cudaErrorInvalidValue;
+        if (fp8) return res_launch<128, true, 64, false, true>(tm_q, tm_k, q, plan, batch, stream);
+        if (row_bytes == 256)
+            return compact ? res_launch<256, false, 64, true, true>(tm_q, tm_k, q, plan, batch, stream)
+                           : res_launch<256, false, 64, false, true>(tm_q, tm_k, q, plan, batch, stream);
+        return res_launch<128, false, 64, false, true>(tm_q, tm_k, q, plan, batch, stream);
+    }
     if (fp8)
         return mrows == 64 ? res_launch<128, true, 64>(tm_q, tm_k, q, plan, batch, stream)
                            : res_launch<128, true, 128>(tm_q, tm_k, q, plan, batch, stream);
     if (row_bytes == 256 && mrows == 64) {
-        if (plan.tiles_per_cta <= kResCompactTiles && plan.cluster * p.slot_cols <= kResCompactRecv)
-            return res_launch<256, false, 64, true>(tm_q, tm_k, q, plan, batch, stream);
+        if (compact) return res_launch<256, false, 64, true>(tm_q, tm_k, q, plan, batch, stream);
         return res_launch<256, false, 64>(tm_q, tm_k, q, plan, batch, stream);
     }
     if (row_bytes == 256) return res_launch<256, false, 128>(tm_q, tm_k, q, plan, batch, stream);
