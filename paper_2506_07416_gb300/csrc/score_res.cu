@@ -466,6 +466,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
         const uint32_t tcol = tmem + lane_off;
         for (int tl = 0; tl < mt; ++tl) accw[tl * kTileRows + vrow] = 0.f;
         auto lane_valid = [&](int tl) { return tl < mt && (tile_begin + tl) * kTileRows + vrow < N; };
+        const bool tail_tile = mt > 0 && (tile_begin + mt) * kTileRows > N;  // the request's last, partial tile
         // slot tl of buffer b is read by this warp: hand it back to the MMA warp
         // (one arrival per warp and slot)
         auto release = [&](int b_, int tl_) {
@@ -485,8 +486,12 @@ __global__ void __launch_bounds__(kResThreads, 1)
             // again four heads later would arrive twice on it)
             if (et == 0 && !*abort_flag) mbar_arrive_expect_tx(BAR(STATS + slot), (uint32_t)(csize * n2 * 8));
             for (int ch = 0; ch < nch; ++ch) {
+                const int cw = min(kResChunk, cpw - kResChunk * ch);  // 4, 8, 12 or 16
                 const uint32_t col0 = (uint32_t)(c_begin + kResChunk * ch);
-                // ---- A: column maxima, per thread over its slots, then over the lanes
+                // ---- A: column maxima, per thread over its slots, then over the lanes.
+                // A request's last tile may hold rows past its end: their logits
+                // become -inf in tensor memory (this warpgroup's columns), so that B
+                // needs no per-value select (2^-inf = 0) and C adds nothing for them.
                 float cm[16];
 #pragma unroll
                 for (int c = 0; c < 16; ++c) cm[c] = -INFINITY;
@@ -524,6 +529,17 @@ __global__ void __launch_bounds__(kResThreads, 1)
                         }
                     }
                     tmem_wait_ld();
+                    // only the CTA's last tile can run past the request's end
+                    if (tail_tile && !__all_sync(0xffffffffu, lane_valid(mt - 1))) {
+                        const uint32_t ta = tbuf + (uint32_t)((mt - 1) * scols) + col0;
+                        tmem_ld16(ta, va);
+                        tmem_wait_ld();
+                        const bool okv = lane_valid(mt - 1);
+#pragma unroll
+                        for (int c = 0; c < 16; ++c) va[c] = okv ? va[c] : -INFINITY;
+                        tmem_st_cols16(ta, va, cw);
+                        tmem_wait_st();  // B reads these rows
+                    }
                 }
 #pragma unroll
                 for (int c = 0; c < 16; ++c) cm[c] = warp_max_f32(cm[c]);
@@ -564,17 +580,17 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     const uint32_t ta = tbuf + (uint32_t)(tl * scols) + col0;
                     tmem_ld16(ta, v);
                     tmem_wait_ld();
-                    const bool ok = lane_valid(tl);
                     const float2 cl2 = make_float2(cl, cl);
+                    // rows past the request's end hold -inf (pass A), so their e is 0
 #pragma unroll
                     for (int c = 0; c < 16; c += 4) {
                         const float4 m4 = *reinterpret_cast<const float4*>(mcw + kResChunk * ch + c);
                         const float2 x01 = ffma2(make_float2(v[c], v[c + 1]), cl2, make_float2(m4.x, m4.y));
                         const float2 x23 = ffma2(make_float2(v[c + 2], v[c + 3]), cl2, make_float2(m4.z, m4.w));
-                        const float e0 = ok ? ex2(x01.x) : 0.f;
-                        const float e1 = ok ? ex2(x01.y) : 0.f;
-                        const float e2 = ok ? ex2(x23.x) : 0.f;
-                        const float e3 = ok ? ex2(x23.y) : 0.f;
+                        const float e0 = ex2(x01.x);
+                        const float e1 = ex2(x01.y);
+                        const float e2 = ex2(x23.x);
+                        const float e3 = ex2(x23.y);
                         v[c] = e0;
                         v[c + 1] = e1;
                         v[c + 2] = e2;
