@@ -572,9 +572,17 @@ __global__ void __launch_bounds__(kResThreads, 1)
                 const uint32_t col0 = (uint32_t)(c_begin + kResChunk * ch);
                 // ---- B: e = 2^(s*c - m*c) written back over the logits (this warpgroup's
                 // columns only); per-thread column sums of e, then over the warp's lanes
-                float sm[16];
+                float sm[16], mh[16];  // column sums; the shifts -m*c, in registers for all tiles
 #pragma unroll
                 for (int c = 0; c < 16; ++c) sm[c] = 0.f;
+#pragma unroll
+                for (int c = 0; c < 16; c += 4) {
+                    const float4 m4 = *reinterpret_cast<const float4*>(mcw + kResChunk * ch + c);
+                    mh[c] = m4.x;
+                    mh[c + 1] = m4.y;
+                    mh[c + 2] = m4.z;
+                    mh[c + 3] = m4.w;
+                }
                 for (int tl = 0; tl < mt; ++tl) {
                     float v[16];
                     const uint32_t ta = tbuf + (uint32_t)(tl * scols) + col0;
@@ -584,9 +592,8 @@ __global__ void __launch_bounds__(kResThreads, 1)
                     // rows past the request's end hold -inf (pass A), so their e is 0
 #pragma unroll
                     for (int c = 0; c < 16; c += 4) {
-                        const float4 m4 = *reinterpret_cast<const float4*>(mcw + kResChunk * ch + c);
-                        const float2 x01 = ffma2(make_float2(v[c], v[c + 1]), cl2, make_float2(m4.x, m4.y));
-                        const float2 x23 = ffma2(make_float2(v[c + 2], v[c + 3]), cl2, make_float2(m4.z, m4.w));
+                        const float2 x01 = ffma2(make_float2(v[c], v[c + 1]), cl2, make_float2(mh[c], mh[c + 1]));
+                        const float2 x23 = ffma2(make_float2(v[c + 2], v[c + 3]), cl2, make_float2(mh[c + 2], mh[c + 3]));
                         const float e0 = ex2(x01.x);
                         const float e1 = ex2(x01.y);
                         const float e2 = ex2(x23.x);
