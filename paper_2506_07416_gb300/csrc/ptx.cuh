@@ -286,44 +286,6 @@ __device__ __forceinline__ void mma_f8(uint32_t d_tmem, uint64_t a_desc, uint64_
         : "memory");
 }
 
-// The same two contractions issued by lane 0 of a converged warp only: the
-// whole warp executes the instruction (so the descriptors can stay in the
-// warp-uniform datapath) and `leader` (1 in lane 0, 0 elsewhere) predicates it.
-__device__ __forceinline__ void mma_f16_lead(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                             uint32_t accumulate, uint32_t leader)
-{
-    asm volatile(
-        "{\n\t.reg .pred p, e;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "setp.ne.b32 e, %5, 0;\n\t"
-        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(leader)
-        : "memory");
-}
-
-__device__ __forceinline__ void mma_f8_lead(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                            uint32_t accumulate, uint32_t leader)
-{
-    asm volatile(
-        "{\n\t.reg .pred p, e;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "setp.ne.b32 e, %5, 0;\n\t"
-        "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(leader)
-        : "memory");
-}
-
-// tcgen05.commit by lane 0 of a converged warp (the lane that issued the contractions)
-__device__ __forceinline__ void mma_commit_lead(uint32_t bar, uint32_t leader)
-{
-    asm volatile(
-        "{\n\t.reg .pred e;\n\t"
-        "setp.ne.b32 e, %1, 0;\n\t"
-        "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(bar),
-        "r"(leader)
-        : "memory");
-}
-
 // arrive (once) on an mbarrier when all prior tcgen05 async ops of this thread complete
 __device__ __forceinline__ void mma_commit(uint32_t bar)
 {
@@ -412,15 +374,6 @@ __device__ __forceinline__ void tmem_ld16x2_32(uint32_t taddr, float* v)
         : "r"(taddr), "n"(SPLIT));
 }
 
-// 32 lanes x 8 consecutive 32-bit columns
-__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v)
-{
-    uint32_t* r = reinterpret_cast<uint32_t*>(v);
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                 : "r"(taddr));
-}
-
 // 32 lanes x 32 consecutive 32-bit columns written from registers (thread t -> lane base + t)
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v)
 {
@@ -487,20 +440,6 @@ __device__ __forceinline__ void tmem_st_cols16(uint32_t taddr, const float* v, i
     }
 }
 
-// Stores exactly n (8, 16, 24 or 32, the same for the whole warp) columns.
-__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const float* v, int n)
-{
-    switch (n) {
-    case 32: tmem_st32(taddr, v); break;
-    case 24:
-        tmem_st16(taddr, v);
-        tmem_st8(taddr + 16, v + 16);
-        break;
-    case 16: tmem_st16(taddr, v); break;
-    default: tmem_st8(taddr, v); break;
-    }
-}
-
 __device__ __forceinline__ void tmem_wait_st()
 {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
@@ -523,19 +462,6 @@ __device__ __forceinline__ void st_async_f2(uint32_t cluster_addr, float a, floa
                      cluster_addr),
                  "f"(a), "f"(b), "r"(cluster_bar)
                  : "memory");
-}
-
-// 16 lanes x 16 columns, twice (threads 16..31 at column offset SPLIT).
-template <int SPLIT>
-__device__ __forceinline__ void tmem_ld16x2_16(uint32_t taddr, float* v)
-{
-    uint32_t* r = reinterpret_cast<uint32_t*>(v);
-    asm volatile(
-        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16], %17;"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr), "n"(SPLIT));
 }
 
 }  // namespace lvs
