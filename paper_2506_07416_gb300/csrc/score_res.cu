@@ -29,7 +29,14 @@
 // one another's TMEM-load and exponential latencies; each warpgroup keeps its
 // own partial score rows, added in a fixed order at the end. With several head
 // groups the CTAs write partial rows and a per-tile ticket lets the last writer
-// of each tile add them (fixed group order).
+// of each tile add them (fixed group order). Rows past a request's end (only in
+// a CTA's last tile) get -inf logits in pass A, so B and C need no row mask.
+//
+// Schedules: one cluster per (request, head group), or for batches whose
+// requests all have the same token counts the batch's (request, head) pairs
+// split evenly over every cluster that fits at once (flat_n > 0). With the
+// query split (template parameter QS) each head's text rows run as two
+// pseudo-heads of at most 64 rows.
 //
 // Warp roles (608 threads): warp 0 = TMA producer, warp 1 = TMEM allocator
 // and MMA issuer of the even tiles, warp 2 = MMA issuer of the odd tiles,
