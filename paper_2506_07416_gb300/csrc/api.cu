@@ -8,6 +8,7 @@
 
 #include <algorithm>
 #include <cstdio>
+#include <cstring>
 #include <mutex>
 #include <new>
 #include <string>
@@ -15,6 +16,10 @@
 
 #include "../../include/litevlm_select.h"
 #include "internal.h"
+
+#ifdef LITEVLM_NVTX
+#include <nvtx3/nvToolsExt.h>
+#endif
 
 struct litevlm_select {
     litevlm_select_config_t cfg;
@@ -62,6 +67,45 @@ litevlm_status_t cuda_fail(litevlm_select_t h, cudaError_t e, const char* where)
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// An NVTX range around one C-ABI call, named after the call (builds with
+// LITEVLM_NVTX; an empty object otherwise).
+struct CallRange {
+#ifdef LITEVLM_NVTX
+    explicit CallRange(const char* name) { nvtxRangePushA(name); }
+    ~CallRange() { nvtxRangePop(); }
+#else
+    explicit CallRange(const char*) {}
+#endif
+};
+
+// Debug builds (LITEVLM_DEBUG): a device array must equal its host mirror.
+// Checked before anything is enqueued, with a synchronous copy after the
+// stream's earlier work (so not under stream capture); a mismatch is
+// INVALID_ARG. Release builds check nothing here.
+litevlm_status_t debug_mirror(litevlm_select_t h, const int32_t* d, const int32_t* host, int64_t n, const char* what,
+                              litevlm_stream_t stream)
+{
+#ifdef LITEVLM_DEBUG
+    if (!d || !host || n <= 0) return LITEVLM_OK;
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "debug mirror check");
+    std::vector<int32_t> tmp((size_t)n);
+    e = cudaMemcpy(tmp.data(), d, sizeof(int32_t) * (size_t)n, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(h, e, "debug mirror check");
+    if (std::memcmp(tmp.data(), host, sizeof(int32_t) * (size_t)n) != 0)
+        return fail(h, LITEVLM_ERR_INVALID_ARG,
+                    std::string(what) + " on the device differs from its host mirror (debug build)");
+#else
+    (void)h;
+    (void)d;
+    (void)host;
+    (void)n;
+    (void)what;
+    (void)stream;
+#endif
+    return LITEVLM_OK;
+}
 
 // Checks an offsets mirror: offs[0] = 0, non-decreasing, total within `max_total`.
 litevlm_status_t check_offsets(litevlm_select_t h, const int32_t* offs, int32_t batch, int64_t max_total,
@@ -292,6 +336,7 @@ extern "C" {
 
 const char* litevlm_status_string(litevlm_status_t s)
 {
+    const CallRange range_(__func__);
     switch (s) {
     case LITEVLM_OK: return "ok";
     case LITEVLM_ERR_INVALID_ARG: return "invalid argument";
@@ -306,6 +351,7 @@ const char* litevlm_status_string(litevlm_status_t s)
 
 const char* litevlm_select_last_error(litevlm_select_t h)
 {
+    const CallRange range_(__func__);
     return h ? h->last_error.c_str() : g_create_error.c_str();
 }
 
@@ -313,6 +359,7 @@ int32_t litevlm_select_last_launches(litevlm_select_t h) { return h ? h->last_la
 
 litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm_select_t* out)
 {
+    const CallRange range_(__func__);
     g_create_error.clear();
     if (!out) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "out is NULL");
     *out = nullptr;
@@ -388,6 +435,7 @@ litevlm_status_t litevlm_select_create(const litevlm_select_config_t* c, litevlm
 
 litevlm_status_t litevlm_select_destroy(litevlm_select_t h)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_OK;
     if (h->partials) cudaFree(h->partials);
     if (h->counters) cudaFree(h->counters);
@@ -440,6 +488,7 @@ litevlm_status_t check_score_shape(litevlm_select_t h, int32_t batch, const int3
 litevlm_status_t litevlm_select_score_plan(litevlm_select_t h, int32_t batch, const int32_t* text_offsets_h,
                                            const int32_t* seq_offsets_h, int32_t* plan)
 {
+    const CallRange range_(__func__);
     if (!h || !plan) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -505,6 +554,11 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
         if (!aligned16(ctx->k_text) || (ctx->k_sys && !aligned16(ctx->k_sys)))
             return fail(h, LITEVLM_ERR_INVALID_ARG, "k_sys and k_text must be 16-byte aligned");
     }
+    s = debug_mirror(h, seq_offsets_d, seq_offsets_h, (int64_t)batch + 1, "seq_offsets", stream);
+    if (s == LITEVLM_OK) s = debug_mirror(h, text_offsets_d, text_offsets_h, (int64_t)batch + 1, "text_offsets", stream);
+    if (s == LITEVLM_OK && ctx)
+        s = debug_mirror(h, ctx->sys_offsets_d, ctx->sys_offsets_h, (int64_t)batch + 1, "sys_offsets", stream);
+    if (s != LITEVLM_OK) return s;
     const ScoreChoice choice = choose_score_kernel(h, batch, seq_offsets_h, max_t, row_bytes, fp8,
                                                    uniform_batch(batch, seq_offsets_h, text_offsets_h));
     const lvs::ScorePlan& plan = choice.plan;
@@ -608,6 +662,7 @@ litevlm_status_t litevlm_select_score(litevlm_select_t h, int32_t batch, const v
                                       const int32_t* seq_offsets_h, float q_scale, float k_scale, float* scores,
                                       litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -623,6 +678,7 @@ litevlm_status_t litevlm_select_score_full_keys(litevlm_select_t h, int32_t batc
                                                 const void* k_text, float q_scale, float k_scale, float* scores,
                                                 litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -700,16 +756,20 @@ litevlm_status_t litevlm_select_topk(litevlm_select_t h, int32_t batch, const fl
                                      int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
                                      litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
     int max_n = 0;
     int64_t total_k = 0, tot_n = 0;
     bool run = false;
-    const litevlm_status_t s = topk_prepare(h, batch, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h,
-                                            keep_ratio, kept_idx, out_offsets_d, out_offsets_h, &max_n, &total_k,
-                                            &tot_n, &run);
+    litevlm_status_t s = topk_prepare(h, batch, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h,
+                                      keep_ratio, kept_idx, out_offsets_d, out_offsets_h, &max_n, &total_k, &tot_n,
+                                      &run);
     if (s != LITEVLM_OK || !run) return s;
+    s = debug_mirror(h, seq_offsets_d, seq_offsets_h, (int64_t)batch + 1, "seq_offsets", stream);
+    if (s == LITEVLM_OK) s = debug_mirror(h, keep_k_d, keep_k_h, batch, "keep_k", stream);
+    if (s != LITEVLM_OK) return s;
     // scores are only read (no deferred fold here)
     const cudaError_t e = lvs::launch_topk(batch, const_cast<float*>(scores), seq_offsets_d, keep_k_d, keep_ratio,
                                            kept_idx, out_offsets_d, max_n, h->topk_shape, (cudaStream_t)stream);
@@ -726,6 +786,7 @@ litevlm_status_t litevlm_select_score_topk(litevlm_select_t h, int32_t batch, co
                                            int32_t* kept_idx, int32_t* out_offsets_d, int32_t* out_offsets_h,
                                            litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -735,6 +796,8 @@ litevlm_status_t litevlm_select_score_topk(litevlm_select_t h, int32_t batch, co
     litevlm_status_t s = topk_prepare(h, batch, scores, seq_offsets_d, seq_offsets_h, keep_k_d, keep_k_h,
                                       keep_ratio, kept_idx, out_offsets_d, out_offsets_h, &max_n, &total_k, &tot_n,
                                       &run);
+    if (s != LITEVLM_OK) return s;
+    s = debug_mirror(h, keep_k_d, keep_k_h, batch, "keep_k", stream);
     if (s != LITEVLM_OK) return s;
     // the top-k kernel can take over the head-group fold when it holds the
     // request's keys in registers and has the sizes by value
@@ -765,6 +828,7 @@ litevlm_status_t litevlm_select_compact(litevlm_select_t h, int64_t total_kept, 
                                         int64_t src_rows, int32_t num_tensors, const void* const* src,
                                         void* const* dst, const int64_t* row_bytes, litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -803,6 +867,7 @@ litevlm_status_t litevlm_select_splice(litevlm_select_t h, int32_t batch, const 
                                        int32_t* out_offsets_d, int32_t* out_offsets_h, int32_t* position_ids,
                                        litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -837,6 +902,12 @@ litevlm_status_t litevlm_select_splice(litevlm_select_t h, int32_t batch, const 
         return fail(h, LITEVLM_ERR_INVALID_ARG, "a device row pointer is NULL");
     const bool vec16 = row_bytes % 16 == 0 && aligned16(sys_rows) && aligned16(vis_rows) && aligned16(txt_rows) &&
                        aligned16(out_rows);
+    const int64_t nb1 = (int64_t)batch + 1;
+    s = debug_mirror(h, sys_offsets_d, sys_offsets_h, nb1, "sys_offsets", stream);
+    if (s == LITEVLM_OK) s = debug_mirror(h, seq_offsets_d, seq_offsets_h, nb1, "seq_offsets", stream);
+    if (s == LITEVLM_OK) s = debug_mirror(h, kept_offsets_d, kept_offsets_h, nb1, "kept_offsets", stream);
+    if (s == LITEVLM_OK) s = debug_mirror(h, text_offsets_d, text_offsets_h, nb1, "text_offsets", stream);
+    if (s != LITEVLM_OK) return s;
     lvs::SpliceArgs a{};
     a.sys_off = sys_offsets_d;
     a.seq_off = seq_offsets_d;
@@ -864,6 +935,7 @@ litevlm_status_t litevlm_select_views(litevlm_select_t h, int32_t batch, int32_t
                                       int32_t* view_offsets, int32_t* selected_views, int32_t* seq_offsets,
                                       int32_t* seq_offsets_h, litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -913,6 +985,7 @@ litevlm_status_t litevlm_select_views(litevlm_select_t h, int32_t batch, int32_t
 litevlm_status_t litevlm_select_fold_norm(litevlm_select_t h, int32_t out_features, int32_t hidden, const void* w,
                                           const float* gamma, void* w_folded, litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -930,6 +1003,7 @@ litevlm_status_t litevlm_select_fold_norm(litevlm_select_t h, int32_t out_featur
 litevlm_status_t litevlm_select_rope_table(litevlm_select_t h, int32_t max_positions, int32_t head_dim,
                                            float rope_base, float* table, litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -953,6 +1027,7 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
                                         int32_t head_dim, const int32_t* positions, const float* rope_table,
                                         int32_t max_positions, float out_scale, void* y, litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     h->last_launches = 0;
@@ -1002,6 +1077,7 @@ litevlm_status_t litevlm_select_project(litevlm_select_t h, int64_t rows, int32_
 
 litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     int32_t word = 0;
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
@@ -1018,6 +1094,7 @@ litevlm_status_t litevlm_select_check_device(litevlm_select_t h, litevlm_stream_
 
 litevlm_status_t litevlm_select_host_view(litevlm_select_t h, const void* host, void** device_view)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     if (!host || !device_view) return fail(h, LITEVLM_ERR_INVALID_ARG, "host and device_view must not be NULL");
@@ -1034,6 +1111,7 @@ litevlm_status_t litevlm_select_host_view(litevlm_select_t h, const void* host, 
 litevlm_status_t litevlm_select_keep_offsets(int32_t batch, const int32_t* seq_offsets_h, const int32_t* keep_k_h,
                                              float keep_ratio, int32_t* out_offsets_h)
 {
+    const CallRange range_(__func__);
     g_create_error.clear();
     if (batch < 0) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "batch must be >= 0");
     if (!out_offsets_h) return fail(nullptr, LITEVLM_ERR_INVALID_ARG, "out_offsets_h is NULL");
@@ -1066,6 +1144,7 @@ litevlm_status_t litevlm_select_keep_offsets(int32_t batch, const int32_t* seq_o
 
 litevlm_status_t litevlm_select_set_debug_flags(litevlm_select_t h, int32_t flags)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     if (flags & ~LITEVLM_DEBUG_STALL_SCORE) return fail(h, LITEVLM_ERR_INVALID_ARG, "unknown debug flag");
@@ -1075,6 +1154,7 @@ litevlm_status_t litevlm_select_set_debug_flags(litevlm_select_t h, int32_t flag
 
 litevlm_status_t litevlm_select_set_wait_budget(litevlm_select_t h, int64_t cycles)
 {
+    const CallRange range_(__func__);
     if (!h) return LITEVLM_ERR_INVALID_ARG;
     h->last_error.clear();
     if (cycles < 0) return fail(h, LITEVLM_ERR_INVALID_ARG, "cycles must be >= 0 (0 restores the default)");
@@ -1176,6 +1256,7 @@ extern "C" litevlm_status_t litevlm_select_score_noalloc(int32_t num_q_heads, in
                                                          const int32_t* seq_offsets_h, float q_scale, float k_scale,
                                                          float* scores, int32_t* err_d, litevlm_stream_t stream)
 {
+    const CallRange range_(__func__);
     g_create_error.clear();
     // ---- host-only checks, before any CUDA call
     if (num_q_heads <= 0 || num_kv_heads <= 0 || num_q_heads % num_kv_heads != 0)

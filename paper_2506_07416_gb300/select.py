@@ -17,7 +17,9 @@ from typing import List, Optional, Sequence
 import numpy as np
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "liblitevlm_select.so")
+# LITEVLM_LIB may name another build of the library (e.g. the debug variant,
+# liblitevlm_select_debug.so); by default the release build in the package
+LIB_PATH = os.environ.get("LITEVLM_LIB") or os.path.join(_PKG, "liblitevlm_select.so")
 
 STATUS = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "WORKSPACE", 4: "CUDA", 5: "TIMEOUT",
           6: "DEVICE_BOUNDS"}
@@ -362,9 +364,11 @@ class Selector:
         return mask[:batch], vo, sv, so, so_h
 
     def score_topk(self, q, text_offsets, k, seq_offsets, q_scale=1.0, k_scale=1.0, keep_k=None,
-                   keep_ratio: float = 0.0, text_offsets_h=None, seq_offsets_h=None, stream=None):
+                   keep_ratio: float = 0.0, text_offsets_h=None, seq_offsets_h=None, stream=None, out=None,
+                   kept_idx=None, out_offsets=None):
         """Scores and top-k in one call. Returns (scores, kept_idx, out_offsets
-        device, out_offsets host numpy)."""
+        device, out_offsets host numpy); out / kept_idx / out_offsets are
+        optional caller buffers."""
         import torch
         so_h = _host_i32(seq_offsets if seq_offsets_h is None else seq_offsets_h)
         to_h = _host_i32(text_offsets if text_offsets_h is None else text_offsets_h)
@@ -375,9 +379,9 @@ class Selector:
             kk_d = keep_k if isinstance(keep_k, torch.Tensor) and keep_k.is_cuda else \
                 torch.from_numpy(kk_h).to(k.device)
         total = int(keep_offsets(so_h, kk_h, keep_ratio)[-1])
-        scores = torch.empty(max(1, int(so_h[-1])), dtype=torch.float32, device=k.device)
-        kept = torch.empty(max(total, 1), dtype=torch.int32, device=k.device)
-        off_d = torch.empty(batch + 1, dtype=torch.int32, device=k.device)
+        scores = out if out is not None else torch.empty(max(1, int(so_h[-1])), dtype=torch.float32, device=k.device)
+        kept = kept_idx if kept_idx is not None else torch.empty(max(total, 1), dtype=torch.int32, device=k.device)
+        off_d = out_offsets if out_offsets is not None else torch.empty(batch + 1, dtype=torch.int32, device=k.device)
         off_h = np.zeros(batch + 1, np.int32)
         score_topk(self.handle, batch, q, text_offsets, to_h, k, seq_offsets, so_h, q_scale, k_scale, scores, kk_d,
                    kk_h, keep_ratio, kept, off_d, off_h, stream)
