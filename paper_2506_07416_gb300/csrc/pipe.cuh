@@ -142,6 +142,10 @@ __device__ __forceinline__ int fold_ticket_index(int b, int n0, int t) { return 
 // (default: the head groups) that own a tile adds the partials of that tile
 // in index order and writes the scores. `nthreads` threads (ids 0..nthreads-1, synchronised by
 // named barrier `bar_id`) take part; `flags` is shared memory for mt ints.
+// Each thread sums R rows at a time, with the loads of all R rows (up to 16
+// partials each) in flight together: a CTA that folds a long request's tiles
+// alone pays one L2 round trip per R rows instead of one per row.
+template <int R = 1>
 __device__ __forceinline__ void fold_tiles(const ScoreLaunch& p, int b, int n0, int N, int T, int tile_begin,
                                            int mt, int tid, int nthreads, uint32_t bar_id, volatile int* flags,
                                            int parts = 0)
@@ -159,24 +163,61 @@ __device__ __forceinline__ void fold_tiles(const ScoreLaunch& p, int b, int n0, 
     named_bar_sync(bar_id, nthreads);
     __threadfence();
     const float denom = (float)p.hq * (float)T;
-    // (tile, row) pairs spread over all threads; up to 16 group partials in
-    // flight per row, added in group order
-    for (int x = tid; x < mt * kTileRows; x += nthreads) {
-        const int tl = x / kTileRows;
-        if (!flags[tl]) continue;
-        const int j = (tile_begin + tl) * kTileRows + (x - tl * kTileRows);
-        if (j >= N) continue;
-        const float* src = p.partials + n0 + j;
-        float sum = 0.f;
-        for (int g = 0; g < parts; g += 16) {
-            float v[16];
+    if constexpr (R == 1) {
+        // (tile, row) pairs spread over all threads; up to 16 group partials in
+        // flight per row, added in group order
+        for (int x = tid; x < mt * kTileRows; x += nthreads) {
+            const int tl = x / kTileRows;
+            if (!flags[tl]) continue;
+            const int j = (tile_begin + tl) * kTileRows + (x - tl * kTileRows);
+            if (j >= N) continue;
+            const float* src = p.partials + n0 + j;
+            float sum = 0.f;
+            for (int g = 0; g < parts; g += 16) {
+                float v[16];
 #pragma unroll
-            for (int q = 0; q < 16; ++q) v[q] = g + q < parts ? __ldcg(src + (int64_t)(g + q) * p.total_vis) : 0.f;
+                for (int q = 0; q < 16; ++q) v[q] = g + q < parts ? __ldcg(src + (int64_t)(g + q) * p.total_vis) : 0.f;
 #pragma unroll
-            for (int q = 0; q < 16; ++q)
-                if (g + q < parts) sum += v[q];
+                for (int q = 0; q < 16; ++q)
+                    if (g + q < parts) sum += v[q];
+            }
+            p.out[n0 + j] = sum / denom;
         }
-        p.out[n0 + j] = sum / denom;
+    } else {
+        // thread tid takes rows x = tid + k * nthreads, R of them at a time, their
+        // group partials added in group order
+        for (int x0 = tid; x0 < mt * kTileRows; x0 += R * nthreads) {
+            int j[R];
+            bool live[R];
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const int x = x0 + r * nthreads;
+                const int tl = x / kTileRows;
+                j[r] = (tile_begin + tl) * kTileRows + (x - tl * kTileRows);
+                live[r] = x < mt * kTileRows && flags[tl] && j[r] < N;
+            }
+            float sum[R];
+#pragma unroll
+            for (int r = 0; r < R; ++r) sum[r] = 0.f;
+            for (int g = 0; g < parts; g += 16) {
+                float v[R][16];
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+#pragma unroll
+                    for (int q = 0; q < 16; ++q)
+                        v[r][q] = live[r] && g + q < parts
+                                      ? __ldcg(p.partials + n0 + j[r] + (int64_t)(g + q) * p.total_vis)
+                                      : 0.f;
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+#pragma unroll
+                    for (int q = 0; q < 16; ++q)
+                        if (g + q < parts) sum[r] += v[r][q];
+            }
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+                if (live[r]) p.out[n0 + j[r]] = sum[r] / denom;
+        }
     }
 }
 

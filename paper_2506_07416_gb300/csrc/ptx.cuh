@@ -204,11 +204,6 @@ __device__ __forceinline__ float2 ld_shared_cluster_f2(uint32_t addr)
     return v;
 }
 
-__device__ __forceinline__ void fence_acq_rel_cluster()
-{
-    asm volatile("fence.acq_rel.cluster;" ::: "memory");
-}
-
 // ----------------------------------------------------------------------------
 // TMA
 // ----------------------------------------------------------------------------

@@ -399,11 +399,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         stats_s[(s % kStatSlots) * kMaxText + prow] = make_float2(m, l);
                     }
                     named_bar_sync(2, 128);
-                    if (et == 0) {
-                        fence_acq_rel_cluster();
-                        const uint32_t sb = BAR(STATS + s % kStatSlots);
-                        for (uint32_t r = 0; r < csize; ++r) mbar_arrive_remote(mapa_shared(sb, r));
-                    }
+                    // one release arrival per CTA of the cluster, each from its own
+                    // thread: a release at cluster scope covers the rows the other
+                    // threads wrote before the named barrier, and the arrivals'
+                    // fences (each waits for this SM's memory traffic to settle)
+                    // overlap instead of running one after another
+                    if (et < (int)csize) mbar_arrive_remote(mapa_shared(BAR(STATS + s % kStatSlots), (uint32_t)et));
                 }
             }
             if (s >= lag) {
@@ -477,7 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 else p.partials[(int64_t)hg * p.total_vis + n0 + j] = a;
             }
         }
-        if (multi && !p.defer_fold) fold_tiles(p, b, n0, N, T, tile_begin, mt, et, kEpiThreads, 1, fold_flags);
+        if (multi && !p.defer_fold) fold_tiles<4>(p, b, n0, N, T, tile_begin, mt, et, kEpiThreads, 1, fold_flags);
         tc_fence_before();
     }
 
