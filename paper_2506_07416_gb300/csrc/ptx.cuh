@@ -190,6 +190,23 @@ __device__ __forceinline__ void cluster_sync_all()
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// The same barriers without release semantics on the arrival: for a barrier
+// that only has to order the peers' mbarrier initialisation (which
+// fence.mbarrier_init.release.cluster already releases) or keep every CTA of
+// the cluster resident until all are done, with no memory access of a peer to
+// order. A release arrival waits until the thread's earlier writes are visible
+// at cluster scope, which takes microseconds while the SM's copies are in
+// flight.
+__device__ __forceinline__ void cluster_arrive_relaxed()
+{
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_sync_relaxed()
+{
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;\n\tbarrier.cluster.wait.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank)
 {
     uint32_t r;

@@ -274,8 +274,10 @@ __global__ void __launch_bounds__(kResThreads, 1)
     // exist) and waits only before its first access to a peer's shared memory
     // (the epilogue, below) or before the final barrier (producer, MMA warp),
     // so the first copies and contractions do not wait for the slowest CTA of
-    // the cluster to get here.
-    cluster_arrive();
+    // the cluster to get here. The arrival needs no release: the barriers' set-up
+    // is released by fence.mbarrier_init above, and no other write of this CTA
+    // is read by a peer.
+    cluster_arrive_relaxed();
     const uint32_t tmem = *tmem_slot;
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
@@ -292,7 +294,7 @@ __global__ void __launch_bounds__(kResThreads, 1)
             tmem_dealloc(tmem, kResTmemCols);
         }
         cluster_wait();
-        cluster_sync_all();
+        cluster_sync_relaxed();
         return;
     }
     const int tile_begin = shp.tile_begin;
@@ -799,7 +801,11 @@ __global__ void __launch_bounds__(kResThreads, 1)
         tmem_dealloc(tmem, kResTmemCols);
     }
     if (p.extra) griddep_wait();  // returns at once for threads that already waited
-    cluster_sync_all();
+    // Every CTA stays resident until the cluster is done: the statistics a peer
+    // sends land (st.async) in this CTA's shared memory, and every one of them
+    // has completed on this CTA's barriers before its epilogue ends; no peer
+    // reads this CTA's memory, so the arrival needs no release.
+    cluster_sync_relaxed();
 #undef LVS_HQE
 }
 

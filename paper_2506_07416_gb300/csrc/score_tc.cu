@@ -202,8 +202,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Cluster barrier, split: every thread arrives now (its CTA's barriers
     // exist) and waits only before its first remote arrival (the epilogue) or
     // before the final barrier (producer, MMA warp), so the first copies and
-    // contractions do not wait for the slowest CTA of the cluster.
-    cluster_arrive();
+    // contractions do not wait for the slowest CTA of the cluster. The arrival
+    // needs no release: the barriers' set-up is released by fence.mbarrier_init
+    // above, and the statistics peers read are released by their own arrivals.
+    cluster_arrive_relaxed();
     const uint32_t tmem = *tmem_slot;
     const Ctl ctl{abort_flag, p.err, p.wait_budget};
 
