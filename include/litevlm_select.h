@@ -451,9 +451,8 @@ litevlm_status_t litevlm_select_set_wait_budget(litevlm_select_t handle, int64_t
 
 /*
  * Debug switches of a handle, for tests of the failure path (no counterpart in
- * the paper). LITEVLM_DEBUG_STALL_SCORE: in the score launches that use the
- * TMEM-resident kernel (litevlm_select_score_plan reports plan[0] of 2, 3 or 4),
- * the TMA producer first waits on an mbarrier that nothing completes, so that
+ * the paper). LITEVLM_DEBUG_STALL_SCORE: in the score launches (either score
+ * kernel), the TMA producer first waits on an mbarrier that nothing completes, so that
  * wait runs out of the wait budget before any copy or contraction is issued;
  * every other wait of the launch then gives up as well. The launch writes
  * invalid scores, and litevlm_select_check_device reports LITEVLM_ERR_TIMEOUT.

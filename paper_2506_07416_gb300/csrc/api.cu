@@ -585,7 +585,7 @@ litevlm_status_t score_impl(litevlm_select_t h, int32_t batch, const void* q_tex
     p.hkv = c.num_kv_heads;
     p.c_log2 = (float)((double)q_scale * (double)k_scale / sqrt((double)c.head_dim) * 1.4426950408889634);
     p.wait_budget = h->wait_budget;
-    p.stall = (h->debug_flags & LITEVLM_DEBUG_STALL_SCORE) != 0 && choice.resident;
+    p.stall = (h->debug_flags & LITEVLM_DEBUG_STALL_SCORE) != 0;
     p.slot_cols = ((qsplit ? (max_t + 1) / 2 : max_t) + 15) & ~15;
     p.qsplit = qsplit ? 2 : 1;
     p.query_last = (c.flags & LITEVLM_FLAG_QUERY_LAST_TOKEN) != 0;

@@ -80,7 +80,7 @@ struct SmemLayout {
     static constexpr int OFF_BAR = OFF_FLAGS + kMaxTilesPerCta * 4;
     // k_full[S], k_empty[S], q_full[QBUF], q_empty[QBUF], t1_full[2], t1_empty[2],
     // t2_full[2], t2_empty[2], stats[4], drain
-    static constexpr int NBAR = 2 * kStages + 2 * QBUF + 2 * 4 + kStatSlots + 1;
+    static constexpr int NBAR = 2 * kStages + 2 * QBUF + 2 * 4 + kStatSlots + 2;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
     static constexpr int BYTES = OFF_MISC + 16;
     static constexpr int ALLOC = BYTES + 1024;  // slack for 1024-byte alignment
@@ -159,7 +159,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // contractions of both passes, in issue order (unit u uses buffer u % 4)
     const int K_FULL = 0, K_EMPTY = kStages, Q_FULL = 2 * kStages, Q_EMPTY = Q_FULL + QBUF, U_FULL = Q_EMPTY + QBUF,
               U_EMPTY = U_FULL + 4, STATS = U_EMPTY + 4,
-              DRAIN = STATS + kStatSlots;
+              DRAIN = STATS + kStatSlots, STALL = DRAIN + 1;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
     volatile int* fold_flags = reinterpret_cast<volatile int*>(smem + L::OFF_FLAGS);
@@ -185,6 +185,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < kStatSlots; ++i) mbar_init(BAR(STATS + i), csize);
         mbar_init(BAR(DRAIN), 1);
+        mbar_init(BAR(STALL), 1);  // nothing ever arrives (the debug stall below)
         *abort_flag = 0;
         fence_mbar_init_cluster();
     }
@@ -218,7 +219,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             int q_issued[QBUF];
             for (int s = 0; s < QBUF; ++s) q_issued[s] = 0;
             for (int s = 0; s < kStages; ++s) k_issued[s] = 0;
-            bool ok = true;
+            // Debug stall (p.stall, a test of the failure path): wait on a barrier
+            // that nothing completes before issuing any copy, so this wait runs out
+            // of budget and every other wait of the launch runs out or sees the
+            // abort flag, with no copy or contraction in flight.
+            bool ok = !p.stall || wait_phase(BAR(STALL), 0, ctl);
             auto load_tiles = [&](int g) {
                 for (int t = tile_begin; t < tile_end && ok; ++t) {
                     if (!wait_phase(BAR(K_EMPTY + ks), kph ^ 1, ctl)) { ok = false; break; }

@@ -2,8 +2,8 @@
 without faulting, trapping or hanging the GPU.
 
 Every wait of the kernels (mbarrier phases, cluster arrivals) is bounded by the
-handle's wait budget. With LITEVLM_DEBUG_STALL_SCORE the TMA producer of the
-TMEM-resident score kernel first waits on an mbarrier that nothing completes,
+handle's wait budget. With LITEVLM_DEBUG_STALL_SCORE the TMA producer of either
+score kernel first waits on an mbarrier that nothing completes,
 before it issues any copy, so that wait runs out of budget; every other wait of
 the launch then gives up too, with no copy or contraction in flight. The test
 checks that the launch ends by itself, that check_device reports TIMEOUT, and
@@ -74,6 +74,39 @@ def test_wait_timeout_is_reported_and_the_handle_recovers(sel):
     g3 = _score(s, x, xd).cpu().numpy()
     s.check_device()
     assert np.array_equal(g.view(np.uint32), g3.view(np.uint32))
+    fresh.close()
+    s.close()
+
+
+def test_wait_timeout_in_the_reread_kernel(sel):
+    """The same failure path in the kernel that streams K twice per head: its
+    producer stalls the same way, the launch gives up within the budget, and the
+    handle is exact again afterwards (the heads are split over CTA groups, so
+    the fold tickets are in use here too)."""
+    w = inputs.workload("single")
+    x = inputs.make_numpy(w)
+    xd = to_device(x, w)
+    s = sel.Selector(w.batch, w.total_vis, w.total_txt, w.hq, w.hkv, w.head_dim, w.dtype, score_kernel="reread")
+    plan = s.score_plan(x["text_offsets"], x["seq_offsets"])
+    assert plan[0] == 1 and plan[3] > 1, plan  # re-read kernel, heads split over CTA groups
+
+    s.set_wait_budget(20000)
+    s.set_debug_flags(sel.DEBUG_STALL_SCORE)
+    _score(s, x, xd)
+    with pytest.raises(sel.LitevlmError) as ei:
+        s.check_device()
+    assert ei.value.name == "TIMEOUT"
+
+    s.set_debug_flags(0)
+    s.set_wait_budget(0)
+    g = _score(s, x, xd).cpu().numpy()
+    s.check_device()
+    o = oracle.score(x["q"], x["k"], x["seq_offsets"], x["text_offsets"], w.hq, w.hkv, w.head_dim, w.dtype)
+    assert_scores_close(g, o, w.dtype)
+    fresh = sel.Selector(w.batch, w.total_vis, w.total_txt, w.hq, w.hkv, w.head_dim, w.dtype, score_kernel="reread")
+    g2 = _score(fresh, x, xd).cpu().numpy()
+    fresh.check_device()
+    assert np.array_equal(g.view(np.uint32), g2.view(np.uint32))
     fresh.close()
     s.close()
 
