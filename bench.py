@@ -47,6 +47,9 @@ SUB_STEPS = {"single": (500, 20), "highres": (300, 10), "fp8_ragged": (60, 5), "
 KERNEL_SOURCES = ["paper_2506_07416_gb300/csrc/score_tc.cu", "paper_2506_07416_gb300/csrc/score_res.cu",
                   "paper_2506_07416_gb300/csrc/pipe.cuh", "paper_2506_07416_gb300/csrc/ptx.cuh",
                   "paper_2506_07416_gb300/csrc/score.h"]
+# the files each score kernel is compiled from: its own source and the shared headers
+KERNEL_FILES = {"score_tc": [KERNEL_SOURCES[0]] + KERNEL_SOURCES[2:],
+                "score_res": KERNEL_SOURCES[1:]}
 WORKLOADS = ["sweep", "single", "highres", "fp8_ragged"]
 
 
@@ -160,22 +163,29 @@ def peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
 
 
-def kernel_source_sha():
+def kernel_source_sha(kernel=None):
+    """First 16 hex digits of the sha256 of the score kernels' sources: all of
+    them (kernel=None), or the files one kernel is compiled from ("score_tc",
+    "score_res")."""
     h = hashlib.sha256()
-    for f in KERNEL_SOURCES:
+    for f in (KERNEL_FILES[kernel] if kernel else KERNEL_SOURCES):
         h.update(open(os.path.join(ROOT, f), "rb").read())
     return h.hexdigest()[:16]
 
 
 def committed_traffic(workload):
     """DRAM bytes per score launch from the committed ncu summary, if it was
-    taken on the current kernel source; else None."""
+    taken on the current sources of the kernel that serves the workload; else
+    None."""
     p = os.path.join(ROOT, "profiles", "score_traffic.json")
     if not os.path.exists(p):
         return None
     d = json.load(open(p))
     ent = d.get(workload)
-    if not ent or ent.get("source_sha") != kernel_source_sha():
+    if not ent:
+        return None
+    kernel = "score_res" if ent.get("kernel", "").startswith("score_res") else "score_tc"
+    if ent.get("kernel_sha") != kernel_source_sha(kernel):
         return None
     return ent.get("dram_bytes_per_launch")
 
