@@ -74,3 +74,30 @@ def test_batch_option_takes_the_first_requests():
     w = bench.workload_for(A())
     full = inputs.workload("fp8_ragged")
     assert w.batch == 5 and list(w.n_vis) == list(full.n_vis[:5]) and list(w.n_txt) == list(full.n_txt[:5])
+
+
+def test_committed_traffic_follows_the_workloads_own_kernel(tmp_path, monkeypatch):
+    """A DRAM figure is reported only while the files of the kernel that serves
+    the workload still hash to the recorded kernel_sha; a change to the other
+    kernel's source leaves it valid."""
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    csrc = tmp_path / "paper_2506_07416_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    for f in bench.KERNEL_SOURCES:
+        (tmp_path / f).write_text("source of " + os.path.basename(f))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    res, tc = bench.kernel_source_sha("score_res"), bench.kernel_source_sha("score_tc")
+    assert res != tc
+    import json
+    (prof / "score_traffic.json").write_text(json.dumps({
+        "sweep": {"kernel": "score_res_kernel<256, 0, 64, 1, 0>", "kernel_sha": res, "dram_bytes_per_launch": 7},
+        "highres": {"kernel": "score_tc_kernel<256, 0, 128>", "kernel_sha": tc, "dram_bytes_per_launch": 9}}))
+    assert bench.committed_traffic("sweep") == 7 and bench.committed_traffic("highres") == 9
+    assert bench.committed_traffic("single") is None  # no entry
+    # the re-read kernel's source changes: its figure goes stale, the resident kernel's stays
+    (tmp_path / bench.KERNEL_SOURCES[0]).write_text("changed score_tc.cu")
+    assert bench.committed_traffic("highres") is None and bench.committed_traffic("sweep") == 7
+    # a shared header changes: both go stale
+    (tmp_path / bench.KERNEL_SOURCES[2]).write_text("changed pipe.cuh")
+    assert bench.committed_traffic("sweep") is None
